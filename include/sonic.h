@@ -1,0 +1,255 @@
+/*
+ * sonic.h -- C ABI of libsonic, the GB300 (sm_103a) attention path over a
+ * Nexus-compressed KV cache (SONIC, arXiv 2601.21927).
+ *
+ * Three operations, in the order a dialogue goes through them:
+ *
+ *   sonic_compact_kv    keep only the system-prompt, Nexus and current-turn
+ *                       K/V rows of every sequence and layer (the retention
+ *                       rule: Sec. 1, the Fig. 2 caption, Sec. 3.2 "Historical
+ *                       Body Removal", App. C effective context I_sys + N + Q_n).
+ *   sonic_attn_prefill  softmax attention of a sequence's query rows under the
+ *                       hierarchical visibility mask of Sec. 3.2 (Eq. 3 causal
+ *                       rule, Eq. 4 body removal, Eq. 5 bidirectional Nexus).
+ *   sonic_attn_decode   one generation step with grouped-query heads over the
+ *                       retained cache (App. C, Eq. 15: generation conditions
+ *                       on I_sys, the Nexus state and the current query only).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Every tensor and metadata pointer is a DEVICE pointer owned by the
+ *    caller.  The library never allocates, frees or synchronises; each call
+ *    enqueues kernels on `stream` (a cudaStream_t; NULL is the legacy default
+ *    stream) and returns.  Scratch memory comes from the caller's
+ *    `workspace` (query its size first).
+ *  - Host-detectable errors (NULL where a pointer is required, bad sizes,
+ *    unsupported head_dim or head ratio, workspace too small, misaligned
+ *    pointers) return a status before anything is launched.  Conditions only
+ *    the GPU can see (output capacity exceeded, an inconsistent layout, a
+ *    bounded wait that ran out) are written to the optional device word
+ *    `*status` (first error wins; the caller zeroes it) and the affected
+ *    blocks stop early; nothing traps.  sonic_read_status() fetches it.
+ *  - Roles are per-token uint8 values (sonic_role_t); segment numbers are
+ *    int32 (0 = system prompt, i = history segment m_i, h+1 = current turn,
+ *    non-decreasing along a sequence).  Positions p, q of the mask are row
+ *    numbers within one sequence, in S_aug order (Eq. 1).
+ *  - Token rows of K and V hold all KV heads: element (row t, head j, dim d)
+ *    sits at t * n_heads_kv * head_dim + j * head_dim + d.  Query rows hold
+ *    all query heads the same way.  Query head h reads KV head
+ *    h / (n_heads_q / n_heads_kv).
+ *  - Attention tensors are bf16 (stored as uint16 bit patterns), accumulate
+ *    in fp32 and write bf16 outputs rounded to nearest even.
+ *  - Calls are stateless and may be issued from several host threads.
+ */
+#ifndef SONIC_H
+#define SONIC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SONIC_ABI_VERSION 1
+
+#if defined(__GNUC__)
+#define SONIC_API __attribute__((visibility("default")))
+#else
+#define SONIC_API
+#endif
+
+/* cudaStream_t without including the CUDA headers. */
+typedef struct CUstream_st *sonic_stream_t;
+
+/* Per-token role in the augmented sequence S_aug (Sec. 3.1, Eq. 1). */
+typedef enum {
+    SONIC_ROLE_SYS = 0,   /* system prompt I_sys                     */
+    SONIC_ROLE_BODY = 1,  /* text of a history segment, B_i          */
+    SONIC_ROLE_NEXUS = 2, /* Nexus token of a history segment, N_i   */
+    SONIC_ROLE_CURR = 3   /* current query / current turn, Q_curr    */
+} sonic_role_t;
+
+typedef enum {
+    SONIC_OK = 0,
+    SONIC_ERR_INVALID_ARGUMENT = 1,
+    SONIC_ERR_UNSUPPORTED = 2,
+    SONIC_ERR_WORKSPACE = 3,
+    SONIC_ERR_CAPACITY = 4,
+    SONIC_ERR_DEVICE_TIMEOUT = 5,
+    SONIC_ERR_CUDA = 6,
+    SONIC_ERR_LAYOUT = 7
+} sonic_status_t;
+
+/* Which Nexus tokens a Nexus token sees (Eq. 5 and its reading).
+ * FULL: every Nexus token of every segment (Eq. 5 as printed).
+ * CAUSAL_SEGMENTS: Nexus tokens of its own and earlier segments only (the
+ * reading under which Nexus state is kept across a session, Sec. 6.4).
+ * Rows that are not Nexus tokens see the same keys under both. */
+typedef enum {
+    SONIC_NEXUS_FULL = 0,
+    SONIC_NEXUS_CAUSAL_SEGMENTS = 1
+} sonic_nexus_vis_t;
+
+/* ------------------------------------------------------------------------- */
+/* Compaction                                                                */
+/* ------------------------------------------------------------------------- */
+
+typedef struct {
+    int32_t batch;               /* B >= 0 sequences                                    */
+    int32_t n_layers;            /* >= 1; K/V of every layer are compacted in one call  */
+    const int32_t *k_start;      /* device [B]: first packed row of sequence b           */
+    const int32_t *k_len;        /* device [B]: rows of sequence b (raw S_aug length)    */
+    const int32_t *reserve;      /* device [B] or NULL: free rows left after sequence
+                                    b's retained rows (room to append new tokens)       */
+    int64_t row_bytes;           /* bytes of one token row (all KV heads); multiple of 16 */
+    int64_t in_layer_bytes;      /* byte stride between layers of K and V; multiple of 16 */
+    int64_t out_layer_bytes;     /* byte stride between layers of out_K and out_V       */
+    int32_t out_capacity_rows;   /* rows available per layer in out_K / out_V           */
+    int32_t *ret_len;            /* device [B] or NULL: retained rows of sequence b      */
+    int32_t *src_idx;            /* device [out_capacity_rows] or NULL: packed source row
+                                    of each output row, -1 in reserve rows              */
+    uint8_t *out_role;           /* device [out_capacity_rows] or NULL: role of each
+                                    output row (SONIC_ROLE_BODY in reserve rows)        */
+    int32_t *out_seg;            /* device [out_capacity_rows] or NULL: segment of each
+                                    output row (-1 in reserve rows)                     */
+    int32_t *status;             /* device int32 or NULL                                */
+    void *workspace;             /* device, sonic_compact_workspace_size() bytes        */
+    size_t workspace_bytes;
+} sonic_compact_args;
+
+/*
+ * Retention rule (Sec. 3.2 body removal; App. C effective context): row t of
+ * sequence b is kept iff role[t] != SONIC_ROLE_BODY.  Kept rows keep their
+ * order.  Writes
+ *   offsets[b] = sum_{b' < b} (ret_len[b'] + reserve[b'])  (device [B+1],
+ *                offsets[B] = total output rows),
+ * and for every layer l and kept row j of sequence b copies the row_bytes of
+ * K (resp. V) row k_start[b] + (j-th kept position) of layer l to row
+ * offsets[b] + j of layer l of out_K (resp. out_V), bit for bit.  Reserve
+ * rows are not written.  seg_id may be NULL; when given it is checked
+ * (non-decreasing within a sequence, no body row in segment 0) and a
+ * violation sets SONIC_ERR_LAYOUT.  If offsets[B] > out_capacity_rows the
+ * call sets SONIC_ERR_CAPACITY and copies only rows below the capacity.
+ * K/V/out pointers must be 16-byte aligned.
+ */
+SONIC_API sonic_status_t sonic_compact_kv(const void *K, const void *V, const int32_t *seg_id,
+                                const uint8_t *role, void *out_K, void *out_V,
+                                int32_t *offsets, const sonic_compact_args *args,
+                                sonic_stream_t stream);
+
+/* Workspace bytes sonic_compact_kv needs for these args (0 if none). */
+SONIC_API size_t sonic_compact_workspace_size(const sonic_compact_args *args);
+
+/* ------------------------------------------------------------------------- */
+/* Masked prefill                                                            */
+/* ------------------------------------------------------------------------- */
+
+typedef struct {
+    int32_t batch;               /* B >= 0                                              */
+    int32_t n_layers;            /* >= 1                                                */
+    int32_t n_heads_q;           /* Hq, a multiple of n_heads_kv                        */
+    int32_t n_heads_kv;          /* Hkv >= 1                                            */
+    int32_t head_dim;            /* D: 64 or 128                                        */
+    const int32_t *k_start;      /* device [B]: first key row of sequence b in K, V,
+                                    role, seg_id                                        */
+    const int32_t *k_len;        /* device [B]: key rows of sequence b                   */
+    const int32_t *q_start;      /* device [B]: first query row of sequence b in Q, O    */
+    const int32_t *q_len;        /* device [B]: query rows of sequence b, <= k_len[b];
+                                    query i is key position k_len[b] - q_len[b] + i
+                                    (the last q_len rows: bottom-right aligned)         */
+    int32_t max_q_len;           /* host: >= every q_len[b]; sizes the launch grid      */
+    int32_t max_k_len;           /* host: >= every k_len[b], at most 262144             */
+    int32_t total_q_rows;        /* rows per layer of Q and O                           */
+    int32_t total_k_rows;        /* rows per layer of K and V (and of role, seg_id)     */
+    int64_t q_layer_stride;      /* elements between layers of Q                        */
+    int64_t kv_layer_stride;     /* elements between layers of K and V                  */
+    int64_t o_layer_stride;      /* elements between layers of O                        */
+    float softmax_scale;         /* 0 selects 1/sqrt(head_dim)                          */
+    int32_t nexus_vis;           /* sonic_nexus_vis_t                                   */
+    float *lse;                  /* device [n_layers][total_q_rows][Hq] or NULL: natural
+                                    log-sum-exp of each row's scaled visible scores     */
+    int32_t *status;             /* device int32 or NULL                                */
+    void *workspace;             /* device, sonic_prefill_workspace_size() bytes        */
+    size_t workspace_bytes;
+} sonic_prefill_args;
+
+/*
+ * Sec. 3.2 masked attention.  For every layer, sequence b, query row i and
+ * query head h, with p = k_len[b] - q_len[b] + i:
+ *   s_q   = scale * <Q[p, h], K[q, h/G]>  for the key rows q of sequence b,
+ *   vis   = the Sec. 3.2 rule on (role, seg_id) of rows p and q:
+ *             key q a body row:           same segment and q <= p   (Eqs. 3, 4)
+ *             both Nexus rows:            true (FULL) or seg[q] <= seg[p]   (Eq. 5)
+ *             otherwise:                  q <= p                    (Eq. 3)
+ *   O[i, h] = sum_{q in vis} softmax(s)_q V[q, h/G]   (zeros if nothing is visible).
+ * Whole 128x128 key tiles the mask hides are skipped; the rule is applied per
+ * element only on tiles it cuts.  Q, K, V, O are bf16; every row stride and
+ * base pointer must be 16-byte aligned.  role and seg_id are indexed like the
+ * key rows of one layer (shared by all layers).
+ */
+SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
+                                  const int32_t *seg_id, const uint8_t *role, uint16_t *O,
+                                  const sonic_prefill_args *args, sonic_stream_t stream);
+
+SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
+
+/* ------------------------------------------------------------------------- */
+/* Decode                                                                    */
+/* ------------------------------------------------------------------------- */
+
+typedef struct {
+    int32_t batch;               /* B >= 0                                              */
+    int32_t n_layers;            /* >= 1; all layers run in one launch                  */
+    int32_t n_heads_q;           /* Hq, a multiple of n_heads_kv, Hq / Hkv <= 16        */
+    int32_t n_heads_kv;          /* Hkv >= 1                                            */
+    int32_t head_dim;            /* D: 64 or 128                                        */
+    const int32_t *kv_start;     /* device [B]: first retained row of sequence b         */
+    int32_t max_len;             /* host: >= every lens[b]; sizes the split grid        */
+    int32_t total_kv_rows;       /* rows per layer of K_ret and V_ret                   */
+    int64_t q_layer_stride;      /* elements between layers of q                        */
+    int64_t kv_layer_stride;     /* elements between layers of K_ret and V_ret          */
+    int64_t o_layer_stride;      /* elements between layers of O                        */
+    float softmax_scale;         /* 0 selects 1/sqrt(head_dim)                          */
+    int32_t chunk_len;           /* keys per split, multiple of 64; 0 = automatic       */
+    float *lse;                  /* device [n_layers][B][Hq] or NULL                    */
+    int32_t *status;             /* device int32 or NULL                                */
+    void *workspace;             /* device, sonic_decode_workspace_size() bytes         */
+    size_t workspace_bytes;
+} sonic_decode_args;
+
+/*
+ * One decode step (App. C).  q and O are [n_layers][B][Hq][D] (layer strides
+ * given); for sequence b the retained rows kv_start[b] .. kv_start[b] +
+ * lens[b] - 1 of K_ret / V_ret (the new token's own row included) are all
+ * visible:  O[l, b, h] = sum_t softmax_t(scale <q[l,b,h], K[t, h/G]>) V[t, h/G].
+ * The keys are split into chunks of chunk_len; each (layer, sequence, KV
+ * head, chunk) block produces a partial (max, sum, accumulator) in the
+ * workspace, and a second kernel merges them by log-sum-exp.  lens[b] = 0
+ * gives zeros (and lse = -inf).  bf16 in/out, fp32 arithmetic.
+ */
+SONIC_API sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
+                                 const uint16_t *V_ret, const int32_t *lens, uint16_t *O,
+                                 const sonic_decode_args *args, sonic_stream_t stream);
+
+SONIC_API size_t sonic_decode_workspace_size(const sonic_decode_args *args);
+
+/* ------------------------------------------------------------------------- */
+/* Status                                                                    */
+/* ------------------------------------------------------------------------- */
+
+/* Waits for `stream`, then copies the device status word to the host and
+ * returns it (SONIC_ERR_CUDA if the copy itself fails). */
+SONIC_API sonic_status_t sonic_read_status(const int32_t *status, sonic_stream_t stream);
+
+/* Static, human-readable name of a status code. */
+SONIC_API const char *sonic_status_string(sonic_status_t status);
+
+/* SONIC_ABI_VERSION of the loaded library. */
+SONIC_API int32_t sonic_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SONIC_H */

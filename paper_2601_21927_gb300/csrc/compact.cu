@@ -1,0 +1,270 @@
+// KV compaction: keep the system-prompt, Nexus and current-turn rows of every
+// sequence and layer, drop the history bodies.
+//
+// Retention rule (SONIC Sec. 3.2 "Historical Body Removal" and App. C: the
+// effective context is I_sys + Nexus state + current query): a row is kept
+// iff its role is not BODY; kept rows keep their order.
+//
+// Three launches, none of which needs a host round trip:
+//   keep_count    one block per sequence: number of kept rows (and a layout
+//                 check when segment numbers are given);
+//   keep_scatter  one block per sequence: its output offset (sum over
+//                 earlier sequences), then a block-wide prefix scan of the
+//                 keep flags built from warp-shuffle scans, writing the
+//                 source row of every output row (-1 in reserve rows);
+//   kv_gather     all layers, K and V: 16-byte vector copy of every kept row
+//                 to its output row, grid-stride over rows of each layer.
+#include "sonic_dev.cuh"
+#include "sonic_host.h"
+
+namespace sonic {
+namespace {
+
+constexpr int kScanThreads = 512;
+
+__global__ void __launch_bounds__(kScanThreads)
+keep_count_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
+                  const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
+                  int32_t *__restrict__ counts, int32_t *status) {
+    const int b = blockIdx.x;
+    const int32_t start = k_start[b], len = k_len[b];
+    int n = 0;
+    bool bad = false;
+    for (int32_t t = threadIdx.x; t < len; t += blockDim.x) {
+        uint8_t r = role[start + t];
+        n += (r != SONIC_ROLE_BODY);
+        bad |= (r > SONIC_ROLE_CURR);
+        if (seg != nullptr) {
+            int32_t s = seg[start + t];
+            bad |= (r == SONIC_ROLE_BODY && s <= 0);
+            if (t > 0) bad |= (s < seg[start + t - 1]);
+        }
+    }
+    // block reduction
+    __shared__ int red[kScanThreads / 32];
+    __shared__ int bad_any;
+    if (threadIdx.x == 0) bad_any = 0;
+    __syncthreads();
+    for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n;
+    if (bad) bad_any = 1;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int s = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
+        counts[b] = s;
+        if (bad_any) set_status(status, SONIC_ERR_LAYOUT);
+    }
+}
+
+// Inclusive warp scan of v (warp-shuffle).
+__device__ __forceinline__ int warp_inclusive_scan(int v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+    }
+    return v;
+}
+
+__global__ void __launch_bounds__(kScanThreads)
+keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
+                    const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
+                    const int32_t *__restrict__ reserve, const int32_t *__restrict__ counts,
+                    int32_t B, int32_t capacity, int32_t *__restrict__ offsets,
+                    int32_t *__restrict__ ret_len, int32_t *__restrict__ src_idx,
+                    uint8_t *__restrict__ out_role, int32_t *__restrict__ out_seg,
+                    int32_t *status) {
+    const int b = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int kWarps = kScanThreads / 32;
+    __shared__ int warp_tot[kWarps];
+    __shared__ long long base_sh;
+
+    // Output offset of this sequence: sum of (count + reserve) over b' < b.
+    long long part = 0;
+    for (int i = tid; i < b; i += blockDim.x)
+        part += (long long)counts[i] + (reserve ? reserve[i] : 0);
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    __shared__ long long red[kWarps];
+    if (lane == 0) red[warp] = part;
+    __syncthreads();
+    if (tid == 0) {
+        long long s = 0;
+        for (int w = 0; w < kWarps; ++w) s += red[w];
+        base_sh = s;
+    }
+    __syncthreads();
+    const long long base = base_sh;
+    const int32_t count = counts[b];
+    const int32_t res = reserve ? reserve[b] : 0;
+    const long long end = base + count + res;
+    if (tid == 0) {
+        offsets[b] = (int32_t)base;
+        if (b == B - 1) offsets[B] = (int32_t)end;
+        if (ret_len) ret_len[b] = count;
+        if (end > capacity || end > 0x7fffffffLL) set_status(status, SONIC_ERR_CAPACITY);
+    }
+    if (src_idx == nullptr && out_role == nullptr && out_seg == nullptr) return;
+
+    // Block-wide exclusive scan of the keep flags, chunk by chunk.
+    const int32_t start = k_start[b], len = k_len[b];
+    long long running = base;
+    for (int32_t c0 = 0; c0 < len; c0 += blockDim.x) {
+        const int32_t t = c0 + tid;
+        const int keep = (t < len) && (role[start + t] != SONIC_ROLE_BODY);
+        int incl = warp_inclusive_scan(keep);
+        if (lane == 31) warp_tot[warp] = incl;
+        __syncthreads();
+        int warp_base = 0, chunk_tot = 0;
+        for (int w = 0; w < kWarps; ++w) {
+            int v = warp_tot[w];
+            if (w < warp) warp_base += v;
+            chunk_tot += v;
+        }
+        const long long o = running + warp_base + incl - keep;
+        if (keep && o < capacity) {
+            if (src_idx) src_idx[o] = start + t;
+            if (out_role) out_role[o] = role[start + t];
+            if (out_seg) out_seg[o] = seg ? seg[start + t] : 0;
+        }
+        running += chunk_tot;
+        __syncthreads();
+    }
+    // Reserve rows: no source.
+    for (int32_t r = tid; r < res; r += blockDim.x) {
+        const long long o = base + count + r;
+        if (o < capacity) {
+            if (src_idx) src_idx[o] = -1;
+            if (out_role) out_role[o] = SONIC_ROLE_BODY;
+            if (out_seg) out_seg[o] = -1;
+        }
+    }
+}
+
+// 16-byte vector copy of kept rows.  blockIdx.y = layer * 2 + (0: K, 1: V).
+// One warp copies whole rows (lane j takes 16-byte chunks j, j+32, ...); each
+// warp works on two rows at a time with all their loads issued before the
+// stores, so up to 8 x 16 bytes per thread are in flight.
+constexpr int kGatherThreads = 256;
+constexpr int kGatherUnroll = 4;
+
+__device__ __forceinline__ int4 ld_stream(const void *p) {
+    int4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+__global__ void __launch_bounds__(kGatherThreads)
+kv_gather_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
+                 uint8_t *__restrict__ out_K, uint8_t *__restrict__ out_V,
+                 const int32_t *__restrict__ offsets, const int32_t *__restrict__ src_idx,
+                 int32_t B, int32_t capacity, int64_t row_bytes, int64_t in_layer_bytes,
+                 int64_t out_layer_bytes) {
+    const int layer = blockIdx.y >> 1;
+    const bool is_v = blockIdx.y & 1;
+    const uint8_t *src = (is_v ? V : K) + (int64_t)layer * in_layer_bytes;
+    uint8_t *dst = (is_v ? out_V : out_K) + (int64_t)layer * out_layer_bytes;
+    int64_t n_rows = offsets[B];
+    if (n_rows > capacity) n_rows = capacity;
+    const int lane = threadIdx.x & 31;
+    const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int cpr = (int)(row_bytes >> 4);  // 16-byte chunks per row
+    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5); r0 < n_rows;
+         r0 += 2 * n_warps) {
+        const int64_t r1 = r0 + n_warps;
+        const int32_t s0 = src_idx[r0];
+        const int32_t s1 = r1 < n_rows ? src_idx[r1] : -1;
+        const uint8_t *p0 = src + (int64_t)s0 * row_bytes;
+        const uint8_t *p1 = src + (int64_t)s1 * row_bytes;
+        uint8_t *q0 = dst + r0 * row_bytes;
+        uint8_t *q1 = dst + r1 * row_bytes;
+        for (int c0 = lane; c0 < cpr; c0 += 32 * kGatherUnroll) {
+            int4 v0[kGatherUnroll], v1[kGatherUnroll];
+#pragma unroll
+            for (int u = 0; u < kGatherUnroll; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < cpr) {
+                    if (s0 >= 0) v0[u] = ld_stream(p0 + ((int64_t)c << 4));
+                    if (s1 >= 0) v1[u] = ld_stream(p1 + ((int64_t)c << 4));
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kGatherUnroll; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < cpr) {
+                    if (s0 >= 0) *reinterpret_cast<int4 *>(q0 + ((int64_t)c << 4)) = v0[u];
+                    if (s1 >= 0) *reinterpret_cast<int4 *>(q1 + ((int64_t)c << 4)) = v1[u];
+                }
+            }
+        }
+    }
+}
+
+}  // namespace
+}  // namespace sonic
+
+using namespace sonic;
+
+extern "C" size_t sonic_compact_workspace_size(const sonic_compact_args *a) {
+    if (a == nullptr || a->batch < 0) return 0;
+    size_t ws = round_up((size_t)a->batch * sizeof(int32_t), 256);
+    if (a->src_idx == nullptr)
+        ws += round_up((size_t)(a->out_capacity_rows > 0 ? a->out_capacity_rows : 0) *
+                           sizeof(int32_t),
+                       256);
+    return ws;
+}
+
+extern "C" sonic_status_t sonic_compact_kv(const void *K, const void *V, const int32_t *seg_id,
+                                           const uint8_t *role, void *out_K, void *out_V,
+                                           int32_t *offsets, const sonic_compact_args *a,
+                                           sonic_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (a == nullptr || offsets == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch < 0 || a->n_layers < 1 || a->out_capacity_rows < 0)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch == 0) {
+        if (cudaMemsetAsync(offsets, 0, sizeof(int32_t), stream) != cudaSuccess)
+            return SONIC_ERR_CUDA;
+        return SONIC_OK;
+    }
+    if (K == nullptr || V == nullptr || role == nullptr || out_K == nullptr ||
+        out_V == nullptr || a->k_start == nullptr || a->k_len == nullptr)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->row_bytes <= 0 || (a->row_bytes & 15) || (a->in_layer_bytes & 15) ||
+        (a->out_layer_bytes & 15))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->n_layers > 1 && (a->in_layer_bytes <= 0 || a->out_layer_bytes <= 0))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (!aligned16(K) || !aligned16(V) || !aligned16(out_K) || !aligned16(out_V))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->n_layers > 32767) return SONIC_ERR_UNSUPPORTED;
+    const size_t need = sonic_compact_workspace_size(a);
+    if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
+        return SONIC_ERR_WORKSPACE;
+
+    int32_t *counts = static_cast<int32_t *>(a->workspace);
+    int32_t *src_idx = a->src_idx;
+    if (src_idx == nullptr)
+        src_idx = reinterpret_cast<int32_t *>(static_cast<char *>(a->workspace) +
+                                              round_up((size_t)a->batch * 4, 256));
+
+    keep_count_kernel<<<a->batch, kScanThreads, 0, stream>>>(role, seg_id, a->k_start, a->k_len,
+                                                            counts, a->status);
+    keep_scatter_kernel<<<a->batch, kScanThreads, 0, stream>>>(
+        role, seg_id, a->k_start, a->k_len, a->reserve, counts, a->batch, a->out_capacity_rows,
+        offsets, a->ret_len, src_idx, a->out_role, a->out_seg, a->status);
+    const int sms = device_sm_count();
+    // Enough blocks per (layer, K|V) to keep every SM busy with ~8 blocks.
+    const int per_slice = (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers);
+    dim3 grid(per_slice < 1 ? 1 : per_slice, 2 * a->n_layers);
+    kv_gather_kernel<<<grid, kGatherThreads, 0, stream>>>(
+        static_cast<const uint8_t *>(K), static_cast<const uint8_t *>(V),
+        static_cast<uint8_t *>(out_K), static_cast<uint8_t *>(out_V), offsets, src_idx, a->batch,
+        a->out_capacity_rows, a->row_bytes, a->in_layer_bytes, a->out_layer_bytes);
+    return cudaGetLastError() == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
+}

@@ -1,0 +1,522 @@
+// GQA decode over the retained (compacted) KV cache.
+//
+// One generation step (SONIC App. C: generation conditions on I_sys, the
+// Nexus state and the current query, i.e. on exactly the rows compaction
+// kept).  Every retained row of a sequence is visible to its new token.
+//
+// Split-K, HBM-bound design:
+//   decode_split   one block per (key chunk, KV head, sequence, layer).  A
+//                  producer warp streams the chunk's K and V through a ring
+//                  of 64-key shared-memory stages with TMA (128-byte swizzle,
+//                  so both access patterns below are bank-conflict free).
+//                  Four consumer warps take turns on the tiles; each keeps
+//                  its own online softmax for the G query heads that share
+//                  the KV head:
+//                    scores  lane = key (2 keys per lane), full-D dot products
+//                            against q in shared memory (broadcast reads),
+//                            packed fp32x2 FMAs, no cross-lane reduction;
+//                    P . V   lane = 4 (D=128) or 2 (D=64) output dims, keys
+//                            walked in order, p broadcast from shared memory.
+//                  The four warps are merged by log-sum-exp at the end; a
+//                  single-chunk sequence writes O directly, otherwise the
+//                  partial (max, sum, unnormalised accumulator) goes to the
+//                  workspace.
+//   decode_combine log-sum-exp merge of the chunks of each (layer, seq, head).
+// K and V are read exactly once from HBM; softmax runs in base 2 with the
+// scale folded into q.
+#include "sonic_dev.cuh"
+#include "sonic_host.h"
+
+namespace sonic {
+namespace {
+
+constexpr int kTileKeys = 64;
+constexpr int kConsumerWarps = 4;
+constexpr int kDecThreads = (kConsumerWarps + 1) * 32;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kLog2e = 1.4426950408889634f;
+
+template <int D>
+struct DecCfg {
+    static constexpr int kHalves = D / 64;               // 128-byte swizzle rows per key
+    static constexpr int kTileBytes = kTileKeys * D * 2;  // K (or V) tile
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kStages = (D == 128) ? 6 : 12;
+    static constexpr int kChunks = D / 8;  // 16-byte pieces of one key row
+    static constexpr int kDpl = D / 32;    // P.V output dims per lane
+};
+
+struct DecParams {
+    const uint16_t *q;
+    uint16_t *O;
+    const int32_t *lens;
+    const int32_t *kv_start;
+    float *lse;
+    float *part_acc;  // [units][max_chunks][D]
+    float *part_ml;   // [units][max_chunks][2]
+    int32_t *status;
+    int B, Hq, Hkv, G;
+    int64_t q_ls, o_ls;
+    int chunk_len, max_chunks;
+    float scale_log2;
+};
+
+template <int D, int GT>
+constexpr size_t dec_smem_bytes() {
+    using C = DecCfg<D>;
+    constexpr int Gp = (GT + 3) & ~3;
+    return 1024 + (size_t)C::kStages * C::kStageBytes + (size_t)GT * D * 4 +
+           (size_t)kConsumerWarps * kTileKeys * Gp * 4 + 2 * C::kStages * 8 + 16;
+}
+
+__device__ __forceinline__ uint4 lds128(const uint8_t *p) {
+    return *reinterpret_cast<const uint4 *>(p);
+}
+
+__device__ __forceinline__ float2 w2f(uint32_t w) { return make_float2(bf16lo(w), bf16hi(w)); }
+
+template <int D, int GT>
+__global__ void __launch_bounds__(kDecThreads, 1)
+decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, const DecParams p) {
+    using C = DecCfg<D>;
+    constexpr int Gp = (GT + 3) & ~3;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    float *q_s = reinterpret_cast<float *>(smem + C::kStages * C::kStageBytes);
+    float *p_s = q_s + GT * D;
+    uint64_t *full = reinterpret_cast<uint64_t *>(p_s + kConsumerWarps * kTileKeys * Gp);
+    uint64_t *empty = full + C::kStages;
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + C::kStages);
+
+    const int chunk = blockIdx.x, kvh = blockIdx.y;
+    const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
+    int len = p.lens[b];
+    if (len > p.max_chunks * p.chunk_len) {
+        // longer than the host-side bound: attend to the first max_len keys only
+        if (threadIdx.x == 0 && chunk == 0 && kvh == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        len = p.max_chunks * p.chunk_len;
+    }
+    const int key0 = chunk * p.chunk_len;
+    if (key0 >= len || timed_out(p.status)) return;
+    const int nkeys = min(p.chunk_len, len - key0);
+    const int ntiles = (nkeys + kTileKeys - 1) / kTileKeys;
+    const int G = p.G;
+    const int row0 = p.kv_start[b] + key0;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    if (tid == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    // q of the G heads sharing this KV head, pre-scaled into the base-2 domain.
+    const uint16_t *qp = p.q + layer * p.q_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G) * D;
+    for (int i = tid; i < GT * D; i += blockDim.x) {
+        const int g = i / D;
+        float v = 0.f;
+        if (g < G) v = __uint_as_float((uint32_t)qp[i] << 16) * p.scale_log2;
+        q_s[i] = v;
+    }
+    __syncthreads();
+
+    if (warp == kConsumerWarps) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tmK);
+            tma_prefetch_desc(&tmV);
+            int t = 0;
+            for (; t < ntiles; ++t) {
+                const int s = t % C::kStages;
+                if (t >= C::kStages &&
+                    !mbar_wait(&empty[s], ((t / C::kStages) - 1) & 1, p.status, abort_flag))
+                    break;
+                mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+                uint8_t *kd = smem + s * C::kStageBytes;
+                uint8_t *vd = kd + C::kTileBytes;
+                const int r = row0 + t * kTileKeys;
+#pragma unroll
+                for (int h = 0; h < C::kHalves; ++h) {
+                    tma_load_4d(kd + h * kTileKeys * 128, &tmK, &full[s], h * 64, kvh, r, layer);
+                    tma_load_4d(vd + h * kTileKeys * 128, &tmV, &full[s], h * 64, kvh, r, layer);
+                }
+            }
+            if (*abort_flag) {
+                // Let the copies already issued land before the block exits.
+                for (int u = max(0, t - C::kStages); u < t; ++u)
+                    mbar_wait(&full[u % C::kStages], (u / C::kStages) & 1, p.status, abort_flag);
+            }
+        }
+    }
+
+    // ------------------------------------------------------------ consumers
+    float m[GT], l[GT];
+    float2 acc[GT][C::kDpl / 2];
+#pragma unroll
+    for (int g = 0; g < GT; ++g) {
+        m[g] = -INFINITY;
+        l[g] = 0.f;
+#pragma unroll
+        for (int e = 0; e < C::kDpl / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
+    }
+    if (warp < kConsumerWarps) {
+        float *pw = p_s + warp * kTileKeys * Gp;
+        const int kA = lane, kB = lane + 32;
+        const int sw = lane & 7;  // (kA & 7) == (kB & 7)
+        for (int t = warp; t < ntiles; t += kConsumerWarps) {
+            const int s = t % C::kStages;
+            if (!mbar_wait(&full[s], (t / C::kStages) & 1, p.status, abort_flag)) break;
+            const uint8_t *Ks = smem + s * C::kStageBytes;
+            const uint8_t *Vs = Ks + C::kTileBytes;
+            const int valid = min(kTileKeys, nkeys - t * kTileKeys);
+
+            // scores: lane owns keys kA and kB
+            float2 dA[GT], dB[GT];
+#pragma unroll
+            for (int g = 0; g < GT; ++g) dA[g] = dB[g] = make_float2(0.f, 0.f);
+#pragma unroll 2
+            for (int c = 0; c < C::kChunks; ++c) {
+                const int half = c >> 3, jj = c & 7;
+                const uint8_t *base = Ks + half * (kTileKeys * 128) + ((jj ^ sw) << 4);
+                const uint4 ka = lds128(base + kA * 128);
+                const uint4 kb = lds128(base + kB * 128);
+                const float2 a0 = w2f(ka.x), a1 = w2f(ka.y), a2 = w2f(ka.z), a3 = w2f(ka.w);
+                const float2 b0 = w2f(kb.x), b1 = w2f(kb.y), b2 = w2f(kb.z), b3 = w2f(kb.w);
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    const float4 q0 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8);
+                    const float4 q1 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8 + 4);
+                    const float2 x0 = make_float2(q0.x, q0.y), x1 = make_float2(q0.z, q0.w);
+                    const float2 x2 = make_float2(q1.x, q1.y), x3 = make_float2(q1.z, q1.w);
+                    dA[g] = __ffma2_rn(a0, x0, dA[g]);
+                    dA[g] = __ffma2_rn(a1, x1, dA[g]);
+                    dA[g] = __ffma2_rn(a2, x2, dA[g]);
+                    dA[g] = __ffma2_rn(a3, x3, dA[g]);
+                    dB[g] = __ffma2_rn(b0, x0, dB[g]);
+                    dB[g] = __ffma2_rn(b1, x1, dB[g]);
+                    dB[g] = __ffma2_rn(b2, x2, dB[g]);
+                    dB[g] = __ffma2_rn(b3, x3, dB[g]);
+                }
+            }
+            // online softmax (base 2), per query head
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const float sA = kA < valid ? dA[g].x + dA[g].y : -INFINITY;
+                const float sB = kB < valid ? dB[g].x + dB[g].y : -INFINITY;
+                float tmax = fmaxf(sA, sB);
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1)
+                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+                const float mn = fmaxf(m[g], tmax);
+                const float alpha = ex2(m[g] - mn);
+                const float pA = ex2(sA - mn), pB = ex2(sB - mn);
+                l[g] = l[g] * alpha + pA + pB;
+#pragma unroll
+                for (int e = 0; e < C::kDpl / 2; ++e) {
+                    acc[g][e].x *= alpha;
+                    acc[g][e].y *= alpha;
+                }
+                m[g] = mn;
+                pw[kA * Gp + g] = pA;
+                pw[kB * Gp + g] = pB;
+            }
+            __syncwarp();
+            // P . V: lane owns output dims [lane * kDpl, lane * kDpl + kDpl)
+            {
+                const int e0 = lane * C::kDpl;
+                const int half = e0 >> 6, jj = (e0 & 63) >> 3;
+                const int sub = (e0 & 7) * 2;  // byte offset inside the 16-byte piece
+                const uint8_t *vb = Vs + half * (kTileKeys * 128) + sub;
+#pragma unroll 4
+                for (int k = 0; k < valid; ++k) {
+                    const uint8_t *vrow = vb + k * 128 + ((jj ^ (k & 7)) << 4);
+                    float2 v[C::kDpl / 2];
+                    if constexpr (C::kDpl == 4) {
+                        const uint2 w = *reinterpret_cast<const uint2 *>(vrow);
+                        v[0] = w2f(w.x);
+                        v[1] = w2f(w.y);
+                    } else {
+                        v[0] = w2f(*reinterpret_cast<const uint32_t *>(vrow));
+                    }
+                    const float *pk = pw + k * Gp;
+#pragma unroll
+                    for (int g4 = 0; g4 < Gp; g4 += 4) {
+                        const float4 pv = *reinterpret_cast<const float4 *>(pk + g4);
+                        const float pp[4] = {pv.x, pv.y, pv.z, pv.w};
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            if (g4 + u < GT) {
+                                const float2 pp2 = make_float2(pp[u], pp[u]);
+#pragma unroll
+                                for (int e = 0; e < C::kDpl / 2; ++e)
+                                    acc[g4 + u][e] = __ffma2_rn(pp2, v[e], acc[g4 + u][e]);
+                            }
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
+        }
+        // total of the lane partial sums
+#pragma unroll
+        for (int g = 0; g < GT; ++g)
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
+    }
+    __syncthreads();
+    if (*abort_flag) return;
+
+    // ---------------------------------------------------- merge the 4 warps
+    float *macc = reinterpret_cast<float *>(smem);  // [4][GT][D] (stage memory is free now)
+    float *mml = macc + kConsumerWarps * GT * D;    // [4][GT][2]
+    if (warp < kConsumerWarps) {
+#pragma unroll
+        for (int g = 0; g < GT; ++g) {
+#pragma unroll
+            for (int e = 0; e < C::kDpl / 2; ++e)
+                *reinterpret_cast<float2 *>(macc + (warp * GT + g) * D + lane * C::kDpl + 2 * e) =
+                    acc[g][e];
+            if (lane == 0) {
+                mml[(warp * GT + g) * 2 + 0] = m[g];
+                mml[(warp * GT + g) * 2 + 1] = l[g];
+            }
+        }
+    }
+    __syncthreads();
+    const int n_chunks = (len + p.chunk_len - 1) / p.chunk_len;
+    const int64_t unit0 = ((int64_t)layer * p.B + b) * p.Hq + (int64_t)kvh * G;
+    for (int i = tid; i < G * D; i += blockDim.x) {
+        const int g = i / D, d = i - g * D;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, mml[(w * GT + g) * 2]);
+        float L = 0.f, a = 0.f;
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) {
+            const float f = ex2(mml[(w * GT + g) * 2] - M);
+            L += f * mml[(w * GT + g) * 2 + 1];
+            a += f * macc[(w * GT + g) * D + d];
+        }
+        if (n_chunks == 1) {
+            uint16_t *op = p.O + layer * p.o_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G + g) * D;
+            op[d] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
+            if (d == 0 && p.lse != nullptr) p.lse[unit0 + g] = (M + __log2f(L)) * kLn2;
+        } else {
+            const int64_t slot = (unit0 + g) * p.max_chunks + chunk;
+            p.part_acc[slot * D + d] = a;
+            if (d == 0) {
+                p.part_ml[slot * 2 + 0] = M;
+                p.part_ml[slot * 2 + 1] = L;
+            }
+        }
+    }
+}
+
+// One warp per (layer, sequence, query head).
+template <int D>
+__global__ void __launch_bounds__(128)
+decode_combine_kernel(const DecParams p, int n_layers) {
+    const int64_t unit = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t n_units = (int64_t)n_layers * p.B * p.Hq;
+    if (unit >= n_units) return;
+    const int h = (int)(unit % p.Hq);
+    const int64_t lb = unit / p.Hq;
+    const int b = (int)(lb % p.B), layer = (int)(lb / p.B);
+    const int len = min(p.lens[b], p.max_chunks * p.chunk_len);
+    const int n_chunks = (len + p.chunk_len - 1) / p.chunk_len;
+    if (n_chunks == 1) return;  // written by the split kernel
+    uint16_t *op = p.O + layer * p.o_ls + ((int64_t)b * p.Hq + h) * D;
+    constexpr int kDpl = D / 32;
+    if (n_chunks <= 0) {
+#pragma unroll
+        for (int e = 0; e < kDpl; ++e) op[lane * kDpl + e] = 0;
+        if (lane == 0 && p.lse != nullptr) p.lse[unit] = -INFINITY;
+        return;
+    }
+    const float *ml = p.part_ml + unit * p.max_chunks * 2;
+    const float *ac = p.part_acc + unit * p.max_chunks * D;
+    float M = -INFINITY;
+    for (int c = lane; c < n_chunks; c += 32) M = fmaxf(M, ml[2 * c]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float L = 0.f;
+    float a[kDpl];
+#pragma unroll
+    for (int e = 0; e < kDpl; ++e) a[e] = 0.f;
+    for (int c = 0; c < n_chunks; ++c) {
+        const float f = ex2(ml[2 * c] - M);
+        L += f * ml[2 * c + 1];
+#pragma unroll
+        for (int e = 0; e < kDpl; ++e) a[e] += f * ac[(int64_t)c * D + lane * kDpl + e];
+    }
+#pragma unroll
+    for (int e = 0; e < kDpl; ++e)
+        op[lane * kDpl + e] = __bfloat16_as_ushort(__float2bfloat16_rn(a[e] / L));
+    if (lane == 0 && p.lse != nullptr) p.lse[unit] = (M + __log2f(L)) * kLn2;
+}
+
+int g_template(int G) {
+    if (G <= 1) return 1;
+    if (G <= 2) return 2;
+    if (G <= 4) return 4;
+    if (G <= 7) return 7;
+    if (G <= 8) return 8;
+    if (G <= 16) return 16;
+    return 0;
+}
+
+struct Plan {
+    int chunk_len, max_chunks;
+    size_t ws_acc, ws_ml;
+};
+
+Plan make_plan(const sonic_decode_args *a) {
+    Plan pl{};
+    const int max_len = a->max_len > 0 ? a->max_len : 1;
+    int C = a->chunk_len;
+    if (C <= 0) {
+        const long long units = (long long)a->batch * a->n_heads_kv * a->n_layers;
+        const long long target = 4LL * device_sm_count();
+        long long splits = units >= target ? 1 : (target + units - 1) / units;
+        long long c = (max_len + splits - 1) / splits;
+        c = (c + 255) / 256 * 256;
+        C = (int)(c < 256 ? 256 : c);
+    }
+    pl.chunk_len = C;
+    pl.max_chunks = (max_len + C - 1) / C;
+    const size_t units_q = (size_t)a->batch * a->n_heads_q * a->n_layers;
+    if (pl.max_chunks > 1) {
+        pl.ws_acc = round_up(units_q * pl.max_chunks * a->head_dim * sizeof(float), 256);
+        pl.ws_ml = round_up(units_q * pl.max_chunks * 2 * sizeof(float), 256);
+    }
+    return pl;
+}
+
+template <int D, int GT>
+cudaError_t launch_split(const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
+                         dim3 grid, cudaStream_t stream) {
+    constexpr size_t smem = dec_smem_bytes<D, GT>();
+    static_assert(smem <= 232448, "decode shared memory");
+    auto kern = decode_split_kernel<D, GT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kDecThreads, smem, stream>>>(tk, tv, p);
+    return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t dispatch_g(int GT, const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
+                       dim3 grid, cudaStream_t s) {
+    switch (GT) {
+        case 1: return launch_split<D, 1>(tk, tv, p, grid, s);
+        case 2: return launch_split<D, 2>(tk, tv, p, grid, s);
+        case 4: return launch_split<D, 4>(tk, tv, p, grid, s);
+        case 7: return launch_split<D, 7>(tk, tv, p, grid, s);
+        case 8: return launch_split<D, 8>(tk, tv, p, grid, s);
+        case 16: return launch_split<D, 16>(tk, tv, p, grid, s);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace
+}  // namespace sonic
+
+using namespace sonic;
+
+extern "C" size_t sonic_decode_workspace_size(const sonic_decode_args *a) {
+    if (a == nullptr || a->batch <= 0 || a->n_layers < 1 || a->n_heads_q < 1 ||
+        a->head_dim < 1)
+        return 0;
+    Plan pl = make_plan(a);
+    return pl.ws_acc + pl.ws_ml;
+}
+
+extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
+                                            const uint16_t *V_ret, const int32_t *lens,
+                                            uint16_t *O, const sonic_decode_args *a,
+                                            sonic_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (a == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch < 0 || a->n_layers < 1 || a->n_heads_kv < 1 || a->n_heads_q < 1 ||
+        a->n_heads_q % a->n_heads_kv != 0 || a->max_len < 0 || a->total_kv_rows < 0)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch == 0) return SONIC_OK;
+    if (q == nullptr || K_ret == nullptr || V_ret == nullptr || lens == nullptr ||
+        O == nullptr || a->kv_start == nullptr)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    const int D = a->head_dim;
+    if (D != 64 && D != 128) return SONIC_ERR_UNSUPPORTED;
+    const int G = a->n_heads_q / a->n_heads_kv;
+    const int GT = g_template(G);
+    if (GT == 0) return SONIC_ERR_UNSUPPORTED;
+    if (a->chunk_len < 0 || (a->chunk_len % kTileKeys) != 0) return SONIC_ERR_INVALID_ARGUMENT;
+    if (!aligned16(K_ret) || !aligned16(V_ret)) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->n_layers > 1 && (a->kv_layer_stride <= 0 || (a->kv_layer_stride * 2) % 16 != 0))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->total_kv_rows == 0 || a->max_len == 0) {
+        // nothing to attend: every output is zero
+        for (int l = 0; l < a->n_layers; ++l)
+            if (cudaMemsetAsync(O + l * a->o_layer_stride, 0,
+                                (size_t)a->batch * a->n_heads_q * D * 2, stream) != cudaSuccess)
+                return SONIC_ERR_CUDA;
+        return SONIC_OK;
+    }
+    Plan pl = make_plan(a);
+    const size_t need = pl.ws_acc + pl.ws_ml;
+    if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
+        return SONIC_ERR_WORKSPACE;
+    if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_kv > 65535 ||
+        pl.max_chunks > 0x7fffffff)
+        return SONIC_ERR_UNSUPPORTED;
+
+    const uint64_t row_elems = (uint64_t)a->n_heads_kv * D;
+    const uint64_t layer_bytes = a->n_layers > 1 ? (uint64_t)a->kv_layer_stride * 2
+                                                 : (uint64_t)a->total_kv_rows * row_elems * 2;
+    const uint64_t dims[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_kv_rows,
+                              (uint64_t)a->n_layers};
+    const uint64_t strides[3] = {(uint64_t)D * 2, row_elems * 2, layer_bytes};
+    const uint32_t box[4] = {64, 1, (uint32_t)kTileKeys, 1};
+    CUtensorMap tk, tv;
+    if (!make_tmap_bf16_4d(&tk, K_ret, dims, strides, box) ||
+        !make_tmap_bf16_4d(&tv, V_ret, dims, strides, box))
+        return SONIC_ERR_INVALID_ARGUMENT;
+
+    DecParams p{};
+    p.q = q;
+    p.O = O;
+    p.lens = lens;
+    p.kv_start = a->kv_start;
+    p.lse = a->lse;
+    p.part_acc = static_cast<float *>(a->workspace);
+    p.part_ml = reinterpret_cast<float *>(static_cast<char *>(a->workspace) + pl.ws_acc);
+    p.status = a->status;
+    p.B = a->batch;
+    p.Hq = a->n_heads_q;
+    p.Hkv = a->n_heads_kv;
+    p.G = G;
+    p.q_ls = a->q_layer_stride;
+    p.o_ls = a->o_layer_stride;
+    p.chunk_len = pl.chunk_len;
+    p.max_chunks = pl.max_chunks;
+    const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
+    p.scale_log2 = scale * kLog2e;
+
+    dim3 grid(pl.max_chunks, a->n_heads_kv, a->batch * a->n_layers);
+    cudaError_t e = (D == 128) ? dispatch_g<128>(GT, tk, tv, p, grid, stream)
+                               : dispatch_g<64>(GT, tk, tv, p, grid, stream);
+    if (e != cudaSuccess) return SONIC_ERR_CUDA;
+    const long long units = (long long)a->n_layers * a->batch * a->n_heads_q;
+    const unsigned cblocks = (unsigned)((units * 32 + 127) / 128);
+    if (D == 128)
+        decode_combine_kernel<128><<<cblocks, 128, 0, stream>>>(p, a->n_layers);
+    else
+        decode_combine_kernel<64><<<cblocks, 128, 0, stream>>>(p, a->n_layers);
+    return cudaGetLastError() == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
+}

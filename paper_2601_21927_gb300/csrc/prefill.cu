@@ -1,0 +1,647 @@
+// Masked prefill: flash-style attention under SONIC's hierarchical visibility
+// mask (Sec. 3.2: Eq. 3 causal rule, Eq. 4 historical body removal, Eq. 5
+// bidirectional Nexus visibility), on the sm_103a tensor cores.
+//
+// One block computes a 128-row query tile of one (layer, sequence, query
+// head).  Six warps:
+//   warp 0     TMA producer: the Q tile once, then K and V tiles (128 keys)
+//              into a 2-stage ring, with the role/segment numbers of the keys;
+//   warp 1     tcgen05 issuer: S = Q K^T into one of two TMEM buffers (fp32,
+//              128 lanes x 128 columns), and O += P V into a TMEM accumulator,
+//              one elected thread issuing every MMA;
+//   warps 2-5  softmax: thread r owns query row r (TMEM lane r).  It reads its
+//              S row with tcgen05.ld, applies the mask per element only on
+//              tiles the mask cuts, runs the online softmax in base 2, rescales
+//              its O row in TMEM when the running maximum moves, and writes P
+//              (bf16) into shared memory in the 128-byte-swizzled K-major
+//              layout the next MMA reads.
+// Before the loop the block lists the key tiles it must visit: each tile is
+// classified from precomputed per-tile summaries (which roles and segment
+// numbers occur in it) as hidden (skipped entirely), fully visible (no mask
+// work) or cut by the mask.  S(j+1) is computed while the softmax works on
+// S(j).
+#include "sonic_dev.cuh"
+#include "sonic_host.h"
+
+namespace sonic {
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBN = 128;
+constexpr int kPfThreads = 192;
+constexpr int kMaxKTiles = 2048;
+constexpr float kLn2f = 0.6931471805599453f;
+constexpr float kLog2ef = 1.4426950408889634f;
+
+// Summary of one 128-row key tile of one sequence.
+struct TileSum {
+    int32_t flags;     // bit0 body rows, bit1 Nexus rows, bit2 other rows
+    int32_t bseg_min;  // segment range of the body rows
+    int32_t bseg_max;
+    int32_t nseg_min;  // segment range of the Nexus rows
+    int32_t nseg_max;
+    int32_t n_rows;    // rows of the tile inside the sequence
+    int32_t pad0, pad1;
+};
+
+__global__ void __launch_bounds__(128)
+tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
+                    const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
+                    TileSum *__restrict__ out, int max_k_tiles) {
+    const int t = blockIdx.x, b = blockIdx.y;
+    const int len = k_len[b];
+    if (t * kBN >= len && t > 0) return;
+    const int r = t * kBN + threadIdx.x;
+    int flags = 0, bmin = INT_MAX, bmax = INT_MIN, nmin = INT_MAX, nmax = INT_MIN, n = 0;
+    if (r < len) {
+        const int ro = role[k_start[b] + r];
+        const int s = seg[k_start[b] + r];
+        n = 1;
+        if (ro == SONIC_ROLE_BODY) {
+            flags = 1;
+            bmin = bmax = s;
+        } else if (ro == SONIC_ROLE_NEXUS) {
+            flags = 2;
+            nmin = nmax = s;
+        } else {
+            flags = 4;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        flags |= __shfl_xor_sync(0xffffffffu, flags, o);
+        bmin = min(bmin, __shfl_xor_sync(0xffffffffu, bmin, o));
+        bmax = max(bmax, __shfl_xor_sync(0xffffffffu, bmax, o));
+        nmin = min(nmin, __shfl_xor_sync(0xffffffffu, nmin, o));
+        nmax = max(nmax, __shfl_xor_sync(0xffffffffu, nmax, o));
+        n += __shfl_xor_sync(0xffffffffu, n, o);
+    }
+    __shared__ int sh[4][6];
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) {
+        sh[w][0] = flags;
+        sh[w][1] = bmin;
+        sh[w][2] = bmax;
+        sh[w][3] = nmin;
+        sh[w][4] = nmax;
+        sh[w][5] = n;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        TileSum ts{};
+        ts.flags = 0;
+        ts.bseg_min = INT_MAX;
+        ts.bseg_max = INT_MIN;
+        ts.nseg_min = INT_MAX;
+        ts.nseg_max = INT_MIN;
+        ts.n_rows = 0;
+        for (int i = 0; i < 4; ++i) {
+            ts.flags |= sh[i][0];
+            ts.bseg_min = min(ts.bseg_min, sh[i][1]);
+            ts.bseg_max = max(ts.bseg_max, sh[i][2]);
+            ts.nseg_min = min(ts.nseg_min, sh[i][3]);
+            ts.nseg_max = max(ts.nseg_max, sh[i][4]);
+            ts.n_rows += sh[i][5];
+        }
+        out[(int64_t)b * max_k_tiles + t] = ts;
+    }
+}
+
+struct PfParams {
+    const int32_t *k_start, *k_len, *q_start, *q_len;
+    const uint8_t *role;
+    const int32_t *seg;
+    uint16_t *O;
+    float *lse;
+    int32_t *status;
+    const TileSum *sums;
+    int max_k_tiles;
+    int B, Hq, G;
+    int64_t o_ls;
+    int total_q_rows;
+    float scale_log2;
+    int nexus_mode;
+};
+
+template <int D>
+struct PfCfg {
+    static constexpr int kHalves = D / 64;
+    static constexpr int kQBytes = kBM * D * 2;
+    static constexpr int kKVBytes = kBN * D * 2;
+    static constexpr int kPBytes = kBM * kBN * 2;
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffK = kOffQ + kQBytes;
+    static constexpr int kOffV = kOffK + 2 * kKVBytes;
+    static constexpr int kOffP = kOffV + 2 * kKVBytes;
+    static constexpr int kOffRole = kOffP + kPBytes;       // [2][128] uint8
+    static constexpr int kOffSeg = kOffRole + 2 * kBN;     // [2][128] int32
+    static constexpr int kOffList = kOffSeg + 2 * kBN * 4;  // [kMaxKTiles] int32
+    static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
+    static constexpr int kNumBars = 12;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // 16 ints
+    static constexpr int kBytes = kOffMisc + 16 * 4;
+    static constexpr size_t kSmem = 1024 + kBytes;
+};
+
+__device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, int sq,
+                                        int mode) {
+    if (rq == SONIC_ROLE_BODY) return sq == sp && q <= p;                  // Eqs. 3, 4
+    if (rp == SONIC_ROLE_NEXUS && rq == SONIC_ROLE_NEXUS)                  // Eq. 5
+        return mode == SONIC_NEXUS_FULL ? true : sq <= sp;
+    return q <= p;                                                          // Eq. 3
+}
+
+template <int D>
+__global__ void __launch_bounds__(kPfThreads, 1)
+prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const __grid_constant__ CUtensorMap tmV, const PfParams p) {
+    using C = PfCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint8_t *Qs = smem + C::kOffQ;
+    uint8_t *Ks = smem + C::kOffK;
+    uint8_t *Vs = smem + C::kOffV;
+    uint8_t *Ps = smem + C::kOffP;
+    uint8_t *meta_role = smem + C::kOffRole;
+    int32_t *meta_seg = reinterpret_cast<int32_t *>(smem + C::kOffSeg);
+    int32_t *list = reinterpret_cast<int32_t *>(smem + C::kOffList);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
+    uint64_t *q_full = bars + 0;
+    uint64_t *kv_full = bars + 1;   // [2]
+    uint64_t *kv_empty = bars + 3;  // [2]
+    uint64_t *s_full = bars + 5;    // [2]
+    uint64_t *s_free = bars + 7;    // [2]
+    uint64_t *p_full = bars + 9;
+    uint64_t *o_done = bars + 10;
+    uint64_t *mma_idle = bars + 11;
+    int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
+    // misc: 0 tmem base, 1 list length, 2 abort, 3 q flags, 4 q seg min, 5 q seg max,
+    //       6 q nexus seg min, 7 q nexus seg max, 8..15 warp counts
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
+
+    const int qt = blockIdx.x, h = blockIdx.y;
+    const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
+    const int klen = p.k_len[b], qlen = p.q_len[b];
+    if (qt * kBM >= qlen || timed_out(p.status)) return;
+    if (qlen > klen || klen > p.max_k_tiles * kBN) {
+        // the host-side bounds were wrong for this sequence: refuse it
+        if (threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        return;
+    }
+    const int kstart = p.k_start[b];
+    const int kvh = h / p.G;
+    const int p0 = klen - qlen + qt * kBM;          // position of query row 0
+    const int p1 = min(p0 + kBM - 1, klen - 1);     // last valid query position
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // ------------------------------------------------ summary of the query tile
+    if (tid == 0) {
+        misc[2] = 0;
+        misc[3] = 0;
+        misc[4] = INT_MAX;
+        misc[5] = INT_MIN;
+        misc[6] = INT_MAX;
+        misc[7] = INT_MIN;
+    }
+    __syncthreads();
+    if (tid < kBM && p0 + tid <= p1) {
+        const int ro = p.role[kstart + p0 + tid];
+        const int s = p.seg[kstart + p0 + tid];
+        atomicMin(&misc[4], s);
+        atomicMax(&misc[5], s);
+        if (ro == SONIC_ROLE_NEXUS) {
+            atomicOr(&misc[3], 2);
+            atomicMin(&misc[6], s);
+            atomicMax(&misc[7], s);
+        }
+    }
+    __syncthreads();
+    const int q_has_nexus = misc[3] & 2;
+    const int qs_min = misc[4], qs_max = misc[5], qn_min = misc[6], qn_max = misc[7];
+
+    // ------------------------------------------------ list of key tiles to visit
+    const int n_kt = (klen + kBN - 1) / kBN;
+    int n_list = 0;
+    for (int c0 = 0; c0 < n_kt; c0 += kPfThreads) {
+        const int t = c0 + tid;
+        int code = 0;  // 0 hidden, 1 fully visible, 2 cut by the mask
+        if (t < n_kt) {
+            const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
+            const int k0 = t * kBN, k1 = k0 + ts.n_rows - 1;
+            const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
+            const bool causal_part = (k0 <= p1) && (kn || ko);
+            const bool body_part =
+                kb && (k0 <= p1) && !(ts.bseg_max < qs_min || ts.bseg_min > qs_max);
+            const bool nexus_part = kn && q_has_nexus &&
+                                    (p.nexus_mode == SONIC_NEXUS_FULL || ts.nseg_min <= qn_max);
+            if (causal_part || body_part || nexus_part) {
+                const bool full =
+                    ts.n_rows == kBN && k1 <= p0 &&
+                    (!kb || (ts.bseg_min == ts.bseg_max && qs_min == qs_max &&
+                             ts.bseg_min == qs_min)) &&
+                    (p.nexus_mode == SONIC_NEXUS_FULL || !(kn && q_has_nexus) ||
+                     ts.nseg_max <= qn_min);
+                code = full ? 1 : 2;
+            }
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, code != 0);
+        if (lane == 0) misc[8 + warp] = __popc(bal);
+        __syncthreads();
+        int base = n_list;
+        for (int w = 0; w < warp; ++w) base += misc[8 + w];
+        int tot = 0;
+        for (int w = 0; w < kPfThreads / 32; ++w) tot += misc[8 + w];
+        if (code != 0) {
+            const int rank = __popc(bal & ((1u << lane) - 1u));
+            list[base + rank] = (t << 1) | (code == 2 ? 1 : 0);
+        }
+        n_list += tot;
+        __syncthreads();
+    }
+
+    // ------------------------------------------------ barriers and tensor memory
+    if (tid == 0) {
+        mbar_init(q_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&kv_full[s], 32);
+            mbar_init(&kv_empty[s], 1);
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_free[s], kBM);
+        }
+        mbar_init(p_full, kBM);
+        mbar_init(o_done, 1);
+        mbar_init(mma_idle, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = static_cast<uint32_t>(misc[0]);
+    const uint32_t tmem_S0 = tmem, tmem_O = tmem + 256;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tmQ);
+            tma_prefetch_desc(&tmK);
+            tma_prefetch_desc(&tmV);
+            mbar_arrive_expect_tx(q_full, C::kQBytes);
+#pragma unroll
+            for (int hh = 0; hh < C::kHalves; ++hh)
+                tma_load_4d(Qs + hh * (kBM * 128), &tmQ, q_full, hh * 64, h,
+                            p.q_start[b] + qt * kBM, layer);
+        }
+        int i = 0;
+        for (; i < n_list; ++i) {
+            const int st = i & 1;
+            if (i >= 2 && !mbar_wait(&kv_empty[st], ((i >> 1) - 1) & 1, p.status, abort_flag))
+                break;
+            const int kt = list[i] >> 1;
+            // role / segment numbers of the tile's keys (255 marks rows past the sequence)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int c = lane * 4 + u;
+                const int q = kt * kBN + c;
+                uint8_t ro = 255;
+                int32_t sg = 0;
+                if (q < klen) {
+                    ro = p.role[kstart + q];
+                    sg = p.seg[kstart + q];
+                }
+                meta_role[st * kBN + c] = ro;
+                meta_seg[st * kBN + c] = sg;
+            }
+            if (lane == 0) {
+                mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
+                const int row = kstart + kt * kBN;
+#pragma unroll
+                for (int hh = 0; hh < C::kHalves; ++hh) {
+                    tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), &tmK, &kv_full[st],
+                                hh * 64, kvh, row, layer);
+                    tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), &tmV, &kv_full[st],
+                                hh * 64, kvh, row, layer);
+                }
+            } else {
+                mbar_arrive(&kv_full[st]);
+            }
+        }
+        if (lane == 0 && *abort_flag) {
+            // let issued copies land before the block exits
+            mbar_wait(q_full, 0, p.status, abort_flag);
+            for (int u = max(0, i - 2); u < i; ++u)
+                mbar_wait(&kv_full[u & 1], (u >> 1) & 1, p.status, abort_flag);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, 0);
+            constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, 1);
+            const uint32_t q_addr = smem_u32(Qs), k_addr = smem_u32(Ks), v_addr = smem_u32(Vs),
+                           p_addr = smem_u32(Ps);
+            bool ok = mbar_wait(q_full, 0, p.status, abort_flag);
+            auto issue_pv = [&](int j) -> bool {
+                if (!mbar_wait(p_full, j & 1, p.status, abort_flag)) return false;
+                tc_fence_after();
+                const int st = j & 1;
+#pragma unroll
+                for (int kk = 0; kk < kBN / 16; ++kk) {
+                    const uint64_t a = smem_desc_sw128(
+                        p_addr + (kk >> 2) * (kBM * 128) + (kk & 3) * 32, 16, 1024);
+                    const uint64_t bd =
+                        smem_desc_sw128(v_addr + st * C::kKVBytes + kk * (16 * 128),
+                                        kBN * 128, 1024);
+                    tc_mma_ss(tmem_O, a, bd, idPV, (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc_commit(o_done);
+                tc_commit(&kv_empty[st]);
+                return true;
+            };
+            for (int i = 0; ok && i < n_list; ++i) {
+                const int st = i & 1, sb = i & 1;
+                if (!mbar_wait(&kv_full[st], (i >> 1) & 1, p.status, abort_flag)) break;
+                if (i >= 2 && !mbar_wait(&s_free[sb], ((i >> 1) - 1) & 1, p.status, abort_flag))
+                    break;
+                tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
+                    const uint64_t a = smem_desc_sw128(q_addr + off, 16, 1024);
+                    const uint64_t bd = smem_desc_sw128(k_addr + st * C::kKVBytes + off, 16, 1024);
+                    tc_mma_ss(tmem_S0 + sb * kBN, a, bd, idS, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(&s_full[sb]);
+                if (i >= 1 && !issue_pv(i - 1)) break;
+                if (i == n_list - 1) issue_pv(i);
+            }
+            // all MMAs issued by this thread have finished once this arrives
+            tc_commit(mma_idle);
+            mbar_wait(mma_idle, 0, p.status, abort_flag);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax
+        const int quarter = warp & 3;
+        const int r = quarter * 32 + lane;
+        const int pos = p0 + r;
+        const bool row_ok = pos <= p1;
+        int rp = SONIC_ROLE_SYS, sp = 0;
+        if (row_ok) {
+            rp = p.role[kstart + pos];
+            sp = p.seg[kstart + pos];
+        }
+        const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+        float m = -INFINITY, l = 0.f;
+        bool ok = true;
+        for (int i = 0; i < n_list; ++i) {
+            const int sb = i & 1, st = i & 1;
+            if (!mbar_wait(&kv_full[st], (i >> 1) & 1, p.status, abort_flag) ||
+                !mbar_wait(&s_full[sb], (i >> 1) & 1, p.status, abort_flag)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t sr[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_base + sb * kBN + c * 32, sr[c]);
+            tmem_ld_wait();
+#pragma unroll
+            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
+            tc_fence_before();
+            mbar_arrive(&s_free[sb]);
+
+            const int kt = list[i] >> 1;
+            const bool cut = list[i] & 1;
+            float s[kBN];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int e = 0; e < 32; ++e)
+                    s[c * 32 + e] = __uint_as_float(sr[c][e]) * p.scale_log2;
+            if (cut) {
+                const uint8_t *mr = meta_role + st * kBN;
+                const int32_t *ms = meta_seg + st * kBN;
+#pragma unroll
+                for (int c = 0; c < kBN; ++c) {
+                    const int rq = mr[c];
+                    const bool v = rq != 255 &&
+                                   visible(pos, kt * kBN + c, rp, sp, rq, ms[c], p.nexus_mode);
+                    if (!v) s[c] = -INFINITY;
+                }
+            }
+            float mx = m;
+#pragma unroll
+            for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
+            const float mu = (mx == -INFINITY) ? 0.f : mx;
+            const float alpha = ex2(m - mu);
+            float rs = 0.f;
+            uint32_t pk[kBN / 2];
+#pragma unroll
+            for (int c = 0; c < kBN; c += 2) {
+                const float e0 = ex2(s[c] - mu), e1 = ex2(s[c + 1] - mu);
+                rs += e0 + e1;
+                pk[c >> 1] = pack_bf16x2(e0, e1);
+            }
+            l = l * alpha + rs;
+            m = mx;
+
+            // PV(i-1) must be done: P buffer free, O up to date.
+            if (i >= 1) {
+                if (!mbar_wait(o_done, (i - 1) & 1, p.status, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(tmem_O + lane_base + c * 32, o);
+                        tmem_ld_wait();
+                        reg_fence32(o);
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        tmem_st32(tmem_O + lane_base + c * 32, o);
+                    }
+                    tmem_st_wait();
+                }
+            }
+            // Rows of V past the sequence end: zero them so 0 * garbage cannot
+            // reach the accumulator.
+            if (kt * kBN + kBN > klen && kt * kBN + r >= klen) {
+#pragma unroll
+                for (int hh = 0; hh < C::kHalves; ++hh) {
+                    uint4 *vr = reinterpret_cast<uint4 *>(Vs + st * C::kKVBytes +
+                                                          hh * (kBN * 128) + r * 128);
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) vr[u] = make_uint4(0, 0, 0, 0);
+                }
+            }
+            // P row r, K-major, 128-byte swizzle: 16-byte piece j of 64-key block
+            // blk lands at blk * 16 KB + r * 128 + ((j ^ (r & 7)) * 16).
+#pragma unroll
+            for (int cc = 0; cc < kBN / 8; ++cc) {
+                const int blk = cc >> 3, j = cc & 7;
+                uint4 *dst = reinterpret_cast<uint4 *>(Ps + blk * (kBM * 128) + r * 128 +
+                                                       ((j ^ (r & 7)) << 4));
+                *dst = make_uint4(pk[cc * 4 + 0], pk[cc * 4 + 1], pk[cc * 4 + 2], pk[cc * 4 + 3]);
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(p_full);
+        }
+        // ------------------------------------------------------------ epilogue
+        if (ok && n_list > 0 && mbar_wait(o_done, (n_list - 1) & 1, p.status, abort_flag)) {
+            tc_fence_after();
+            const float inv = l > 0.f ? 1.f / l : 0.f;
+            uint16_t *orow = p.O + layer * p.o_ls +
+                             ((int64_t)(p.q_start[b] + qt * kBM + r) * p.Hq + h) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(tmem_O + lane_base + c * 32, o);
+                tmem_ld_wait();
+                reg_fence32(o);
+                if (row_ok) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            w[e] = pack_bf16x2(__uint_as_float(o[u * 8 + 2 * e]) * inv,
+                                               __uint_as_float(o[u * 8 + 2 * e + 1]) * inv);
+                        dst[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                    }
+                }
+            }
+            if (row_ok && p.lse != nullptr)
+                p.lse[((int64_t)layer * p.total_q_rows + p.q_start[b] + qt * kBM + r) * p.Hq + h] =
+                    l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
+        } else if (row_ok && n_list == 0) {
+            uint16_t *orow = p.O + layer * p.o_ls +
+                             ((int64_t)(p.q_start[b] + qt * kBM + r) * p.Hq + h) * D;
+            for (int d = 0; d < D; ++d) orow[d] = 0;
+            if (p.lse != nullptr)
+                p.lse[((int64_t)layer * p.total_q_rows + p.q_start[b] + qt * kBM + r) * p.Hq + h] =
+                    -INFINITY;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+template <int D>
+cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
+                           const PfParams &p, dim3 grid, cudaStream_t s) {
+    constexpr size_t smem = PfCfg<D>::kSmem;
+    static_assert(smem <= 232448, "prefill shared memory");
+    auto kern = prefill_kernel<D>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kPfThreads, smem, s>>>(tq, tk, tv, p);
+    return cudaGetLastError();
+}
+
+int max_k_tiles_of(const sonic_prefill_args *a) {
+    return (a->max_k_len + kBN - 1) / kBN;
+}
+
+}  // namespace
+}  // namespace sonic
+
+using namespace sonic;
+
+extern "C" size_t sonic_prefill_workspace_size(const sonic_prefill_args *a) {
+    if (a == nullptr || a->batch <= 0 || a->max_k_len <= 0) return 0;
+    return round_up((size_t)a->batch * max_k_tiles_of(a) * sizeof(TileSum), 256);
+}
+
+extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K,
+                                             const uint16_t *V, const int32_t *seg_id,
+                                             const uint8_t *role, uint16_t *O,
+                                             const sonic_prefill_args *a,
+                                             sonic_stream_t stream_) {
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (a == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch < 0 || a->n_layers < 1 || a->n_heads_kv < 1 || a->n_heads_q < 1 ||
+        a->n_heads_q % a->n_heads_kv != 0 || a->max_q_len < 0 || a->max_k_len < 0 ||
+        a->total_q_rows < 0 || a->total_k_rows < 0)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->batch == 0 || a->max_q_len == 0) return SONIC_OK;
+    if (Q == nullptr || K == nullptr || V == nullptr || O == nullptr || role == nullptr ||
+        seg_id == nullptr || a->k_start == nullptr || a->k_len == nullptr ||
+        a->q_start == nullptr || a->q_len == nullptr)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    const int D = a->head_dim;
+    if (D != 64 && D != 128) return SONIC_ERR_UNSUPPORTED;
+    if (a->nexus_vis != SONIC_NEXUS_FULL && a->nexus_vis != SONIC_NEXUS_CAUSAL_SEGMENTS)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->max_k_len < a->max_q_len || a->total_k_rows == 0 || a->total_q_rows == 0)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (max_k_tiles_of(a) > kMaxKTiles) return SONIC_ERR_UNSUPPORTED;
+    if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->n_layers > 1 && (a->q_layer_stride <= 0 || a->kv_layer_stride <= 0 ||
+                            a->o_layer_stride <= 0 || (a->q_layer_stride * 2) % 16 != 0 ||
+                            (a->kv_layer_stride * 2) % 16 != 0 ||
+                            (a->o_layer_stride * 2) % 16 != 0))
+        return SONIC_ERR_INVALID_ARGUMENT;
+    const size_t need = sonic_prefill_workspace_size(a);
+    if (a->workspace == nullptr || a->workspace_bytes < need) return SONIC_ERR_WORKSPACE;
+    const long long qtiles = (a->max_q_len + kBM - 1) / kBM;
+    if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_q > 65535 || qtiles > 0x7fffffff)
+        return SONIC_ERR_UNSUPPORTED;
+
+    const uint64_t qrow = (uint64_t)a->n_heads_q * D, krow = (uint64_t)a->n_heads_kv * D;
+    const uint64_t q_layer = a->n_layers > 1 ? (uint64_t)a->q_layer_stride * 2
+                                             : (uint64_t)a->total_q_rows * qrow * 2;
+    const uint64_t k_layer = a->n_layers > 1 ? (uint64_t)a->kv_layer_stride * 2
+                                             : (uint64_t)a->total_k_rows * krow * 2;
+    const uint64_t qd[4] = {(uint64_t)D, (uint64_t)a->n_heads_q, (uint64_t)a->total_q_rows,
+                            (uint64_t)a->n_layers};
+    const uint64_t qs[3] = {(uint64_t)D * 2, qrow * 2, q_layer};
+    const uint64_t kd[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_k_rows,
+                            (uint64_t)a->n_layers};
+    const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, k_layer};
+    const uint32_t box[4] = {64, 1, 128, 1};
+    CUtensorMap tq, tk, tv;
+    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, box) || !make_tmap_bf16_4d(&tk, K, kd, ks, box) ||
+        !make_tmap_bf16_4d(&tv, V, kd, ks, box))
+        return SONIC_ERR_INVALID_ARGUMENT;
+
+    PfParams p{};
+    p.k_start = a->k_start;
+    p.k_len = a->k_len;
+    p.q_start = a->q_start;
+    p.q_len = a->q_len;
+    p.role = role;
+    p.seg = seg_id;
+    p.O = O;
+    p.lse = a->lse;
+    p.status = a->status;
+    p.sums = static_cast<const TileSum *>(a->workspace);
+    p.max_k_tiles = max_k_tiles_of(a);
+    p.B = a->batch;
+    p.Hq = a->n_heads_q;
+    p.G = a->n_heads_q / a->n_heads_kv;
+    p.o_ls = a->o_layer_stride;
+    p.total_q_rows = a->total_q_rows;
+    const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
+    p.scale_log2 = scale * kLog2ef;
+    p.nexus_mode = a->nexus_vis;
+
+    tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
+        role, seg_id, a->k_start, a->k_len, static_cast<TileSum *>(a->workspace), p.max_k_tiles);
+    dim3 grid((unsigned)qtiles, a->n_heads_q, a->batch * a->n_layers);
+    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
+                               : launch_prefill<64>(tq, tk, tv, p, grid, stream);
+    return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
+}

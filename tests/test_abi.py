@@ -1,0 +1,103 @@
+"""The C ABI (no GPU needed): the library loads, exports every entry point
+declared in include/sonic.h, the ctypes structs match the C layout, and host
+validation rejects bad arguments before anything is launched."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2601_21927_gb300 import sonic
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sonic.h")
+
+
+def _declared():
+    txt = open(HEADER).read()
+    return sorted(set(re.findall(r"SONIC_API\s+[\w\s\*]+?\b(sonic_\w+)\s*\(", txt)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = sonic.load()
+    names = _declared()
+    assert len(names) >= 9
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(sonic.SIGNATURES)
+    assert lib.sonic_abi_version() == 1
+    assert lib.sonic_status_string(4) == b"output capacity exceeded"
+
+
+def test_struct_layout_matches_c(tmp_path):
+    structs = {"sonic_compact_args": sonic.sonic_compact_args,
+               "sonic_prefill_args": sonic.sonic_prefill_args,
+               "sonic_decode_args": sonic.sonic_decode_args}
+    src = ['#include <stdio.h>', '#include <stddef.h>', '#include "sonic.h"', 'int main(void){']
+    for name, cls in structs.items():
+        src.append(f'printf("{name} %zu\\n", sizeof({name}));')
+        for f, _ in cls._fields_:
+            src.append(f'printf("{name}.{f} %zu\\n", offsetof({name}, {f}));')
+    src.append("return 0;}")
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                 check=True).stdout.splitlines())
+    for name, cls in structs.items():
+        assert int(out[name]) == ctypes.sizeof(cls), name
+        for f, _ in cls._fields_:
+            assert int(out[f"{name}.{f}"]) == getattr(cls, f).offset, f"{name}.{f}"
+
+
+def test_host_validation_rejects_before_launch():
+    lib = sonic.load()
+    # NULL args / offsets
+    assert lib.sonic_compact_kv(None, None, None, None, None, None, None, None, None) == 1
+    a = sonic.sonic_compact_args()
+    a.batch, a.n_layers = 2, 1
+    assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, None, ctypes.byref(a), None) == 1
+    a.row_bytes = 24  # not a multiple of 16
+    a.k_start = a.k_len = 16
+    assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 1
+    a.row_bytes = 32
+    assert lib.sonic_compact_kv(17, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 1  # misaligned
+    assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 3  # no workspace
+
+    p = sonic.sonic_prefill_args()
+    p.batch, p.n_layers, p.n_heads_q, p.n_heads_kv, p.head_dim = 1, 1, 6, 4, 128
+    p.max_q_len = p.max_k_len = p.total_q_rows = p.total_k_rows = 8
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 1  # 6 % 4
+    p.n_heads_q, p.head_dim = 8, 96
+    p.k_start = p.k_len = p.q_start = p.q_len = 16
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 2  # D = 96
+    p.head_dim = 128
+    p.max_k_len = 300000
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 2  # too long
+    p.max_k_len = 8
+    p.nexus_vis = 5
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 1
+    p.nexus_vis = 0
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 3  # workspace
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256
+
+    d = sonic.sonic_decode_args()
+    d.batch, d.n_layers, d.n_heads_q, d.n_heads_kv, d.head_dim = 2, 1, 40, 2, 128
+    d.kv_start, d.max_len, d.total_kv_rows = 16, 10, 20
+    assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 2  # G = 20 > 16
+    d.n_heads_q = 8
+    d.chunk_len = 100
+    assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 1  # not x64
+    d.chunk_len, d.head_dim = 0, 80
+    assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 2
+
+
+def test_python_binding_has_no_cpu_path():
+    src = open(os.path.join(ROOT, "paper_2601_21927_gb300", "sonic.py")).read()
+    assert "import oracle" not in src and "from oracle" not in src
+    for f in os.listdir(os.path.join(ROOT, "paper_2601_21927_gb300")):
+        if f.endswith(".py"):
+            t = open(os.path.join(ROOT, "paper_2601_21927_gb300", f)).read()
+            assert "oracle" not in re.findall(r"^\s*(?:import|from)\s+(\w+)", t, re.M), f
