@@ -1,0 +1,479 @@
+"""Benchmark of the SONIC Nexus-KV attention path on GB300.
+
+One step = one mixed serving step over 28 layers (28 query / 4 KV heads,
+D = 128, bf16), the whole hot path in order:
+  1. compaction: the 8 sequences that resume with a new turn drop the bodies
+     of their raw histories (~U[4k, 64k] tokens each) -- retention rule;
+  2. masked prefill: their new turns (~U[256, 2048] tokens) attend over the
+     retained cache plus themselves under the Sec. 3.2 mask;
+  3. decode: the other 56 sequences decode one token over retained caches of
+     ~1k-18k rows.
+All three calls go through the C ABI on one CUDA stream.
+
+Reported:
+  value        prefill TFLOP/s (algorithmic: 4 * D * Hq * visible pairs) over
+               the prefill launches of the timed steps (the dominant kernel);
+  decode       HBM GB/s (retained K/V read + q/O) over the decode launches;
+  compaction   HBM GB/s (kept rows read + written) over the compaction launches;
+  e2e          the same metric with every step's inputs copied from pinned
+               host memory and its outputs read back inside the timed region;
+  roofline     the prefill kernel against the measured bf16 peak;
+  cpu_baseline the double-precision oracle timed on a bounded sample.
+`--impl reference` times the oracle itself on that sample (reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "Nexus-KV attn: decode HBM GB/s & prefill TFLOP/s vs GB300 peak"
+WORKLOAD = ("mixed serving step: 64 ragged sequences, 28 layers, 28/4 heads, D=128, bf16; "
+            "8 compact a 4k-64k raw history then prefill a 256-2048-token turn, 56 decode "
+            "over 1k-18k retained rows")
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"],
+                    bf16_sus=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+# ---------------------------------------------------------------------------
+# Workload (host side: layout bookkeeping only)
+# ---------------------------------------------------------------------------
+
+class Layout:
+    def __init__(self, seed: int = 1):
+        from paper_2601_21927_gb300 import inputs
+        self.ms = ms = inputs.mixed_serving(seed=seed)
+        h = ms.heads
+        self.NL, self.HQ, self.HKV, self.D = h.n_layers, h.hq, h.hkv, h.d
+        self.row_bytes = self.HKV * self.D * 2
+        # raw histories of the prefill sequences (packed)
+        self.raw = inputs.Batch(ms.raw_hist)
+        self.n_pre = len(ms.raw_hist)
+        self.q_len = np.array(ms.prefill_q, np.int32)
+        self.ret_pre = np.array([d.recipe_retained for d in ms.raw_hist], np.int32)
+        # retained-cache buffer: decode sequences first, then the prefill region
+        self.dec_len = np.array([d.recipe_retained + 1 for d in ms.decode_hist], np.int32)
+        self.n_dec = len(self.dec_len)
+        self.dec_start = np.concatenate([[0], np.cumsum(self.dec_len)[:-1]]).astype(np.int32)
+        self.T_dec = int(self.dec_len.sum())
+        self.pre_off = np.concatenate([[0], np.cumsum(self.ret_pre + self.q_len)[:-1]]).astype(np.int32)
+        self.T_pre = int((self.ret_pre + self.q_len).sum())
+        self.T_ret = self.T_dec + self.T_pre
+        self.k_start_pre = (self.T_dec + self.pre_off).astype(np.int32)
+        self.k_len_pre = (self.ret_pre + self.q_len).astype(np.int32)
+        self.q_start = np.concatenate([[0], np.cumsum(self.q_len)[:-1]]).astype(np.int32)
+        self.T_q = int(self.q_len.sum())
+        # role / segment numbers of every row of the retained buffer
+        role = np.zeros(self.T_ret, np.uint8)
+        seg = np.zeros(self.T_ret, np.int32)
+        for b, d in enumerate(ms.decode_hist):
+            r, s = d.retained_arrays()
+            s0 = self.dec_start[b]
+            role[s0:s0 + len(r)] = r
+            seg[s0:s0 + len(r)] = s
+            role[s0 + len(r)] = 3
+            seg[s0 + len(r)] = len(d.segments) + 1
+        for b, d in enumerate(ms.raw_hist):
+            r, s = d.retained_arrays()
+            s0 = self.k_start_pre[b]
+            role[s0:s0 + len(r)] = r
+            seg[s0:s0 + len(r)] = s
+            role[s0 + len(r):s0 + len(r) + self.q_len[b]] = 3
+            seg[s0 + len(r):s0 + len(r) + self.q_len[b]] = len(d.segments) + 1
+        self.role_ret, self.seg_ret = role, seg
+
+    # algorithmic work per step
+    def prefill_flops(self) -> float:
+        pairs = sum(int(q) * int(r) + int(q) * (int(q) + 1) // 2
+                    for q, r in zip(self.q_len, self.ret_pre))
+        return 4.0 * self.D * self.HQ * pairs * self.NL
+
+    def decode_bytes(self) -> float:
+        kv = float(self.dec_len.sum()) * self.row_bytes * 2
+        qo = 2.0 * self.n_dec * self.HQ * self.D * 2
+        meta = self.n_dec * 8.0
+        return (kv + qo + meta) * self.NL
+
+    def compact_bytes(self) -> float:
+        return float(self.ret_pre.sum()) * self.row_bytes * 2 * 2 * self.NL
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+class GpuStep:
+    def __init__(self, lay: Layout, device, seed: int = 0):
+        import torch
+        from paper_2601_21927_gb300 import inputs, sonic
+        self.torch, self.sonic, self.lay = torch, sonic, lay
+        t = lambda a: torch.as_tensor(a).to(device)
+        NL, HQ, HKV, D = lay.NL, lay.HQ, lay.HKV, lay.D
+        bf = torch.bfloat16
+        # KV cache state (resident)
+        self.rawK = inputs.randn((NL, lay.raw.total, HKV, D), seed=seed + 1, device=device)
+        self.rawV = inputs.randn((NL, lay.raw.total, HKV, D), seed=seed + 2, device=device)
+        self.Kret = inputs.randn((NL, lay.T_ret, HKV, D), seed=seed + 3, device=device)
+        self.Vret = inputs.randn((NL, lay.T_ret, HKV, D), seed=seed + 4, device=device)
+        self.raw_role, self.raw_seg = t(lay.raw.role), t(lay.raw.seg)
+        self.raw_kstart, self.raw_klen = t(lay.raw.k_start), t(lay.raw.k_len)
+        self.reserve = t(lay.q_len)
+        self.offsets = torch.zeros(lay.n_pre + 1, dtype=torch.int32, device=device)
+        self.role_ret, self.seg_ret = t(lay.role_ret), t(lay.seg_ret)
+        self.k_start_pre, self.k_len_pre = t(lay.k_start_pre), t(lay.k_len_pre)
+        self.q_start, self.q_len = t(lay.q_start), t(lay.q_len)
+        self.dec_start, self.dec_len = t(lay.dec_start), t(lay.dec_len)
+        # per-step inputs and outputs
+        self.Qp = inputs.randn((NL, lay.T_q, HQ, D), seed=seed + 5, device=device)
+        self.Op = torch.empty_like(self.Qp)
+        self.qd = inputs.randn((NL, lay.n_dec, HQ, D), seed=seed + 6, device=device)
+        self.Od = torch.empty_like(self.qd)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self.outK = self.Kret[:, lay.T_dec:]
+        self.outV = self.Vret[:, lay.T_dec:]
+        # workspaces (caller-owned; sized once)
+        self.ws_c = self.ws_p = self.ws_d = None
+        self.launches_per_step = 3 + 2 + 2
+
+    def compact(self, stream=None):
+        self.ws_c = self.sonic.sonic_compact_kv(
+            self.rawK, self.rawV, self.raw_seg, self.raw_role, self.outK, self.outV,
+            self.offsets, k_start=self.raw_kstart, k_len=self.raw_klen, reserve=self.reserve,
+            status=self.status, workspace=self.ws_c, stream=stream)
+
+    def prefill(self, stream=None):
+        lay = self.lay
+        self.ws_p = self.sonic.sonic_attn_prefill(
+            self.Qp, self.Kret, self.Vret, self.seg_ret, self.role_ret, self.Op,
+            k_start=self.k_start_pre, k_len=self.k_len_pre, q_start=self.q_start,
+            q_len=self.q_len, max_q_len=int(lay.q_len.max()), max_k_len=int(lay.k_len_pre.max()),
+            status=self.status, workspace=self.ws_p, stream=stream)
+
+    def decode(self, stream=None):
+        self.ws_d = self.sonic.sonic_attn_decode(
+            self.qd, self.Kret, self.Vret, self.dec_len, self.Od, kv_start=self.dec_start,
+            max_len=int(self.lay.dec_len.max()), status=self.status, workspace=self.ws_d,
+            stream=stream)
+
+    def step(self, stream=None):
+        self.compact(stream)
+        self.prefill(stream)
+        self.decode(stream)
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [l.strip().split(", ") for l in self.file.read().splitlines() if l.strip()]
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = max(mx, float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip() == "Active":
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def run_gpu(args, rank: int, world: int):
+    import torch
+    import torch.distributed as dist
+    from paper_2601_21927_gb300 import sonic
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    sonic.load()
+    lay = Layout()
+    g = GpuStep(lay, device, seed=17 * rank)
+    stream = torch.cuda.Stream(device)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g.step(stream)
+    torch.cuda.synchronize()
+    if sonic.read_status(g.status) != 0:
+        raise RuntimeError(f"device status {sonic.read_status(g.status)} after warm-up")
+
+    marks = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier()
+    clocks.start()
+    t_start, t_end = ev(), ev()
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for e0, e1, e2, e3 in marks:
+            e0.record(stream)
+            g.compact(stream)
+            e1.record(stream)
+            g.prefill(stream)
+            e2.record(stream)
+            g.decode(stream)
+            e3.record(stream)
+        t_end.record(stream)
+    barrier()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    c_ms = sum(a.elapsed_time(b) for a, b, _, _ in marks)
+    p_ms = sum(b.elapsed_time(c) for _, b, c, _ in marks)
+    d_ms = sum(c.elapsed_time(d) for _, _, c, d in marks)
+    if sonic.read_status(g.status) != 0:
+        raise RuntimeError("device status set during the timed steps")
+
+    # ---------------- end to end: host buffers through the public calls
+    pin = lambda t: t.cpu().pin_memory()
+    hQ, hqd = pin(g.Qp), pin(g.qd)
+    hOp, hOd = torch.empty_like(hQ).pin_memory(), torch.empty_like(hqd).pin_memory()
+    newK = pin(g.Kret[:, lay.T_dec:][:, 0:1].expand(-1, lay.T_q, -1, -1).contiguous())
+    newV = pin(newK.clone())
+    dec_rows = lay.dec_start + lay.dec_len - 1
+    hdecK = pin(g.Kret[:, torch.as_tensor(dec_rows, device=device).long()])
+    hdecV = pin(g.Vret[:, torch.as_tensor(dec_rows, device=device).long()])
+    dst_rows = [(int(lay.k_start_pre[b] + lay.ret_pre[b]), int(lay.q_len[b]), int(lay.q_start[b]))
+                for b in range(lay.n_pre)]
+    dec_rows_dev = torch.as_tensor(dec_rows, device=device).long()
+    h2d = (hQ.numel() + hqd.numel() + newK.numel() + newV.numel() + hdecK.numel() +
+           hdecV.numel()) * 2
+    d2h = (hOp.numel() + hOd.numel()) * 2
+
+    def e2e_step():
+        g.Qp.copy_(hQ, non_blocking=True)
+        g.qd.copy_(hqd, non_blocking=True)
+        for s, n, qs in dst_rows:
+            g.Kret[:, s:s + n].copy_(newK[:, qs:qs + n], non_blocking=True)
+            g.Vret[:, s:s + n].copy_(newV[:, qs:qs + n], non_blocking=True)
+        g.Kret[:, dec_rows_dev] = hdecK.to(device, non_blocking=True)
+        g.Vret[:, dec_rows_dev] = hdecV.to(device, non_blocking=True)
+        g.step(stream)
+        hOp.copy_(g.Op, non_blocking=True)
+        hOd.copy_(g.Od, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup // 2)):
+            e2e_step()
+    barrier()
+    e0, e1 = ev(), ev()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+
+    # max over ranks
+    vals = torch.tensor([total_ms, c_ms, p_ms, d_ms, e2e_ms], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+    total_ms, c_ms, p_ms, d_ms, e2e_ms = vals.tolist()
+    K = args.steps
+    pk = _peaks()
+    pf = lay.prefill_flops()
+    value = pf * K * world / (p_ms * 1e-3) / 1e12
+    dec_gbs = lay.decode_bytes() * K * world / (d_ms * 1e-3) / 1e9
+    cmp_gbs = lay.compact_bytes() * K * world / (c_ms * 1e-3) / 1e9
+    e2e_val = pf * K * world / (e2e_ms * 1e-3) / 1e12
+    prof = _traffic()
+    achieved = pf / (p_ms / K * 1e-3) / 1e12
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": K, "warmup": args.warmup, "ms_per_step": round(total_ms / K, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V/Q; dialogue shapes drawn from the workload recipe)",
+        "config": {"workload": WORKLOAD, "n_layers": lay.NL, "heads_q": lay.HQ,
+                   "heads_kv": lay.HKV, "head_dim": lay.D, "prefill_seqs": lay.n_pre,
+                   "prefill_query_rows": lay.T_q, "decode_seqs": lay.n_dec,
+                   "decode_retained_rows": int(lay.dec_len.sum()),
+                   "raw_history_rows": lay.raw.total, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (decode reads %.1f GB/step)" % (
+                       lay.decode_bytes() / 1e9),
+                   "value_basis": "prefill flops / prefill launch time"},
+        "decode": {"value": round(dec_gbs, 1), "unit": "GB/s",
+                   "ms_per_step": round(d_ms / K, 3),
+                   "roofline": {"bound": "hbm", "achieved": round(dec_gbs / world, 1),
+                                "peak": pk["hbm"], "unit": "GB/s",
+                                "frac": round(dec_gbs / world / pk["hbm"], 4),
+                                "traffic": prof.get("decode")}},
+        "compaction": {"value": round(cmp_gbs, 1), "unit": "GB/s",
+                       "ms_per_step": round(c_ms / K, 3),
+                       "roofline": {"bound": "hbm", "achieved": round(cmp_gbs / world, 1),
+                                    "peak": pk["hbm"], "unit": "GB/s",
+                                    "frac": round(cmp_gbs / world / pk["hbm"], 4),
+                                    "traffic": prof.get("compact")}},
+        "prefill_ms_per_step": round(p_ms / K, 3),
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 2),
+                     "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+                     "frac": round(achieved / pk["bf16_sus"], 4), "traffic": prof.get("prefill"),
+                     "peak_source": pk["source"] + " bf16 sustained"},
+        "e2e": {"value": round(e2e_val, 2), "unit": "TFLOP/s",
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                "ms_per_step": round(e2e_ms / K, 3)},
+        "gpu_launches": g.launches_per_step * K,
+        "clocks": clk,
+    }
+    return out, lay
+
+
+def _traffic():
+    """DRAM bytes per launch from the committed ncu summary (if it matches)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return {}
+    with open(p) as f:
+        return json.load(f)
+
+
+# ---------------------------------------------------------------------------
+# Oracle arm (CPU)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(lay: Layout, n_rows: int = 48, threads: int = None):
+    """Time the oracle on a bounded sample of the step's prefill: n_rows query
+    rows of every prefill sequence (spread over the turn), all 28 heads,
+    layer 0.  Returns (TFLOP/s, seconds, cores, description)."""
+    import oracle
+    from concurrent.futures import ThreadPoolExecutor
+    rng = np.random.default_rng(5)
+    orc = oracle.default()
+    threads = threads or os.cpu_count() or 1
+    jobs = []
+    flops = 0.0
+    for b in range(lay.n_pre):
+        R = int(lay.ret_pre[b])
+        L = R + int(lay.q_len[b])
+        K = rng.standard_normal((L, lay.HKV, lay.D))
+        V = rng.standard_normal((L, lay.HKV, lay.D))
+        role = lay.role_ret[lay.k_start_pre[b]:lay.k_start_pre[b] + L]
+        seg = lay.seg_ret[lay.k_start_pre[b]:lay.k_start_pre[b] + L]
+        rows = np.linspace(R, L - 1, n_rows).astype(np.int64)
+        for r in rows:
+            Q = rng.standard_normal((1, lay.HQ, lay.D))
+            jobs.append((Q, K, V, role, seg, np.array([r])))
+            flops += 4.0 * lay.D * lay.HQ * (r + 1)
+    t0 = time.perf_counter()
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(lambda j: orc.attn_masked(*j), jobs))
+    dt = time.perf_counter() - t0
+    desc = (f"oracle masked attention, {len(jobs)} query rows ({n_rows} per prefill sequence) "
+            f"x {lay.HQ} heads, layer 0, float64, {threads} threads")
+    return flops / dt / 1e12, dt, threads, desc
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="sonic", choices=["sonic", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        lay = Layout()
+        per_step, vals = [], []
+        for i in range(args.warmup + args.steps):
+            v, dt, cores, desc = oracle_sample(lay)
+            if i >= args.warmup:
+                per_step.append(dt)
+                vals.append(v)
+        value = float(np.mean(vals))
+        out = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+               "steps": args.steps, "warmup": args.warmup,
+               "ms_per_step": round(1e3 * float(np.mean(per_step)), 1),
+               "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+               "dtype": "f64", "data": "synthetic", "impl": "reference",
+               "config": {"workload": WORKLOAD, "sample": desc},
+               "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores,
+                                "kind": "oracle", "sample": desc},
+               "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                       "d2h_bytes_per_step": 0}}
+        print(json.dumps(out))
+        return
+
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    out, lay = run_gpu(args, rank, world)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, dt, cores, desc = oracle_sample(lay)
+        out["cpu_baseline"] = {"value": v, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                               "sample": desc, "seconds": round(dt, 2)}
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()
