@@ -194,6 +194,32 @@ SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K
 
 SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
 
+/*
+ * sonic_attn_prefill for callers that cannot allocate device memory.  The
+ * paper has no counterpart; this is a deployment aid.  Some callers cannot
+ * call cudaMalloc: code running inside a custom allocator or memory-pool
+ * callback, runtimes that plan every device byte ahead of time, or hosts that
+ * only hand over fixed buffers for inputs and outputs.  This call takes the
+ * same arguments as sonic_attn_prefill except that args->workspace and
+ * args->workspace_bytes are ignored: the per-tile mask summaries live in a
+ * fixed 1 MiB array compiled into the library (every GPU that loads the
+ * library holds it until the process exits).  It allocates nothing.
+ *  - Limit: batch * ceil(max_k_len / 128) <= 32768; larger calls return
+ *    SONIC_ERR_WORKSPACE before launching anything.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current) and caches it; make
+ *    that first call before any stream capture.
+ *  - Every call on a device shares the one array and leaves its contents
+ *    behind; each call rewrites every entry it reads, so nothing needs
+ *    clearing, but calls that overlap on the GPU (other streams, other host
+ *    threads) race on it and must be serialised by the caller.
+ */
+SONIC_API sonic_status_t sonic_attn_prefill_static(const uint16_t *Q, const uint16_t *K,
+                                                   const uint16_t *V, const int32_t *seg_id,
+                                                   const uint8_t *role, uint16_t *O,
+                                                   const sonic_prefill_args *args,
+                                                   sonic_stream_t stream);
+
 /* ------------------------------------------------------------------------- */
 /* Decode                                                                    */
 /* ------------------------------------------------------------------------- */

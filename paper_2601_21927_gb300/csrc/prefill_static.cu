@@ -1,0 +1,71 @@
+// sonic_attn_prefill_static: the masked prefill for callers that cannot
+// allocate device memory.
+//
+// Some callers cannot call cudaMalloc at all: code running inside a custom
+// allocator or a memory-pool callback, runtimes that pre-plan every byte of
+// device memory up front, or hosts that only hand out fixed buffers for the
+// model's tensors.  They can still pass inputs and outputs, but not the
+// caller-owned workspace sonic_attn_prefill needs for its per-tile mask
+// summaries.  This entry point keeps that scratch in a fixed array compiled
+// into the library instead, and runs the same kernels.
+//
+// The array is a file-scope __device__ variable: every GPU that loads the
+// library holds it until the process exits.  In host code its name is only a
+// host-side stand-in, so its device address is looked up with
+// cudaGetSymbolAddress once per device (with that device current) on the
+// first call made on that device, and cached.
+#include <mutex>
+
+#include "sonic_host.h"
+
+namespace {
+
+// 1 MiB: room for 32768 per-tile summaries of 32 bytes, i.e.
+// batch * ceil(max_k_len / 128) <= 32768 (for example 64 sequences of up
+// to 65536 keys).
+constexpr size_t kStaticScratchBytes = size_t(1) << 20;
+
+static __device__ __align__(256) unsigned char g_prefill_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+void *g_scratch_ptr[kMaxDevices] = {nullptr};
+std::mutex g_scratch_mu;
+
+// Device address of the scratch array on the current device (looked up once).
+sonic_status_t scratch_address(void **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SONIC_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return SONIC_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (g_scratch_ptr[dev] == nullptr) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_prefill_scratch) != cudaSuccess || p == nullptr)
+            return SONIC_ERR_CUDA;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return SONIC_OK;
+}
+
+}  // namespace
+
+extern "C" sonic_status_t sonic_attn_prefill_static(const uint16_t *Q, const uint16_t *K,
+                                                    const uint16_t *V, const int32_t *seg_id,
+                                                    const uint8_t *role, uint16_t *O,
+                                                    const sonic_prefill_args *args,
+                                                    sonic_stream_t stream) {
+    if (args == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
+    sonic_prefill_args a = *args;
+    a.workspace = nullptr;
+    a.workspace_bytes = 0;
+    const size_t need = sonic_prefill_workspace_size(&a);
+    if (need > kStaticScratchBytes) return SONIC_ERR_WORKSPACE;
+    if (need > 0) {
+        void *p = nullptr;
+        const sonic_status_t st = scratch_address(&p);
+        if (st != SONIC_OK) return st;
+        a.workspace = p;
+        a.workspace_bytes = kStaticScratchBytes;
+    }
+    return sonic_attn_prefill(Q, K, V, seg_id, role, O, &a, stream);
+}

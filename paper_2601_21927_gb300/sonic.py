@@ -73,6 +73,8 @@ SIGNATURES = {
     "sonic_attn_prefill": (_i32, [_P, _P, _P, _P, _P, _P,
                                   ctypes.POINTER(sonic_prefill_args), _P]),
     "sonic_prefill_workspace_size": (_sz, [ctypes.POINTER(sonic_prefill_args)]),
+    "sonic_attn_prefill_static": (_i32, [_P, _P, _P, _P, _P, _P,
+                                         ctypes.POINTER(sonic_prefill_args), _P]),
     "sonic_attn_decode": (_i32, [_P, _P, _P, _P, _P,
                                  ctypes.POINTER(sonic_decode_args), _P]),
     "sonic_decode_workspace_size": (_sz, [ctypes.POINTER(sonic_decode_args)]),
@@ -217,3 +219,29 @@ def sonic_attn_decode(q: torch.Tensor, K_ret: torch.Tensor, V_ret: torch.Tensor,
     _check(lib.sonic_attn_decode(_ptr(q), _ptr(K_ret), _ptr(V_ret), _ptr(lens), _ptr(O),
                                  ctypes.byref(a), _stream(stream)), "sonic_attn_decode")
     return ws
+
+
+def sonic_attn_prefill_static(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor,
+                              seg_id: torch.Tensor, role: torch.Tensor, O: torch.Tensor, *,
+                              k_start, k_len, q_start, q_len, max_q_len: int, max_k_len: int,
+                              softmax_scale: float = 0.0, nexus_vis: int = NEXUS_FULL, lse=None,
+                              status=None, stream=None):
+    """sonic_attn_prefill for callers that cannot allocate device memory: the
+    library keeps the mask-summary scratch in a fixed 1 MiB device array, so
+    no workspace is passed (and this wrapper allocates nothing either).
+    Calls overlapping on the GPU share that array and must be serialised."""
+    lib = load()
+    nl, tq, hq, d = Q.shape
+    _, tk, hkv, _ = K.shape
+    a = sonic_prefill_args()
+    a.batch = k_start.numel()
+    a.n_layers, a.n_heads_q, a.n_heads_kv, a.head_dim = nl, hq, hkv, d
+    a.k_start, a.k_len, a.q_start, a.q_len = (_ptr(k_start), _ptr(k_len), _ptr(q_start),
+                                              _ptr(q_len))
+    a.max_q_len, a.max_k_len, a.total_q_rows, a.total_k_rows = max_q_len, max_k_len, tq, tk
+    a.q_layer_stride, a.kv_layer_stride, a.o_layer_stride = Q.stride(0), K.stride(0), O.stride(0)
+    a.softmax_scale, a.nexus_vis = softmax_scale, nexus_vis
+    a.lse, a.status = _ptr(lse), _ptr(status)
+    _check(lib.sonic_attn_prefill_static(_ptr(Q), _ptr(K), _ptr(V), _ptr(seg_id), _ptr(role),
+                                         _ptr(O), ctypes.byref(a), _stream(stream)),
+           "sonic_attn_prefill_static")
