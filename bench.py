@@ -62,11 +62,13 @@ def _peaks():
 # ---------------------------------------------------------------------------
 
 class Layout:
-    def __init__(self, seed: int = 1):
+    def __init__(self, seed: int = 1, n_layers: int = 0):
         from paper_2601_21927_gb300 import inputs
         self.ms = ms = inputs.mixed_serving(seed=seed)
         h = ms.heads
         self.NL, self.HQ, self.HKV, self.D = h.n_layers, h.hq, h.hkv, h.d
+        if n_layers > 0:
+            self.NL = n_layers
         self.row_bytes = self.HKV * self.D * 2
         # raw histories of the prefill sequences (packed)
         self.raw = inputs.Batch(ms.raw_hist)
@@ -242,10 +244,29 @@ def run_gpu(args, rank: int, world: int):
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
     sonic.load()
-    lay = Layout()
+    lay = Layout(n_layers=args.layers)
     g = GpuStep(lay, device, seed=17 * rank)
     stream = torch.cuda.Stream(device)
     torch.cuda.synchronize()
+    if args.only:
+        # one phase alone (small captures for the profiler)
+        fn = {"compact": g.compact, "prefill": g.prefill, "decode": g.decode}[args.only]
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                fn(stream)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(args.steps):
+                fn(stream)
+            b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / max(args.steps, 1)
+        work = {"compact": lay.compact_bytes(), "prefill": lay.prefill_flops(),
+                "decode": lay.decode_bytes()}[args.only]
+        rate = work / (ms * 1e-3) / (1e12 if args.only == "prefill" else 1e9)
+        return {"only": args.only, "n_layers": lay.NL, "ms_per_launch": round(ms, 4),
+                "rate": round(rate, 2), "unit": "TFLOP/s" if args.only == "prefill" else "GB/s",
+                "status": sonic.read_status(g.status)}, lay
 
     def barrier():
         if world > 1:
@@ -392,7 +413,7 @@ def _traffic():
 # Oracle arm (CPU)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(lay: Layout, n_rows: int = 48, threads: int = None):
+def oracle_sample(lay: Layout, n_rows: int = 512, threads: int = None):
     """Time the oracle on a bounded sample of the step's prefill: n_rows query
     rows of every prefill sequence (spread over the turn), all 28 heads,
     layer 0.  Returns (TFLOP/s, seconds, cores, description)."""
@@ -431,6 +452,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="sonic", choices=["sonic", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only", choices=["compact", "prefill", "decode"], default=None,
+                    help="time one phase alone (for profiler captures)")
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -463,7 +487,7 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl")
     out, lay = run_gpu(args, rank, world)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.only:
         v, dt, cores, desc = oracle_sample(lay)
         out["cpu_baseline"] = {"value": v, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                                "sample": desc, "seconds": round(dt, 2)}
