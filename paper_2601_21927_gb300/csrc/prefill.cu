@@ -28,7 +28,7 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kPfThreads = 192;
+constexpr int kPfThreads = 384;
 constexpr int kMaxKTiles = 2048;
 constexpr float kLn2f = 0.6931471805599453f;
 constexpr float kLog2ef = 1.4426950408889634f;
@@ -126,20 +126,18 @@ struct PfParams {
 template <int D>
 struct PfCfg {
     static constexpr int kHalves = D / 64;
-    static constexpr int kQBytes = kBM * D * 2;
+    static constexpr int kQBytes = kBM * D * 2;  // one 128-row Q tile
     static constexpr int kKVBytes = kBN * D * 2;
-    static constexpr int kPBytes = kBM * kBN * 2;
-    static constexpr int kOffQ = 0;
-    static constexpr int kOffK = kOffQ + kQBytes;
-    static constexpr int kOffV = kOffK + 2 * kKVBytes;
-    static constexpr int kOffP = kOffV + 2 * kKVBytes;
-    static constexpr int kOffRole = kOffP + kPBytes;       // [2][128] uint8
-    static constexpr int kOffSeg = kOffRole + 2 * kBN;     // [2][128] int32
-    static constexpr int kOffList = kOffSeg + 2 * kBN * 4;  // [kMaxKTiles] int32
+    static constexpr int kOffQ = 0;                           // [2] Q tiles
+    static constexpr int kOffK = kOffQ + 2 * kQBytes;         // [2] stages
+    static constexpr int kOffV = kOffK + 2 * kKVBytes;        // [2] stages
+    static constexpr int kOffRole = kOffV + 2 * kKVBytes;     // [2][128] uint8
+    static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
+    static constexpr int kOffList = kOffSeg + 2 * kBN * 4;    // [kMaxKTiles] int32
     static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
-    static constexpr int kNumBars = 12;
-    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // 16 ints
-    static constexpr int kBytes = kOffMisc + 16 * 4;
+    static constexpr int kNumBars = 16;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 32 ints
+    static constexpr int kBytes = kOffMisc + 32 * 4;
     static constexpr size_t kSmem = 1024 + kBytes;
 };
 
@@ -151,6 +149,19 @@ __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, in
     return q <= p;                                                          // Eq. 3
 }
 
+// Largest rise of the running row maximum (base 2) absorbed without
+// rescaling O: probabilities stay below 2^8 until the next rescale.
+constexpr float kRescaleThreshold = 8.0f;
+
+// Two 128-row query tiles (tile 0 = rows 0..127 of the block's 256, tile 1 =
+// rows 128..255) share every K/V tile.  Warp roles:
+//   warp 0       TMA producer (K, V, Q) and key metadata,
+//   warp 1       tcgen05 issuer and TMEM owner,
+//   warps 2-3    idle after set-up,
+//   warps 4-7    softmax of tile 0, warps 8-11 softmax of tile 1.
+// TMEM (512 columns): S/P of tile 0 at 0, of tile 1 at 128, O of tile 0 at
+// 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns
+// of its S block and feeds O += P V straight from tensor memory.
 template <int D>
 __global__ void __launch_bounds__(kPfThreads, 1)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -162,7 +173,6 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint8_t *Qs = smem + C::kOffQ;
     uint8_t *Ks = smem + C::kOffK;
     uint8_t *Vs = smem + C::kOffV;
-    uint8_t *Ps = smem + C::kOffP;
     uint8_t *meta_role = smem + C::kOffRole;
     int32_t *meta_seg = reinterpret_cast<int32_t *>(smem + C::kOffSeg);
     int32_t *list = reinterpret_cast<int32_t *>(smem + C::kOffList);
@@ -170,20 +180,19 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint64_t *q_full = bars + 0;
     uint64_t *kv_full = bars + 1;   // [2]
     uint64_t *kv_empty = bars + 3;  // [2]
-    uint64_t *s_full = bars + 5;    // [2]
-    uint64_t *s_free = bars + 7;    // [2]
-    uint64_t *p_full = bars + 9;
-    uint64_t *o_done = bars + 10;
+    uint64_t *s_full = bars + 5;    // [2] per query tile
+    uint64_t *p_full = bars + 7;    // [2] per query tile
+    uint64_t *o_done = bars + 9;    // [2] per query tile
     uint64_t *mma_idle = bars + 11;
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
-    // misc: 0 tmem base, 1 list length, 2 abort, 3 q flags, 4 q seg min, 5 q seg max,
-    //       6 q nexus seg min, 7 q nexus seg max, 8..15 warp counts
+    // misc: 0 tmem base, 2 abort, 4..13 query-tile summaries (5 per tile),
+    //       16..27 per-warp counts
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
 
     const int qt = blockIdx.x, h = blockIdx.y;
     const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
     const int klen = p.k_len[b], qlen = p.q_len[b];
-    if (qt * kBM >= qlen || timed_out(p.status)) return;
+    if (qt * 2 * kBM >= qlen || timed_out(p.status)) return;
     if (qlen > klen || klen > p.max_k_tiles * kBN) {
         // the host-side bounds were wrong for this sequence: refuse it
         if (threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
@@ -191,71 +200,70 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
     const int kstart = p.k_start[b];
     const int kvh = h / p.G;
-    const int p0 = klen - qlen + qt * kBM;          // position of query row 0
-    const int p1 = min(p0 + kBM - 1, klen - 1);     // last valid query position
+    const int pbase = klen - qlen + qt * 2 * kBM;  // position of query row 0 of tile 0
+    const bool tile1 = qt * 2 * kBM + kBM < qlen;   // tile 1 has rows
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-    // ------------------------------------------------ summary of the query tile
-    if (tid == 0) {
-        misc[2] = 0;
-        misc[3] = 0;
-        misc[4] = INT_MAX;
-        misc[5] = INT_MIN;
-        misc[6] = INT_MAX;
-        misc[7] = INT_MIN;
-    }
+    // ------------------------------------------------ summaries of the query tiles
+    if (tid < 10) misc[4 + tid] = (tid % 5 == 0) ? 0 : ((tid % 5) & 1 ? INT_MAX : INT_MIN);
     __syncthreads();
-    if (tid < kBM && p0 + tid <= p1) {
-        const int ro = p.role[kstart + p0 + tid];
-        const int s = p.seg[kstart + p0 + tid];
-        atomicMin(&misc[4], s);
-        atomicMax(&misc[5], s);
+    if (tid < 2 * kBM && pbase + tid <= klen - 1) {
+        int32_t *qs = misc + 4 + 5 * (tid >> 7);  // flags, seg min, seg max, nexus min, nexus max
+        const int ro = p.role[kstart + pbase + tid];
+        const int s = p.seg[kstart + pbase + tid];
+        atomicMin(&qs[1], s);
+        atomicMax(&qs[2], s);
         if (ro == SONIC_ROLE_NEXUS) {
-            atomicOr(&misc[3], 2);
-            atomicMin(&misc[6], s);
-            atomicMax(&misc[7], s);
+            atomicOr(&qs[0], 2);
+            atomicMin(&qs[3], s);
+            atomicMax(&qs[4], s);
         }
     }
     __syncthreads();
-    const int q_has_nexus = misc[3] & 2;
-    const int qs_min = misc[4], qs_max = misc[5], qn_min = misc[6], qn_max = misc[7];
 
-    // ------------------------------------------------ list of key tiles to visit
+    // ------------------------------------------------ key tiles to visit
+    // list entry: (tile << 2) | (tile 0 needs the mask) | (tile 1 needs it) << 1
     const int n_kt = (klen + kBN - 1) / kBN;
     int n_list = 0;
     for (int c0 = 0; c0 < n_kt; c0 += kPfThreads) {
         const int t = c0 + tid;
-        int code = 0;  // 0 hidden, 1 fully visible, 2 cut by the mask
+        int entry = 0;
+        bool keep = false;
         if (t < n_kt) {
             const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
             const int k0 = t * kBN, k1 = k0 + ts.n_rows - 1;
             const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
-            const bool causal_part = (k0 <= p1) && (kn || ko);
-            const bool body_part =
-                kb && (k0 <= p1) && !(ts.bseg_max < qs_min || ts.bseg_min > qs_max);
-            const bool nexus_part = kn && q_has_nexus &&
-                                    (p.nexus_mode == SONIC_NEXUS_FULL || ts.nseg_min <= qn_max);
-            if (causal_part || body_part || nexus_part) {
+            for (int qi = 0; qi < 2; ++qi) {
+                const int p0 = pbase + qi * kBM;
+                const int p1 = min(p0 + kBM - 1, klen - 1);
+                if (p0 > p1) continue;
+                const int *qs = misc + 4 + 5 * qi;
+                const bool q_has_nexus = qs[0] & 2;
+                const bool causal_part = (k0 <= p1) && (kn || ko);
+                const bool body_part =
+                    kb && (k0 <= p1) && !(ts.bseg_max < qs[1] || ts.bseg_min > qs[2]);
+                const bool nexus_part =
+                    kn && q_has_nexus &&
+                    (p.nexus_mode == SONIC_NEXUS_FULL || ts.nseg_min <= qs[4]);
+                const bool any = causal_part || body_part || nexus_part;
                 const bool full =
-                    ts.n_rows == kBN && k1 <= p0 &&
-                    (!kb || (ts.bseg_min == ts.bseg_max && qs_min == qs_max &&
-                             ts.bseg_min == qs_min)) &&
+                    any && ts.n_rows == kBN && k1 <= p0 &&
+                    (!kb || (ts.bseg_min == ts.bseg_max && qs[1] == qs[2] &&
+                             ts.bseg_min == qs[1])) &&
                     (p.nexus_mode == SONIC_NEXUS_FULL || !(kn && q_has_nexus) ||
-                     ts.nseg_max <= qn_min);
-                code = full ? 1 : 2;
+                     ts.nseg_max <= qs[3]);
+                keep |= any;
+                if (!full) entry |= 1 << qi;
             }
         }
-        const unsigned bal = __ballot_sync(0xffffffffu, code != 0);
-        if (lane == 0) misc[8 + warp] = __popc(bal);
+        const unsigned bal = __ballot_sync(0xffffffffu, keep);
+        if (lane == 0) misc[16 + warp] = __popc(bal);
         __syncthreads();
         int base = n_list;
-        for (int w = 0; w < warp; ++w) base += misc[8 + w];
+        for (int w = 0; w < warp; ++w) base += misc[16 + w];
         int tot = 0;
-        for (int w = 0; w < kPfThreads / 32; ++w) tot += misc[8 + w];
-        if (code != 0) {
-            const int rank = __popc(bal & ((1u << lane) - 1u));
-            list[base + rank] = (t << 1) | (code == 2 ? 1 : 0);
-        }
+        for (int w = 0; w < kPfThreads / 32; ++w) tot += misc[16 + w];
+        if (keep) list[base + __popc(bal & ((1u << lane) - 1u))] = (t << 2) | entry;
         n_list += tot;
         __syncthreads();
     }
@@ -267,11 +275,11 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             mbar_init(&kv_full[s], 32);
             mbar_init(&kv_empty[s], 1);
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], kBM);
+            mbar_init(&p_full[s], kBM);
+            mbar_init(&o_done[s], 1);
         }
-        mbar_init(p_full, kBM);
-        mbar_init(o_done, 1);
         mbar_init(mma_idle, 1);
+        *abort_flag = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -282,7 +290,6 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
-    const uint32_t tmem_S0 = tmem, tmem_O = tmem + 256;
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -290,24 +297,24 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tma_prefetch_desc(&tmQ);
             tma_prefetch_desc(&tmK);
             tma_prefetch_desc(&tmV);
-            mbar_arrive_expect_tx(q_full, C::kQBytes);
+            mbar_arrive_expect_tx(q_full, (tile1 ? 2 : 1) * C::kQBytes);
+            for (int qi = 0; qi < (tile1 ? 2 : 1); ++qi)
 #pragma unroll
-            for (int hh = 0; hh < C::kHalves; ++hh)
-                tma_load_4d(Qs + hh * (kBM * 128), &tmQ, q_full, hh * 64, h,
-                            p.q_start[b] + qt * kBM, layer);
+                for (int hh = 0; hh < C::kHalves; ++hh)
+                    tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full, hh * 64,
+                                h, p.q_start[b] + qt * 2 * kBM + qi * kBM, layer);
         }
         int i = 0;
         for (; i < n_list; ++i) {
             const int st = i & 1;
             if (i >= 2 && !mbar_wait(&kv_empty[st], ((i >> 1) - 1) & 1, p.status, abort_flag))
                 break;
-            const int kt = list[i] >> 1;
-            // role / segment numbers of the tile's keys (255 marks rows past the sequence)
+            const int kt = list[i] >> 2;
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int c = lane * 4 + u;
                 const int q = kt * kBN + c;
-                uint8_t ro = 255;
+                uint8_t ro = 255;  // rows past the sequence
                 int32_t sg = 0;
                 if (q < klen) {
                     ro = p.role[kstart + q];
@@ -341,138 +348,167 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, 0);
             constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, 1);
-            const uint32_t q_addr = smem_u32(Qs), k_addr = smem_u32(Ks), v_addr = smem_u32(Vs),
-                           p_addr = smem_u32(Ps);
-            bool ok = mbar_wait(q_full, 0, p.status, abort_flag);
-            auto issue_pv = [&](int j) -> bool {
-                if (!mbar_wait(p_full, j & 1, p.status, abort_flag)) return false;
-                tc_fence_after();
-                const int st = j & 1;
-#pragma unroll
-                for (int kk = 0; kk < kBN / 16; ++kk) {
-                    const uint64_t a = smem_desc_sw128(
-                        p_addr + (kk >> 2) * (kBM * 128) + (kk & 3) * 32, 16, 1024);
-                    const uint64_t bd =
-                        smem_desc_sw128(v_addr + st * C::kKVBytes + kk * (16 * 128),
-                                        kBN * 128, 1024);
-                    tc_mma_ss(tmem_O, a, bd, idPV, (j > 0 || kk > 0) ? 1u : 0u);
-                }
-                tc_commit(o_done);
-                tc_commit(&kv_empty[st]);
-                return true;
-            };
-            for (int i = 0; ok && i < n_list; ++i) {
-                const int st = i & 1, sb = i & 1;
-                if (!mbar_wait(&kv_full[st], (i >> 1) & 1, p.status, abort_flag)) break;
-                if (i >= 2 && !mbar_wait(&s_free[sb], ((i >> 1) - 1) & 1, p.status, abort_flag))
-                    break;
-                tc_fence_after();
+            const uint32_t q_addr = smem_u32(Qs), k_addr = smem_u32(Ks), v_addr = smem_u32(Vs);
+            const int nq = tile1 ? 2 : 1;
+            auto issue_s = [&](int qi, int st) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
-                    const uint64_t a = smem_desc_sw128(q_addr + off, 16, 1024);
+                    const uint64_t a = smem_desc_sw128(q_addr + qi * C::kQBytes + off, 16, 1024);
                     const uint64_t bd = smem_desc_sw128(k_addr + st * C::kKVBytes + off, 16, 1024);
-                    tc_mma_ss(tmem_S0 + sb * kBN, a, bd, idS, kk > 0 ? 1u : 0u);
+                    tc_mma_ss(tmem + qi * kBN, a, bd, idS, kk > 0 ? 1u : 0u);
                 }
-                tc_commit(&s_full[sb]);
-                if (i >= 1 && !issue_pv(i - 1)) break;
-                if (i == n_list - 1) issue_pv(i);
+                tc_commit(&s_full[qi]);
+            };
+            auto issue_pv = [&](int qi, int st, int j) {
+#pragma unroll
+                for (int kk = 0; kk < kBN / 16; ++kk) {
+                    const uint64_t bd = smem_desc_sw128(v_addr + st * C::kKVBytes + kk * (16 * 128),
+                                                        kBN * 128, 1024);
+                    tc_mma_ts(tmem + 256 + qi * 128, tmem + qi * kBN + kk * 8, bd, idPV,
+                              (j > 0 || kk > 0) ? 1u : 0u);
+                }
+            };
+            bool ok = mbar_wait(q_full, 0, p.status, abort_flag) && n_list > 0 &&
+                      mbar_wait(&kv_full[0], 0, p.status, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                for (int qi = 0; qi < nq; ++qi) issue_s(qi, 0);
             }
-            // all MMAs issued by this thread have finished once this arrives
+            for (int j = 0; ok && j < n_list; ++j) {
+                const int st = j & 1, nst = (j + 1) & 1;
+                const bool more = j + 1 < n_list;
+                for (int qi = 0; qi < nq; ++qi) {
+                    if (!mbar_wait(&p_full[qi], j & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    issue_pv(qi, st, j);
+                    if (!more) tc_commit(&o_done[qi]);
+                    if (qi == nq - 1) tc_commit(&kv_empty[st]);
+                    if (more) {
+                        if (qi == 0 &&
+                            !mbar_wait(&kv_full[nst], ((j + 1) >> 1) & 1, p.status, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        issue_s(qi, nst);
+                    }
+                }
+            }
+            // every MMA issued by this thread has finished once this arrives
             tc_commit(mma_idle);
             mbar_wait(mma_idle, 0, p.status, abort_flag);
         }
-    } else {
+    } else if (warp >= 4 && (warp < 8 || tile1)) {
         // ------------------------------------------------------------ softmax
+        const int qi = (warp - 4) >> 2;
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
-        const int pos = p0 + r;
-        const bool row_ok = pos <= p1;
+        const int pos = pbase + qi * kBM + r;
+        const bool row_ok = pos <= klen - 1 && qt * 2 * kBM + qi * kBM + r < qlen;
         int rp = SONIC_ROLE_SYS, sp = 0;
         if (row_ok) {
             rp = p.role[kstart + pos];
             sp = p.seg[kstart + pos];
         }
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-        float m = -INFINITY, l = 0.f;
+        const uint32_t tS = tmem + lane_base + qi * kBN;
+        const uint32_t tO = tmem + lane_base + 256 + qi * 128;
+        float m_used = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int i = 0; i < n_list; ++i) {
-            const int sb = i & 1, st = i & 1;
-            if (!mbar_wait(&kv_full[st], (i >> 1) & 1, p.status, abort_flag) ||
-                !mbar_wait(&s_full[sb], (i >> 1) & 1, p.status, abort_flag)) {
+        for (int j = 0; j < n_list; ++j) {
+            const int st = j & 1;
+            if (!mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag) ||
+                !mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            uint32_t sr[4][32];
+            const int kt = list[j] >> 2;
+            const bool cut = (list[j] >> qi) & 1;
+            // pass 1: row maximum (and the mask bits of a cut tile)
+            uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
+            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_base + sb * kBN + c * 32, sr[c]);
-            tmem_ld_wait();
-#pragma unroll
-            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
-            tc_fence_before();
-            mbar_arrive(&s_free[sb]);
-
-            const int kt = list[i] >> 1;
-            const bool cut = list[i] & 1;
-            float s[kBN];
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                    s[c * 32 + e] = __uint_as_float(sr[c][e]) * p.scale_log2;
-            if (cut) {
-                const uint8_t *mr = meta_role + st * kBN;
-                const int32_t *ms = meta_seg + st * kBN;
-#pragma unroll
-                for (int c = 0; c < kBN; ++c) {
-                    const int rq = mr[c];
-                    const bool v = rq != 255 &&
-                                   visible(pos, kt * kBN + c, rp, sp, rq, ms[c], p.nexus_mode);
-                    if (!v) s[c] = -INFINITY;
-                }
-            }
-            float mx = m;
-#pragma unroll
-            for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
-            const float mu = (mx == -INFINITY) ? 0.f : mx;
-            const float alpha = ex2(m - mu);
-            float rs = 0.f;
-            uint32_t pk[kBN / 2];
-#pragma unroll
-            for (int c = 0; c < kBN; c += 2) {
-                const float e0 = ex2(s[c] - mu), e1 = ex2(s[c + 1] - mu);
-                rs += e0 + e1;
-                pk[c >> 1] = pack_bf16x2(e0, e1);
-            }
-            l = l * alpha + rs;
-            m = mx;
-
-            // PV(i-1) must be done: P buffer free, O up to date.
-            if (i >= 1) {
-                if (!mbar_wait(o_done, (i - 1) & 1, p.status, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                if (__any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        uint32_t o[32];
-                        tmem_ld32(tmem_O + lane_base + c * 32, o);
-                        tmem_ld_wait();
-                        reg_fence32(o);
-#pragma unroll
-                        for (int e = 0; e < 32; ++e)
-                            o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        tmem_st32(tmem_O + lane_base + c * 32, o);
+            for (int c = 0; c < 4; ++c) {
+                uint32_t sr[32];
+                tmem_ld32(tS + c * 32, sr);
+                tmem_ld_wait();
+                reg_fence32(sr);
+                if (cut) {
+                    const uint8_t *mr = meta_role + st * kBN + c * 32;
+                    const int32_t *ms = meta_seg + st * kBN + c * 32;
+                    uint32_t bits = 0;
+#pragma unroll 4
+                    for (int e = 0; e < 32; ++e) {
+                        const int rq = mr[e];
+                        const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp, rq,
+                                                            ms[e], p.nexus_mode);
+                        bits |= (v ? 1u : 0u) << e;
                     }
-                    tmem_st_wait();
+                    mbits[c] = bits;
+                }
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const float v = ((mbits[c] >> e) & 1) ? __uint_as_float(sr[e]) : -INFINITY;
+                    mx4[e & 3] = fmaxf(mx4[e & 3], v);
                 }
             }
+            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
+            float alpha = 1.f, m_new = m_used;
+            if (j == 0) {
+                m_new = mx;
+            } else if (mx > m_used + kRescaleThreshold) {
+                m_new = mx;
+                alpha = ex2(m_used - m_new);
+            }
+            const float mref = (m_new == -INFINITY) ? 0.f : m_new;
+            // pass 2: probabilities, written as bf16 pairs over the S columns
+            float rs4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t sr[32];
+                tmem_ld32(tS + c * 32, sr);
+                tmem_ld_wait();
+                reg_fence32(sr);
+                uint32_t pk[16];
+#pragma unroll
+                for (int e = 0; e < 32; e += 2) {
+                    const float s0 = ((mbits[c] >> e) & 1)
+                                         ? fmaf(__uint_as_float(sr[e]), p.scale_log2, -mref)
+                                         : -INFINITY;
+                    const float s1 = ((mbits[c] >> (e + 1)) & 1)
+                                         ? fmaf(__uint_as_float(sr[e + 1]), p.scale_log2, -mref)
+                                         : -INFINITY;
+                    const float e0 = ex2(s0), e1 = ex2(s1);
+                    rs4[(e >> 1) & 3] += e0 + e1;
+                    pk[e >> 1] = pack_bf16x2(e0, e1);
+                }
+                tmem_st16(tS + c * 16, pk);
+            }
+            l = l * alpha + ((rs4[0] + rs4[1]) + (rs4[2] + rs4[3]));
+            // O rescale (PV of the previous tile is complete: S of this tile was
+            // issued after it, and S is done)
+            if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(tO + c * 32, o);
+                    tmem_ld_wait();
+                    reg_fence32(o);
+#pragma unroll
+                    for (int e = 0; e < 32; ++e)
+                        o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                    tmem_st32(tO + c * 32, o);
+                }
+            }
+            tmem_st_wait();
             // Rows of V past the sequence end: zero them so 0 * garbage cannot
-            // reach the accumulator.
-            if (kt * kBN + kBN > klen && kt * kBN + r >= klen) {
+            // reach the accumulator (tile 0's warps; its PV is issued first).
+            if (qi == 0 && kt * kBN + kBN > klen && kt * kBN + r >= klen) {
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh) {
                     uint4 *vr = reinterpret_cast<uint4 *>(Vs + st * C::kKVBytes +
@@ -480,30 +516,22 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                     for (int u = 0; u < 8; ++u) vr[u] = make_uint4(0, 0, 0, 0);
                 }
+                fence_proxy_async_smem();
             }
-            // P row r, K-major, 128-byte swizzle: 16-byte piece j of 64-key block
-            // blk lands at blk * 16 KB + r * 128 + ((j ^ (r & 7)) * 16).
-#pragma unroll
-            for (int cc = 0; cc < kBN / 8; ++cc) {
-                const int blk = cc >> 3, j = cc & 7;
-                uint4 *dst = reinterpret_cast<uint4 *>(Ps + blk * (kBM * 128) + r * 128 +
-                                                       ((j ^ (r & 7)) << 4));
-                *dst = make_uint4(pk[cc * 4 + 0], pk[cc * 4 + 1], pk[cc * 4 + 2], pk[cc * 4 + 3]);
-            }
-            fence_proxy_async_smem();
             tc_fence_before();
-            mbar_arrive(p_full);
+            mbar_arrive(&p_full[qi]);
+            m_used = m_new;
         }
         // ------------------------------------------------------------ epilogue
-        if (ok && n_list > 0 && mbar_wait(o_done, (n_list - 1) & 1, p.status, abort_flag)) {
+        if (ok && n_list > 0 && mbar_wait(&o_done[qi], 0, p.status, abort_flag)) {
             tc_fence_after();
             const float inv = l > 0.f ? 1.f / l : 0.f;
-            uint16_t *orow = p.O + layer * p.o_ls +
-                             ((int64_t)(p.q_start[b] + qt * kBM + r) * p.Hq + h) * D;
+            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
+            uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
-                tmem_ld32(tmem_O + lane_base + c * 32, o);
+                tmem_ld32(tO + c * 32, o);
                 tmem_ld_wait();
                 reg_fence32(o);
                 if (row_ok) {
@@ -520,15 +548,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
             }
             if (row_ok && p.lse != nullptr)
-                p.lse[((int64_t)layer * p.total_q_rows + p.q_start[b] + qt * kBM + r) * p.Hq + h] =
-                    l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
+                p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] =
+                    l > 0.f ? (m_used + __log2f(l)) * kLn2f : -INFINITY;
         } else if (row_ok && n_list == 0) {
-            uint16_t *orow = p.O + layer * p.o_ls +
-                             ((int64_t)(p.q_start[b] + qt * kBM + r) * p.Hq + h) * D;
+            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
+            uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
             for (int d = 0; d < D; ++d) orow[d] = 0;
             if (p.lse != nullptr)
-                p.lse[((int64_t)layer * p.total_q_rows + p.q_start[b] + qt * kBM + r) * p.Hq + h] =
-                    -INFINITY;
+                p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = -INFINITY;
         }
     }
     tc_fence_before();
@@ -596,7 +623,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         return SONIC_ERR_INVALID_ARGUMENT;
     const size_t need = sonic_prefill_workspace_size(a);
     if (a->workspace == nullptr || a->workspace_bytes < need) return SONIC_ERR_WORKSPACE;
-    const long long qtiles = (a->max_q_len + kBM - 1) / kBM;
+    const long long qtiles = (a->max_q_len + 2 * kBM - 1) / (2 * kBM);
     if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_q > 65535 || qtiles > 0x7fffffff)
         return SONIC_ERR_UNSUPPORTED;
 
