@@ -429,35 +429,49 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tc_fence_after();
             const int kt = list[j] >> 2;
             const bool cut = (list[j] >> qi) & 1;
-            // pass 1: row maximum (and the mask bits of a cut tile)
+            // pass 1: row maximum (and the mask bits of a cut tile), two 32-column
+            // chunks per tensor-memory round trip
             uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            float mxa = -INFINITY, mxb = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t sr[32];
-                tmem_ld32(tS + c * 32, sr);
+            for (int c2 = 0; c2 < 2; ++c2) {
+                uint32_t sa[32], sb[32];
+                tmem_ld32(tS + c2 * 64, sa);
+                tmem_ld32(tS + c2 * 64 + 32, sb);
                 tmem_ld_wait();
-                reg_fence32(sr);
-                if (cut) {
-                    const uint8_t *mr = meta_role + st * kBN + c * 32;
-                    const int32_t *ms = meta_seg + st * kBN + c * 32;
-                    uint32_t bits = 0;
-#pragma unroll 4
-                    for (int e = 0; e < 32; ++e) {
-                        const int rq = mr[e];
-                        const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp, rq,
-                                                            ms[e], p.nexus_mode);
-                        bits |= (v ? 1u : 0u) << e;
-                    }
-                    mbits[c] = bits;
-                }
+                reg_fence32(sa);
+                reg_fence32(sb);
+                if (!cut) {
 #pragma unroll
-                for (int e = 0; e < 32; ++e) {
-                    const float v = ((mbits[c] >> e) & 1) ? __uint_as_float(sr[e]) : -INFINITY;
-                    mx4[e & 3] = fmaxf(mx4[e & 3], v);
+                    for (int e = 0; e < 32; e += 2) {
+                        mxa = fmax3(mxa, __uint_as_float(sa[e]), __uint_as_float(sa[e + 1]));
+                        mxb = fmax3(mxb, __uint_as_float(sb[e]), __uint_as_float(sb[e + 1]));
+                    }
+                } else {
+#pragma unroll
+                    for (int hc = 0; hc < 2; ++hc) {
+                        const int c = c2 * 2 + hc;
+                        const uint8_t *mr = meta_role + st * kBN + c * 32;
+                        const int32_t *ms = meta_seg + st * kBN + c * 32;
+                        uint32_t bits = 0;
+#pragma unroll 4
+                        for (int e = 0; e < 32; ++e) {
+                            const int rq = mr[e];
+                            const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp,
+                                                                rq, ms[e], p.nexus_mode);
+                            bits |= (v ? 1u : 0u) << e;
+                        }
+                        mbits[c] = bits;
+                        const uint32_t *sv = hc ? sb : sa;
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) {
+                            const float v = ((bits >> e) & 1) ? __uint_as_float(sv[e]) : -INFINITY;
+                            if (hc) mxb = fmaxf(mxb, v); else mxa = fmaxf(mxa, v);
+                        }
+                    }
                 }
             }
-            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
+            const float mx = fmaxf(mxa, mxb) * p.scale_log2;
             float alpha = 1.f, m_new = m_used;
             if (j == 0) {
                 m_new = mx;
@@ -467,29 +481,42 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             }
             const float mref = (m_new == -INFINITY) ? 0.f : m_new;
             // pass 2: probabilities, written as bf16 pairs over the S columns
-            float rs4[4] = {0.f, 0.f, 0.f, 0.f};
+            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
+            const float2 nm2 = make_float2(-mref, -mref);
+            float2 rs2a = make_float2(0.f, 0.f), rs2b = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t sr[32];
-                tmem_ld32(tS + c * 32, sr);
+            for (int c2 = 0; c2 < 2; ++c2) {
+                uint32_t sa[32], sb[32];
+                tmem_ld32(tS + c2 * 64, sa);
+                tmem_ld32(tS + c2 * 64 + 32, sb);
                 tmem_ld_wait();
-                reg_fence32(sr);
-                uint32_t pk[16];
+                reg_fence32(sa);
+                reg_fence32(sb);
 #pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const float s0 = ((mbits[c] >> e) & 1)
-                                         ? fmaf(__uint_as_float(sr[e]), p.scale_log2, -mref)
-                                         : -INFINITY;
-                    const float s1 = ((mbits[c] >> (e + 1)) & 1)
-                                         ? fmaf(__uint_as_float(sr[e + 1]), p.scale_log2, -mref)
-                                         : -INFINITY;
-                    const float e0 = ex2(s0), e1 = ex2(s1);
-                    rs4[(e >> 1) & 3] += e0 + e1;
-                    pk[e >> 1] = pack_bf16x2(e0, e1);
+                for (int hc = 0; hc < 2; ++hc) {
+                    const uint32_t *sv = hc ? sb : sa;
+                    const uint32_t bits = mbits[c2 * 2 + hc];
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        float2 x = __ffma2_rn(
+                            make_float2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2,
+                            nm2);
+                        if (cut) {
+                            x.x = ((bits >> e) & 1) ? x.x : -INFINITY;
+                            x.y = ((bits >> (e + 1)) & 1) ? x.y : -INFINITY;
+                        }
+                        const float2 ev = make_float2(ex2(x.x), ex2(x.y));
+                        if ((e >> 1) & 1)
+                            rs2b = __fadd2_rn(rs2b, ev);
+                        else
+                            rs2a = __fadd2_rn(rs2a, ev);
+                        pk[e >> 1] = pack_bf16x2(ev.x, ev.y);
+                    }
+                    tmem_st16(tS + (c2 * 2 + hc) * 16, pk);
                 }
-                tmem_st16(tS + c * 16, pk);
             }
-            l = l * alpha + ((rs4[0] + rs4[1]) + (rs4[2] + rs4[3]));
+            l = l * alpha + ((rs2a.x + rs2a.y) + (rs2b.x + rs2b.y));
             // O rescale (PV of the previous tile is complete: S of this tile was
             // issued after it, and S is done)
             if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
