@@ -237,7 +237,8 @@ typedef struct {
     int64_t kv_layer_stride;     /* elements between layers of K_ret and V_ret          */
     int64_t o_layer_stride;      /* elements between layers of O                        */
     float softmax_scale;         /* 0 selects 1/sqrt(head_dim)                          */
-    int32_t chunk_len;           /* keys per split, multiple of 64; 0 = automatic       */
+    int32_t chunk_len;           /* keys per split (0 = automatic), rounded up to the key
+                                    tile: 128 keys at head_dim 128, 32 at head_dim 64   */
     float *lse;                  /* device [n_layers][B][Hq] or NULL                    */
     int32_t *status;             /* device int32 or NULL                                */
     void *workspace;             /* device, sonic_decode_workspace_size() bytes         */

@@ -7,17 +7,17 @@
 // Split-K, HBM-bound design:
 //   decode_split   one block per (key chunk, KV head, sequence, layer).  A
 //                  producer warp streams the chunk's K and V through a ring
-//                  of 64-key shared-memory stages with TMA (128-byte swizzle,
+//                  of 32-key shared-memory stages with TMA (128-byte swizzle,
 //                  so both access patterns below are bank-conflict free).
-//                  Four consumer warps take turns on the tiles; each keeps
+//                  Eight consumer warps take turns on the tiles; each keeps
 //                  its own online softmax for the G query heads that share
 //                  the KV head:
-//                    scores  lane = key (2 keys per lane), full-D dot products
+//                    scores  lane = key (32-key tiles), full-D dot products
 //                            against q in shared memory (broadcast reads),
 //                            packed fp32x2 FMAs, no cross-lane reduction;
 //                    P . V   lane = 4 (D=128) or 2 (D=64) output dims, keys
 //                            walked in order, p broadcast from shared memory.
-//                  The four warps are merged by log-sum-exp at the end; a
+//                  The warps are merged by log-sum-exp at the end; a
 //                  single-chunk sequence writes O directly, otherwise the
 //                  partial (max, sum, unnormalised accumulator) goes to the
 //                  workspace.
@@ -30,8 +30,8 @@
 namespace sonic {
 namespace {
 
-constexpr int kTileKeys = 64;
-constexpr int kConsumerWarps = 4;
+constexpr int kTileKeys = 32;
+constexpr int kConsumerWarps = 8;
 constexpr int kDecThreads = (kConsumerWarps + 1) * 32;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -41,7 +41,7 @@ struct DecCfg {
     static constexpr int kHalves = D / 64;               // 128-byte swizzle rows per key
     static constexpr int kTileBytes = kTileKeys * D * 2;  // K (or V) tile
     static constexpr int kStageBytes = 2 * kTileBytes;
-    static constexpr int kStages = (D == 128) ? 6 : 12;
+    static constexpr int kStages = (D == 128) ? 12 : 24;
     static constexpr int kChunks = D / 8;  // 16-byte pieces of one key row
     static constexpr int kDpl = D / 32;    // P.V output dims per lane
 };
@@ -75,6 +75,13 @@ __device__ __forceinline__ uint4 lds128(const uint8_t *p) {
 
 __device__ __forceinline__ float2 w2f(uint32_t w) { return make_float2(bf16lo(w), bf16hi(w)); }
 
+// Maximum of v over the 32 lanes of the warp, in one instruction.
+__device__ __forceinline__ float warp_max(float v) {
+    float r;
+    asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+    return r;
+}
+
 template <int D, int GT>
 __global__ void __launch_bounds__(kDecThreads, 1)
 decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -90,12 +97,14 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
     uint64_t *empty = full + C::kStages;
     volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + C::kStages);
 
-    const int chunk = blockIdx.x, kvh = blockIdx.y;
-    const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
+    // The KV head is the fastest grid index: the blocks reading the head slices
+    // of the same rows are launched together and share DRAM pages.
+    const int kvh = blockIdx.x % p.Hkv, chunk = blockIdx.x / p.Hkv;
+    const int b = blockIdx.y % p.B, layer = blockIdx.y / p.B;
     int len = p.lens[b];
     if (len > p.max_chunks * p.chunk_len) {
         // longer than the host-side bound: attend to the first max_len keys only
-        if (threadIdx.x == 0 && chunk == 0 && kvh == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        if (threadIdx.x == 0 && blockIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
         len = p.max_chunks * p.chunk_len;
     }
     const int key0 = chunk * p.chunk_len;
@@ -165,8 +174,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
     }
     if (warp < kConsumerWarps) {
         float *pw = p_s + warp * kTileKeys * Gp;
-        const int kA = lane, kB = lane + 32;
-        const int sw = lane & 7;  // (kA & 7) == (kB & 7)
+        const int sw = lane & 7;
         for (int t = warp; t < ntiles; t += kConsumerWarps) {
             const int s = t % C::kStages;
             if (!mbar_wait(&full[s], (t / C::kStages) & 1, p.status, abort_flag)) break;
@@ -174,55 +182,41 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
             const uint8_t *Vs = Ks + C::kTileBytes;
             const int valid = min(kTileKeys, nkeys - t * kTileKeys);
 
-            // scores: lane owns keys kA and kB
-            float2 dA[GT], dB[GT];
+            // scores: lane owns key `lane` of the tile
+            float2 dk[GT];
 #pragma unroll
-            for (int g = 0; g < GT; ++g) dA[g] = dB[g] = make_float2(0.f, 0.f);
+            for (int g = 0; g < GT; ++g) dk[g] = make_float2(0.f, 0.f);
 #pragma unroll 2
             for (int c = 0; c < C::kChunks; ++c) {
                 const int half = c >> 3, jj = c & 7;
-                const uint8_t *base = Ks + half * (kTileKeys * 128) + ((jj ^ sw) << 4);
-                const uint4 ka = lds128(base + kA * 128);
-                const uint4 kb = lds128(base + kB * 128);
-                const float2 a0 = w2f(ka.x), a1 = w2f(ka.y), a2 = w2f(ka.z), a3 = w2f(ka.w);
-                const float2 b0 = w2f(kb.x), b1 = w2f(kb.y), b2 = w2f(kb.z), b3 = w2f(kb.w);
+                const uint4 kw =
+                    lds128(Ks + half * (kTileKeys * 128) + lane * 128 + ((jj ^ sw) << 4));
+                const float2 a0 = w2f(kw.x), a1 = w2f(kw.y), a2 = w2f(kw.z), a3 = w2f(kw.w);
 #pragma unroll
                 for (int g = 0; g < GT; ++g) {
                     const float4 q0 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8);
                     const float4 q1 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8 + 4);
-                    const float2 x0 = make_float2(q0.x, q0.y), x1 = make_float2(q0.z, q0.w);
-                    const float2 x2 = make_float2(q1.x, q1.y), x3 = make_float2(q1.z, q1.w);
-                    dA[g] = __ffma2_rn(a0, x0, dA[g]);
-                    dA[g] = __ffma2_rn(a1, x1, dA[g]);
-                    dA[g] = __ffma2_rn(a2, x2, dA[g]);
-                    dA[g] = __ffma2_rn(a3, x3, dA[g]);
-                    dB[g] = __ffma2_rn(b0, x0, dB[g]);
-                    dB[g] = __ffma2_rn(b1, x1, dB[g]);
-                    dB[g] = __ffma2_rn(b2, x2, dB[g]);
-                    dB[g] = __ffma2_rn(b3, x3, dB[g]);
+                    dk[g] = __ffma2_rn(a0, make_float2(q0.x, q0.y), dk[g]);
+                    dk[g] = __ffma2_rn(a1, make_float2(q0.z, q0.w), dk[g]);
+                    dk[g] = __ffma2_rn(a2, make_float2(q1.x, q1.y), dk[g]);
+                    dk[g] = __ffma2_rn(a3, make_float2(q1.z, q1.w), dk[g]);
                 }
             }
             // online softmax (base 2), per query head
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
-                const float sA = kA < valid ? dA[g].x + dA[g].y : -INFINITY;
-                const float sB = kB < valid ? dB[g].x + dB[g].y : -INFINITY;
-                float tmax = fmaxf(sA, sB);
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1)
-                    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
-                const float mn = fmaxf(m[g], tmax);
+                const float sc = lane < valid ? dk[g].x + dk[g].y : -INFINITY;
+                const float mn = fmaxf(m[g], warp_max(sc));
                 const float alpha = ex2(m[g] - mn);
-                const float pA = ex2(sA - mn), pB = ex2(sB - mn);
-                l[g] = l[g] * alpha + pA + pB;
+                const float pr = ex2(sc - mn);
+                l[g] = l[g] * alpha + pr;
 #pragma unroll
                 for (int e = 0; e < C::kDpl / 2; ++e) {
                     acc[g][e].x *= alpha;
                     acc[g][e].y *= alpha;
                 }
                 m[g] = mn;
-                pw[kA * Gp + g] = pA;
-                pw[kB * Gp + g] = pB;
+                pw[lane * Gp + g] = pr;
             }
             __syncwarp();
             // P . V: lane owns output dims [lane * kDpl, lane * kDpl + kDpl)
@@ -272,8 +266,8 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
     if (*abort_flag) return;
 
     // ---------------------------------------------------- merge the 4 warps
-    float *macc = reinterpret_cast<float *>(smem);  // [4][GT][D] (stage memory is free now)
-    float *mml = macc + kConsumerWarps * GT * D;    // [4][GT][2]
+    float *macc = reinterpret_cast<float *>(smem);  // [warps][GT][D] (stage memory is free now)
+    float *mml = macc + kConsumerWarps * GT * D;    // [warps][GT][2]
     if (warp < kConsumerWarps) {
 #pragma unroll
         for (int g = 0; g < GT; ++g) {
@@ -315,6 +309,330 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
             }
         }
     }
+}
+
+// ---------------------------------------------------------------------------
+// Tensor-core decode (head_dim 128).  Both contractions run on tcgen05 with the
+// keys in the M dimension: S^T = K q^T (M = 128 keys of a tile, N = 16 query
+// heads padded, K = D) and O^T += V^T P^T (M = D, N = 16, K = 128 keys, V read
+// MN-major straight from the TMA stage).  Warp 0 streams K/V tiles through a
+// 3-stage ring, warp 1 issues the MMAs, warps 2-5 (thread = key = TMEM lane)
+// run a block-wide online softmax per head and write P (bf16) to shared
+// memory; a running maximum that rises by less than 2^8 does not trigger an
+// O rescale.  S^T and P are double buffered so S^T of the next tile overlaps
+// the softmax and P.V of the current one.
+// ---------------------------------------------------------------------------
+constexpr int kTcKeys = 128;
+constexpr int kTcStages = 3;
+constexpr int kTcThreads = 192;
+constexpr int kTcN = 16;  // query heads per MMA (padded)
+constexpr float kTcRescale = 8.0f;
+
+struct TcCfg {
+    static constexpr int D = 128;
+    static constexpr int kTileBytes = kTcKeys * D * 2;           // K or V tile: 32 KB
+    static constexpr int kStageBytes = 2 * kTileBytes;           // 64 KB
+    static constexpr int kOffQ = kTcStages * kStageBytes;        // q, 16 x 128 bf16, swizzled
+    static constexpr int kQBytes = kTcN * D * 2;                 // 4 KB
+    static constexpr int kOffP = kOffQ + kQBytes;                // P, [2][16 x 128 keys] bf16
+    static constexpr int kPBytes = kTcN * kTcKeys * 2;           // 4 KB
+    static constexpr int kOffRed = kOffP + 2 * kPBytes;          // [2][4][16] float
+    static constexpr int kOffL = kOffRed + 2 * 4 * kTcN * 4;     // [4][16] float
+    static constexpr int kOffBar = kOffL + 4 * kTcN * 4;
+    static constexpr int kNumBars = 2 * kTcStages + 2 + 5;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+    static constexpr size_t kSmem = 1024 + kOffMisc + 16;
+};
+
+template <int GT>
+__global__ void __launch_bounds__(kTcThreads, 1)
+decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                 const DecParams p) {
+    constexpr int D = 128;
+    using C = TcCfg;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint8_t *q_s = smem + C::kOffQ;
+    uint8_t *P_s = smem + C::kOffP;
+    float *red = reinterpret_cast<float *>(smem + C::kOffRed);
+    float *lred = reinterpret_cast<float *>(smem + C::kOffL);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
+    uint64_t *full = bars;                    // [stages]
+    uint64_t *empty = bars + kTcStages;       // [stages]
+    uint64_t *s_full = bars + 2 * kTcStages;  // [2]
+    uint64_t *p_full = s_full + 2;
+    uint64_t *o_done = p_full + 1;
+    uint64_t *mma_idle = o_done + 1;
+    uint64_t *sm_sync = mma_idle + 1;  // the 128 softmax threads, once per tile + epilogue
+    uint64_t *o_last = sm_sync + 1;    // completes once, after the last P.V
+    int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 1);
+
+    const int kvh = blockIdx.x % p.Hkv, chunk = blockIdx.x / p.Hkv;
+    const int b = blockIdx.y % p.B, layer = blockIdx.y / p.B;
+    int len = p.lens[b];
+    if (len > p.max_chunks * p.chunk_len) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        len = p.max_chunks * p.chunk_len;
+    }
+    const int key0 = chunk * p.chunk_len;
+    if (key0 >= len || timed_out(p.status)) return;
+    const int nkeys = min(p.chunk_len, len - key0);
+    const int ntiles = (nkeys + kTcKeys - 1) / kTcKeys;
+    const int G = p.G;
+    const int row0 = p.kv_start[b] + key0;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // q of the G heads (rows >= G zero) in the 128-byte-swizzled K-major layout;
+    // both P buffers zeroed (their rows >= G stay zero).
+    const uint16_t *qp = p.q + layer * p.q_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G) * D;
+    for (int i = tid; i < kTcN * (D / 8); i += blockDim.x) {
+        const int g = i / (D / 8), c = i % (D / 8);
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (g < G) v = *reinterpret_cast<const uint4 *>(qp + g * D + c * 8);
+        *reinterpret_cast<uint4 *>(q_s + (c >> 3) * (kTcN * 128) + g * 128 +
+                                   (((c & 7) ^ (g & 7)) << 4)) = v;
+    }
+    for (int i = tid; i < 2 * C::kPBytes / 16; i += blockDim.x)
+        reinterpret_cast<uint4 *>(P_s)[i] = make_uint4(0, 0, 0, 0);
+    if (tid == 0) {
+        for (int s = 0; s < kTcStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(&s_full[0], 1);
+        mbar_init(&s_full[1], 1);
+        mbar_init(p_full, 128);
+        mbar_init(o_done, 1);
+        mbar_init(mma_idle, 1);
+        mbar_init(sm_sync, 128);
+        mbar_init(o_last, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 64);
+        tmem_relinquish();
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = static_cast<uint32_t>(misc[0]);
+    const uint32_t tS = tmem, tO = tmem + 32;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tmK);
+            tma_prefetch_desc(&tmV);
+            int t = 0;
+            for (; t < ntiles; ++t) {
+                const int s = t % kTcStages;
+                if (t >= kTcStages &&
+                    !mbar_wait(&empty[s], ((t / kTcStages) - 1) & 1, p.status, abort_flag))
+                    break;
+                mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+                uint8_t *kd = smem + s * C::kStageBytes;
+                uint8_t *vd = kd + C::kTileBytes;
+                const int r = row0 + t * kTcKeys;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], hh * 64, kvh, r, layer);
+                    tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], hh * 64, kvh, r, layer);
+                }
+            }
+            if (*abort_flag)
+                for (int u = max(0, t - kTcStages); u < t; ++u)
+                    mbar_wait(&full[u % kTcStages], (u / kTcStages) & 1, p.status, abort_flag);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16_f32(kTcKeys, kTcN, 0, 0);
+            constexpr uint32_t idPV = idesc_bf16_f32(D, kTcN, 0, 1);
+            const uint32_t base = smem_u32(smem), q_addr = smem_u32(q_s), p_addr = smem_u32(P_s);
+            auto issue_s = [&](int t) {
+                const uint32_t k_addr = base + (t % kTcStages) * C::kStageBytes;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint64_t a = smem_desc_sw128(
+                        k_addr + (kk >> 2) * (kTcKeys * 128) + (kk & 3) * 32, 16, 1024);
+                    const uint64_t bd =
+                        smem_desc_sw128(q_addr + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
+                    tc_mma_ss(tS + (t & 1) * kTcN, a, bd, idS, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(&s_full[t & 1]);
+            };
+            bool ok = mbar_wait(&full[0], 0, p.status, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                issue_s(0);
+            }
+            for (int t = 0; ok && t < ntiles; ++t) {
+                if (t + 1 < ntiles) {
+                    const int s1 = (t + 1) % kTcStages;
+                    if (!mbar_wait(&full[s1], ((t + 1) / kTcStages) & 1, p.status, abort_flag))
+                        break;
+                    tc_fence_after();
+                    issue_s(t + 1);
+                }
+                if (!mbar_wait(p_full, t & 1, p.status, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t v_addr = base + (t % kTcStages) * C::kStageBytes + C::kTileBytes;
+                const uint32_t pb = p_addr + (t & 1) * C::kPBytes;
+#pragma unroll
+                for (int kk = 0; kk < kTcKeys / 16; ++kk) {
+                    const uint64_t a = smem_desc_sw128(v_addr + kk * (16 * 128), kTcKeys * 128, 1024);
+                    const uint64_t bd =
+                        smem_desc_sw128(pb + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
+                    tc_mma_ss(tO, a, bd, idPV, (t > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc_commit(o_done);
+                tc_commit(&empty[t % kTcStages]);
+                if (t == ntiles - 1) tc_commit(o_last);
+            }
+            tc_commit(mma_idle);
+            mbar_wait(mma_idle, 0, p.status, abort_flag);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax
+        const int quarter = warp & 3;
+        const int r = quarter * 32 + lane;  // key row of the tile, and d row of O^T
+        const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+        float m[GT], l[GT];
+#pragma unroll
+        for (int g = 0; g < GT; ++g) {
+            m[g] = -INFINITY;
+            l[g] = 0.f;
+        }
+        bool ok = true;
+        for (int t = 0; t < ntiles; ++t) {
+            if (!mbar_wait(&s_full[t & 1], (t >> 1) & 1, p.status, abort_flag)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t sr[16];
+            tmem_ld16(tS + lane_base + (t & 1) * kTcN, sr);
+            tmem_ld_wait();
+            reg_fence16(sr);
+            const bool valid = t * kTcKeys + r < nkeys;
+            float sv[GT];
+            float *rd = red + (t & 1) * 4 * kTcN;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                sv[g] = valid ? __uint_as_float(sr[g]) * p.scale_log2 : -INFINITY;
+                const float wm = warp_max(sv[g]);
+                if (lane == 0) rd[quarter * kTcN + g] = wm;
+            }
+            // all four warps' maxima visible (bounded: a wait that gives up ends the loop)
+            mbar_arrive(sm_sync);
+            if (!mbar_wait(sm_sync, t & 1, p.status, abort_flag)) {
+                ok = false;
+                break;
+            }
+            float alpha[GT];
+            bool resc = false;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const float mt = fmaxf(fmaxf(rd[g], rd[kTcN + g]),
+                                       fmaxf(rd[2 * kTcN + g], rd[3 * kTcN + g]));
+                alpha[g] = 1.f;
+                if (t == 0) {
+                    m[g] = mt;
+                } else if (mt > m[g] + kTcRescale) {
+                    alpha[g] = ex2(m[g] - mt);
+                    m[g] = mt;
+                    resc = true;
+                }
+            }
+            // P^T column r (this key) in the swizzled K-major P buffer
+            uint8_t *pb = P_s + (t & 1) * C::kPBytes + (r >> 6) * (kTcN * 128) + (r & 7) * 2;
+            const int jj = (r & 63) >> 3;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const float pr = ex2(sv[g] - m[g]);
+                l[g] = l[g] * alpha[g] + pr;
+                *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) =
+                    __float2bfloat16_rn(pr);
+            }
+            if (!valid) {
+                // V rows past the keys: zero, so 0 * garbage cannot reach O
+                uint8_t *vrow = smem + (t % kTcStages) * C::kStageBytes + C::kTileBytes + r * 128;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                    for (int u = 0; u < 8; ++u)
+                        reinterpret_cast<uint4 *>(vrow + hh * (kTcKeys * 128))[u] =
+                            make_uint4(0, 0, 0, 0);
+            }
+            if (resc) {  // block-uniform
+                if (!mbar_wait(o_done, (t - 1) & 1, p.status, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                uint32_t o[16];
+                tmem_ld16(tO + lane_base, o);
+                tmem_ld_wait();
+                reg_fence16(o);
+#pragma unroll
+                for (int g = 0; g < GT; ++g) o[g] = __float_as_uint(__uint_as_float(o[g]) * alpha[g]);
+                tmem_st16(tO + lane_base, o);
+                tmem_st_wait();
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(p_full);
+        }
+        // ------------------------------------------------------------ epilogue
+        // o_done may still be two phases behind here (S of a tile is issued before
+        // the previous tile's P.V), so the end of the last P.V has its own barrier.
+        if (ok && mbar_wait(o_last, 0, p.status, abort_flag)) {
+            tc_fence_after();
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                float v = l[g];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == 0) lred[quarter * kTcN + g] = v;
+            }
+            mbar_arrive(sm_sync);
+            if (mbar_wait(sm_sync, ntiles & 1, p.status, abort_flag)) {
+            uint32_t o[16];
+            tmem_ld16(tO + lane_base, o);
+            tmem_ld_wait();
+            reg_fence16(o);
+            const int n_chunks = (len + p.chunk_len - 1) / p.chunk_len;
+            const int64_t unit0 = ((int64_t)layer * p.B + b) * p.Hq + (int64_t)kvh * G;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                if (g >= G) break;
+                const float L = lred[g] + lred[kTcN + g] + lred[2 * kTcN + g] + lred[3 * kTcN + g];
+                const float a = __uint_as_float(o[g]);
+                if (n_chunks == 1) {
+                    uint16_t *op =
+                        p.O + layer * p.o_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G + g) * D;
+                    op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
+                    if (r == 0 && p.lse != nullptr) p.lse[unit0 + g] = (m[g] + __log2f(L)) * kLn2;
+                } else {
+                    const int64_t slot = (unit0 + g) * p.max_chunks + chunk;
+                    p.part_acc[slot * D + r] = a;
+                    if (r == 0) {
+                        p.part_ml[slot * 2 + 0] = m[g];
+                        p.part_ml[slot * 2 + 1] = L;
+                    }
+                }
+            }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, 64);
 }
 
 // One warp per (layer, sequence, query head).
@@ -379,7 +697,10 @@ struct Plan {
 Plan make_plan(const sonic_decode_args *a) {
     Plan pl{};
     const int max_len = a->max_len > 0 ? a->max_len : 1;
-    int C = a->chunk_len;
+    // explicit split lengths are rounded up to the kernel's key tile
+    const int tile = a->head_dim == 128 ? kTcKeys : kTileKeys;
+    const long long c0 = a->chunk_len < max_len ? a->chunk_len : max_len;
+    int C = (int)((c0 + tile - 1) / tile * tile);
     if (C <= 0) {
         const long long units = (long long)a->batch * a->n_heads_kv * a->n_layers;
         const long long target = 4LL * device_sm_count();
@@ -409,6 +730,32 @@ cudaError_t launch_split(const CUtensorMap &tk, const CUtensorMap &tv, const Dec
     if (e != cudaSuccess) return e;
     kern<<<grid, kDecThreads, smem, stream>>>(tk, tv, p);
     return cudaGetLastError();
+}
+
+template <int GT>
+cudaError_t launch_tc(const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p, dim3 grid,
+                      cudaStream_t stream) {
+    constexpr size_t smem = TcCfg::kSmem;
+    static_assert(smem <= 232448, "decode shared memory");
+    auto kern = decode_tc_kernel<GT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kTcThreads, smem, stream>>>(tk, tv, p);
+    return cudaGetLastError();
+}
+
+cudaError_t dispatch_tc(int GT, const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
+                        dim3 grid, cudaStream_t s) {
+    switch (GT) {
+        case 1: return launch_tc<1>(tk, tv, p, grid, s);
+        case 2: return launch_tc<2>(tk, tv, p, grid, s);
+        case 4: return launch_tc<4>(tk, tv, p, grid, s);
+        case 7: return launch_tc<7>(tk, tv, p, grid, s);
+        case 8: return launch_tc<8>(tk, tv, p, grid, s);
+        case 16: return launch_tc<16>(tk, tv, p, grid, s);
+    }
+    return cudaErrorInvalidValue;
 }
 
 template <int D>
@@ -456,8 +803,9 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const int G = a->n_heads_q / a->n_heads_kv;
     const int GT = g_template(G);
     if (GT == 0) return SONIC_ERR_UNSUPPORTED;
-    if (a->chunk_len < 0 || (a->chunk_len % kTileKeys) != 0) return SONIC_ERR_INVALID_ARGUMENT;
-    if (!aligned16(K_ret) || !aligned16(V_ret)) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->chunk_len < 0) return SONIC_ERR_INVALID_ARGUMENT;
+    if (!aligned16(K_ret) || !aligned16(V_ret) || !aligned16(q) || (a->q_layer_stride * 2) % 16)
+        return SONIC_ERR_INVALID_ARGUMENT;
     if (a->n_layers > 1 && (a->kv_layer_stride <= 0 || (a->kv_layer_stride * 2) % 16 != 0))
         return SONIC_ERR_INVALID_ARGUMENT;
     if (a->total_kv_rows == 0 || a->max_len == 0) {
@@ -472,8 +820,8 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const size_t need = pl.ws_acc + pl.ws_ml;
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
-    if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_kv > 65535 ||
-        pl.max_chunks > 0x7fffffff)
+    if ((long long)a->batch * a->n_layers > 65535 ||
+        (long long)pl.max_chunks * a->n_heads_kv > 0x7fffffffLL)
         return SONIC_ERR_UNSUPPORTED;
 
     const uint64_t row_elems = (uint64_t)a->n_heads_kv * D;
@@ -482,7 +830,7 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_kv_rows,
                               (uint64_t)a->n_layers};
     const uint64_t strides[3] = {(uint64_t)D * 2, row_elems * 2, layer_bytes};
-    const uint32_t box[4] = {64, 1, (uint32_t)kTileKeys, 1};
+    const uint32_t box[4] = {64, 1, (uint32_t)(D == 128 ? kTcKeys : kTileKeys), 1};
     CUtensorMap tk, tv;
     if (!make_tmap_bf16_4d(&tk, K_ret, dims, strides, box) ||
         !make_tmap_bf16_4d(&tv, V_ret, dims, strides, box))
@@ -508,8 +856,8 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
     p.scale_log2 = scale * kLog2e;
 
-    dim3 grid(pl.max_chunks, a->n_heads_kv, a->batch * a->n_layers);
-    cudaError_t e = (D == 128) ? dispatch_g<128>(GT, tk, tv, p, grid, stream)
+    dim3 grid(pl.max_chunks * a->n_heads_kv, a->batch * a->n_layers);
+    cudaError_t e = (D == 128) ? dispatch_tc(GT, tk, tv, p, grid, stream)
                                : dispatch_g<64>(GT, tk, tv, p, grid, stream);
     if (e != cudaSuccess) return SONIC_ERR_CUDA;
     const long long units = (long long)a->n_layers * a->batch * a->n_heads_q;

@@ -209,7 +209,25 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
         : "memory");
 }
 
-// 16 consecutive 32-bit columns of this thread's TMEM lane.
+// 16 consecutive 32-bit columns of this thread's TMEM lane (load).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void reg_fence16(uint32_t (&r)[16]) {
+    asm volatile(""
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]));
+}
+
+// 16 consecutive 32-bit columns of this thread's TMEM lane (store).
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
@@ -256,16 +274,23 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
 }
 
 // Instruction descriptor, kind::f16: bf16 A and B, fp32 D, dense.
-// b_mn_major selects an MN-major B operand (K-major otherwise); A is K-major.
+// b_mn_major / a_mn_major select MN-major operands (K-major otherwise).
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N,
-                                                      uint32_t b_mn_major) {
+                                                      uint32_t b_mn_major,
+                                                      uint32_t a_mn_major = 0) {
     return (1u << 4)            // D format: f32
            | (1u << 7)          // A format: bf16
            | (1u << 10)         // B format: bf16
-           | (0u << 15)         // A K-major
+           | (a_mn_major << 15) // A major
            | (b_mn_major << 16) // B major
            | ((N >> 3) << 17)   // N / 8
            | ((M >> 4) << 24);  // M / 16
+}
+
+// Barrier among `count` threads (a multiple of 32) on hardware barrier `id`
+// (id 0 is __syncthreads).
+__device__ __forceinline__ void named_barrier(uint32_t id, uint32_t count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 // ---------------------------------------------------------------- math

@@ -88,8 +88,8 @@ def test_host_validation_rejects_before_launch():
     d.kv_start, d.max_len, d.total_kv_rows = 16, 10, 20
     assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 2  # G = 20 > 16
     d.n_heads_q = 8
-    d.chunk_len = 100
-    assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 1  # not x64
+    d.chunk_len = -5
+    assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 1  # negative
     d.chunk_len, d.head_dim = 0, 80
     assert lib.sonic_attn_decode(16, 16, 16, 16, 16, ctypes.byref(d), None) == 2
 
