@@ -2,24 +2,23 @@
 // mask (Sec. 3.2: Eq. 3 causal rule, Eq. 4 historical body removal, Eq. 5
 // bidirectional Nexus visibility), on the sm_103a tensor cores.
 //
-// One block computes a 128-row query tile of one (layer, sequence, query
-// head).  Six warps:
-//   warp 0     TMA producer: the Q tile once, then K and V tiles (128 keys)
+// One block computes two 128-row query tiles of one (layer, sequence, query
+// head).  Ten warps:
+//   warp 0     TMA producer: the Q tiles once, then K and V tiles (128 keys)
 //              into a 2-stage ring, with the role/segment numbers of the keys;
-//   warp 1     tcgen05 issuer: S = Q K^T into one of two TMEM buffers (fp32,
-//              128 lanes x 128 columns), and O += P V into a TMEM accumulator,
-//              one elected thread issuing every MMA;
-//   warps 2-5  softmax: thread r owns query row r (TMEM lane r).  It reads its
-//              S row with tcgen05.ld, applies the mask per element only on
-//              tiles the mask cuts, runs the online softmax in base 2, rescales
-//              its O row in TMEM when the running maximum moves, and writes P
-//              (bf16) into shared memory in the 128-byte-swizzled K-major
-//              layout the next MMA reads.
+//   warp 1     tcgen05 issuer: S_t = Q_t K^T into TMEM (fp32, 128 lanes x 128
+//              columns per tile), and O_t += P_t V with P read from TMEM, one
+//              elected thread issuing every MMA;
+//   warps 2-9  softmax, one warpgroup per query tile: thread r owns query row
+//              r (TMEM lane r).  It reads its S row with tcgen05.ld, applies
+//              the mask per element only on tiles the mask cuts, runs the
+//              online softmax in base 2, rescales its O row in TMEM when the
+//              running maximum has risen by more than 2^8, and writes P (bf16
+//              pairs) back over its S columns.
 // Before the loop the block lists the key tiles it must visit: each tile is
 // classified from precomputed per-tile summaries (which roles and segment
 // numbers occur in it) as hidden (skipped entirely), fully visible (no mask
-// work) or cut by the mask.  S(j+1) is computed while the softmax works on
-// S(j).
+// work) or cut by the mask.  The two tiles' softmax and MMAs interleave.
 #include "sonic_dev.cuh"
 #include "sonic_host.h"
 
@@ -28,7 +27,7 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kPfThreads = 384;
+constexpr int kPfThreads = 320;
 constexpr int kMaxKTiles = 2048;
 constexpr float kLn2f = 0.6931471805599453f;
 constexpr float kLog2ef = 1.4426950408889634f;
@@ -154,11 +153,12 @@ __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, in
 constexpr float kRescaleThreshold = 8.0f;
 
 // Two 128-row query tiles (tile 0 = rows 0..127 of the block's 256, tile 1 =
-// rows 128..255) share every K/V tile.  Warp roles:
+// rows 128..255) share every K/V tile.  Warp roles (320 threads, so every
+// thread can hold a full 128-column S row in registers):
 //   warp 0       TMA producer (K, V, Q) and key metadata,
 //   warp 1       tcgen05 issuer and TMEM owner,
-//   warps 2-3    idle after set-up,
-//   warps 4-7    softmax of tile 0, warps 8-11 softmax of tile 1.
+//   warps 2-5    softmax of tile 0, warps 6-9 softmax of tile 1 (warp w
+//                reaches TMEM lanes 32 * (w % 4) .. + 31).
 // TMEM (512 columns): S/P of tile 0 at 0, of tile 1 at 128, O of tile 0 at
 // 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns
 // of its S block and feeds O += P V straight from tensor memory.
@@ -290,7 +290,6 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
-
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
@@ -402,9 +401,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tc_commit(mma_idle);
             mbar_wait(mma_idle, 0, p.status, abort_flag);
         }
-    } else if (warp >= 4 && (warp < 8 || tile1)) {
+    } else if (warp < 6 || tile1) {
         // ------------------------------------------------------------ softmax
-        const int qi = (warp - 4) >> 2;
+        const int qi = (warp - 2) >> 2;
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
         const int pos = pbase + qi * kBM + r;
@@ -419,59 +418,60 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const uint32_t tO = tmem + lane_base + 256 + qi * 128;
         float m_used = -INFINITY, l = 0.f;
         bool ok = true;
+        // the next list entry is read one tile ahead: shared memory is busy
+        // feeding the tensor cores, so a load on the critical path is slow
+        int entry = n_list > 0 ? list[0] : 0;
         for (int j = 0; j < n_list; ++j) {
             const int st = j & 1;
-            if (!mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag) ||
+            const int kt = entry >> 2;
+            const bool cut = (entry >> qi) & 1;
+            entry = j + 1 < n_list ? list[j + 1] : 0;
+            // the keys' roles/segments are read (and V rows zeroed) on cut tiles only
+            if ((cut && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) ||
                 !mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const int kt = list[j] >> 2;
-            const bool cut = (list[j] >> qi) & 1;
-            // pass 1: row maximum (and the mask bits of a cut tile), two 32-column
-            // chunks per tensor-memory round trip
+            // S row into registers: four 32-column loads, one wait
+            uint32_t sr[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+            tmem_ld_wait();
+#pragma unroll
+            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
+            // row maximum (and the mask bits of a cut tile)
             uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-            float mxa = -INFINITY, mxb = -INFINITY;
+            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (!cut) {
 #pragma unroll
-            for (int c2 = 0; c2 < 2; ++c2) {
-                uint32_t sa[32], sb[32];
-                tmem_ld32(tS + c2 * 64, sa);
-                tmem_ld32(tS + c2 * 64 + 32, sb);
-                tmem_ld_wait();
-                reg_fence32(sa);
-                reg_fence32(sb);
-                if (!cut) {
+                for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        mxa = fmax3(mxa, __uint_as_float(sa[e]), __uint_as_float(sa[e + 1]));
-                        mxb = fmax3(mxb, __uint_as_float(sb[e]), __uint_as_float(sb[e + 1]));
-                    }
-                } else {
+                    for (int e = 0; e < 32; e += 2)
+                        mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][e]),
+                                       __uint_as_float(sr[c][e + 1]));
+            } else {
 #pragma unroll
-                    for (int hc = 0; hc < 2; ++hc) {
-                        const int c = c2 * 2 + hc;
-                        const uint8_t *mr = meta_role + st * kBN + c * 32;
-                        const int32_t *ms = meta_seg + st * kBN + c * 32;
-                        uint32_t bits = 0;
+                for (int c = 0; c < 4; ++c) {
+                    const uint8_t *mr = meta_role + st * kBN + c * 32;
+                    const int32_t *ms = meta_seg + st * kBN + c * 32;
+                    uint32_t bits = 0;
 #pragma unroll 4
-                        for (int e = 0; e < 32; ++e) {
-                            const int rq = mr[e];
-                            const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp,
-                                                                rq, ms[e], p.nexus_mode);
-                            bits |= (v ? 1u : 0u) << e;
-                        }
-                        mbits[c] = bits;
-                        const uint32_t *sv = hc ? sb : sa;
+                    for (int e = 0; e < 32; ++e) {
+                        const int rq = mr[e];
+                        const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp, rq,
+                                                            ms[e], p.nexus_mode);
+                        bits |= (v ? 1u : 0u) << e;
+                    }
+                    mbits[c] = bits;
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) {
-                            const float v = ((bits >> e) & 1) ? __uint_as_float(sv[e]) : -INFINITY;
-                            if (hc) mxb = fmaxf(mxb, v); else mxa = fmaxf(mxa, v);
-                        }
+                    for (int e = 0; e < 32; ++e) {
+                        if (!((bits >> e) & 1)) sr[c][e] = __float_as_uint(-INFINITY);
+                        mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][e]));
                     }
                 }
             }
-            const float mx = fmaxf(mxa, mxb) * p.scale_log2;
+            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
             float alpha = 1.f, m_new = m_used;
             if (j == 0) {
                 m_new = mx;
@@ -480,41 +480,26 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 alpha = ex2(m_used - m_new);
             }
             const float mref = (m_new == -INFINITY) ? 0.f : m_new;
-            // pass 2: probabilities, written as bf16 pairs over the S columns
+            // probabilities, written as bf16 pairs over the S columns
             const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
             const float2 nm2 = make_float2(-mref, -mref);
             float2 rs2a = make_float2(0.f, 0.f), rs2b = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int c2 = 0; c2 < 2; ++c2) {
-                uint32_t sa[32], sb[32];
-                tmem_ld32(tS + c2 * 64, sa);
-                tmem_ld32(tS + c2 * 64 + 32, sb);
-                tmem_ld_wait();
-                reg_fence32(sa);
-                reg_fence32(sb);
+            for (int c = 0; c < 4; ++c) {
+                uint32_t pk[16];
 #pragma unroll
-                for (int hc = 0; hc < 2; ++hc) {
-                    const uint32_t *sv = hc ? sb : sa;
-                    const uint32_t bits = mbits[c2 * 2 + hc];
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        float2 x = __ffma2_rn(
-                            make_float2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2,
-                            nm2);
-                        if (cut) {
-                            x.x = ((bits >> e) & 1) ? x.x : -INFINITY;
-                            x.y = ((bits >> (e + 1)) & 1) ? x.y : -INFINITY;
-                        }
-                        const float2 ev = make_float2(ex2(x.x), ex2(x.y));
-                        if ((e >> 1) & 1)
-                            rs2b = __fadd2_rn(rs2b, ev);
-                        else
-                            rs2a = __fadd2_rn(rs2a, ev);
-                        pk[e >> 1] = pack_bf16x2(ev.x, ev.y);
-                    }
-                    tmem_st16(tS + (c2 * 2 + hc) * 16, pk);
+                for (int e = 0; e < 32; e += 2) {
+                    const float2 x = __ffma2_rn(
+                        make_float2(__uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1])), sc2,
+                        nm2);
+                    const float2 ev = make_float2(ex2(x.x), ex2(x.y));
+                    if ((e >> 1) & 1)
+                        rs2b = __fadd2_rn(rs2b, ev);
+                    else
+                        rs2a = __fadd2_rn(rs2a, ev);
+                    pk[e >> 1] = pack_bf16x2(ev.x, ev.y);
                 }
+                tmem_st16(tS + c * 16, pk);
             }
             l = l * alpha + ((rs2a.x + rs2a.y) + (rs2b.x + rs2b.y));
             // O rescale (PV of the previous tile is complete: S of this tile was
