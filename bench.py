@@ -24,6 +24,7 @@ Reported:
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import math
 import os
@@ -44,6 +45,23 @@ METRIC = "Nexus-KV attn: decode HBM GB/s & prefill TFLOP/s vs GB300 peak"
 WORKLOAD = ("mixed serving step: 64 ragged sequences, 28 layers, 28/4 heads, D=128, bf16; "
             "8 compact a 4k-64k raw history then prefill a 256-2048-token turn, 56 decode "
             "over 1k-18k retained rows")
+
+
+def max_over_ranks(values, device="cpu"):
+    """Element-wise maximum of `values` over all ranks (the timing rule: the
+    slowest rank defines the step); identity on a single process."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def weak_rate(work_per_step: float, steps: int, world: int, ms: float, scale: float) -> float:
+    """Whole-job throughput of N replicas: every rank processes the same work
+    per step, the job time is the slowest rank's."""
+    return work_per_step * steps * world / (ms * 1e-3) / scale
 
 
 def _peaks():
@@ -307,6 +325,13 @@ def run_gpu(args, rank: int, world: int):
         raise RuntimeError("device status set during the timed steps")
 
     # ---------------- end to end: host buffers through the public calls
+    # Every step copies its inputs from pinned host memory (new-turn Q, decode
+    # q, the new tokens' K/V rows) and reads its outputs back (prefill O,
+    # decode O).  Steps are pipelined over three streams, as a server would
+    # run them: inputs of step k+1 and outputs of step k-1 move while step k
+    # computes (Q/O double-buffered); the K/V rows land in one contiguous copy
+    # and are appended into their cache rows by device-to-device strided
+    # copies just before the step that reads them.
     pin = lambda t: t.cpu().pin_memory()
     hQ, hqd = pin(g.Qp), pin(g.qd)
     hOp, hOd = torch.empty_like(hQ).pin_memory(), torch.empty_like(hqd).pin_memory()
@@ -314,51 +339,99 @@ def run_gpu(args, rank: int, world: int):
     newV = pin(newK.clone())
     dec_rows = lay.dec_start + lay.dec_len - 1
     hdecK = pin(g.Kret[:, torch.as_tensor(dec_rows, device=device).long()])
-    hdecV = pin(g.Vret[:, torch.as_tensor(dec_rows, device=device).long()])
-    dst_rows = [(int(lay.k_start_pre[b] + lay.ret_pre[b]), int(lay.q_len[b]), int(lay.q_start[b]))
-                for b in range(lay.n_pre)]
-    dec_rows_dev = torch.as_tensor(dec_rows, device=device).long()
+    hdecV = pin(hdecK.clone())
+    stK, stV = torch.empty_like(newK, device=device), torch.empty_like(newV, device=device)
+    stdK, stdV = torch.empty_like(hdecK, device=device), torch.empty_like(hdecV, device=device)
+    sets = [(g.Qp, g.qd, g.Op, g.Od),
+            (torch.empty_like(g.Qp), torch.empty_like(g.qd), torch.empty_like(g.Op),
+             torch.empty_like(g.Od))]
     h2d = (hQ.numel() + hqd.numel() + newK.numel() + newV.numel() + hdecK.numel() +
            hdecV.numel()) * 2
     d2h = (hOp.numel() + hOd.numel()) * 2
+    rb = lay.row_bytes
+    cuda_rt = _cudart()
+    dpitch = lay.T_ret * rb
+    s_in, s_out = torch.cuda.Stream(device), torch.cuda.Stream(device)
 
-    def e2e_step():
-        g.Qp.copy_(hQ, non_blocking=True)
-        g.qd.copy_(hqd, non_blocking=True)
-        for s, n, qs in dst_rows:
-            g.Kret[:, s:s + n].copy_(newK[:, qs:qs + n], non_blocking=True)
-            g.Vret[:, s:s + n].copy_(newV[:, qs:qs + n], non_blocking=True)
-        g.Kret[:, dec_rows_dev] = hdecK.to(device, non_blocking=True)
-        g.Vret[:, dec_rows_dev] = hdecV.to(device, non_blocking=True)
-        g.step(stream)
-        hOp.copy_(g.Op, non_blocking=True)
-        hOd.copy_(g.Od, non_blocking=True)
+    def copy2d_d2d(dst, src, spitch, width, height):
+        rc = cuda_rt.cudaMemcpy2DAsync(ctypes.c_void_p(dst), ctypes.c_size_t(dpitch),
+                                       ctypes.c_void_p(src), ctypes.c_size_t(spitch),
+                                       ctypes.c_size_t(width), ctypes.c_size_t(height), 3,
+                                       ctypes.c_void_p(stream.cuda_stream))
+        if rc != 0:
+            raise RuntimeError(f"cudaMemcpy2DAsync failed: {rc}")
 
-    with torch.cuda.stream(stream):
-        for _ in range(max(1, args.warmup // 2)):
-            e2e_step()
+    def append_rows():
+        for b in range(lay.n_pre):
+            r0, n, qs = (int(lay.k_start_pre[b] + lay.ret_pre[b]), int(lay.q_len[b]),
+                         int(lay.q_start[b]))
+            copy2d_d2d(g.Kret.data_ptr() + r0 * rb, stK.data_ptr() + qs * rb, lay.T_q * rb,
+                       n * rb, lay.NL)
+            copy2d_d2d(g.Vret.data_ptr() + r0 * rb, stV.data_ptr() + qs * rb, lay.T_q * rb,
+                       n * rb, lay.NL)
+        for i, r in enumerate(dec_rows):
+            copy2d_d2d(g.Kret.data_ptr() + int(r) * rb, stdK.data_ptr() + i * rb,
+                       lay.n_dec * rb, rb, lay.NL)
+            copy2d_d2d(g.Vret.data_ptr() + int(r) * rb, stdV.data_ptr() + i * rb,
+                       lay.n_dec * rb, rb, lay.NL)
+
+    def e2e_run(nsteps):
+        ev_in = [ev() for _ in range(nsteps)]
+        ev_app = [ev() for _ in range(nsteps)]
+        ev_comp = [ev() for _ in range(nsteps)]
+        ev_out = [ev() for _ in range(nsteps)]
+        start, end = ev(), ev()
+        start.record(stream)
+        s_in.wait_event(start)
+        for k in range(nsteps):
+            Qp, qd, Op, Od = sets[k % 2]
+            with torch.cuda.stream(s_in):
+                if k >= 2:
+                    s_in.wait_event(ev_comp[k - 2])  # set k%2 no longer read
+                if k >= 1:
+                    s_in.wait_event(ev_app[k - 1])   # staging buffers consumed
+                Qp.copy_(hQ, non_blocking=True)
+                qd.copy_(hqd, non_blocking=True)
+                stK.copy_(newK, non_blocking=True)
+                stV.copy_(newV, non_blocking=True)
+                stdK.copy_(hdecK, non_blocking=True)
+                stdV.copy_(hdecV, non_blocking=True)
+                ev_in[k].record(s_in)
+            with torch.cuda.stream(stream):
+                stream.wait_event(ev_in[k])
+                if k >= 2:
+                    stream.wait_event(ev_out[k - 2])  # O of set k%2 read back
+                append_rows()
+                ev_app[k].record(stream)
+                g.Qp, g.qd, g.Op, g.Od = Qp, qd, Op, Od
+                g.step(stream)
+                ev_comp[k].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_comp[k])
+                hOp.copy_(Op, non_blocking=True)
+                hOd.copy_(Od, non_blocking=True)
+                ev_out[k].record(s_out)
+        s_out.wait_event(ev_out[nsteps - 1])
+        end.record(s_out)
+        return start, end
+
+    e2e_run(max(2, args.warmup // 2))
     barrier()
-    e0, e1 = ev(), ev()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(args.steps):
-            e2e_step()
-        e1.record(stream)
+    e0, e1 = e2e_run(args.steps)
     barrier()
     e2e_ms = e0.elapsed_time(e1)
+    g.Qp, g.qd, g.Op, g.Od = sets[0]
 
     # max over ranks
-    vals = torch.tensor([total_ms, c_ms, p_ms, d_ms, e2e_ms], dtype=torch.float64, device=device)
-    if world > 1:
-        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
-    total_ms, c_ms, p_ms, d_ms, e2e_ms = vals.tolist()
+    total_ms, c_ms, p_ms, d_ms, e2e_ms = max_over_ranks([total_ms, c_ms, p_ms, d_ms, e2e_ms],
+                                                        device)
     K = args.steps
     pk = _peaks()
     pf = lay.prefill_flops()
-    value = pf * K * world / (p_ms * 1e-3) / 1e12
-    dec_gbs = lay.decode_bytes() * K * world / (d_ms * 1e-3) / 1e9
-    cmp_gbs = lay.compact_bytes() * K * world / (c_ms * 1e-3) / 1e9
-    e2e_val = pf * K * world / (e2e_ms * 1e-3) / 1e12
+    value = weak_rate(pf, K, world, p_ms, 1e12)
+    dec_gbs = weak_rate(lay.decode_bytes(), K, world, d_ms, 1e9)
+    cmp_gbs = weak_rate(lay.compact_bytes(), K, world, c_ms, 1e9)
+    e2e_val = weak_rate(pf, K, world, e2e_ms, 1e12)
     prof = _traffic()
     achieved = pf / (p_ms / K * 1e-3) / 1e12
     out = {
@@ -398,6 +471,19 @@ def run_gpu(args, rank: int, world: int):
         "clocks": clk,
     }
     return out, lay
+
+
+def _cudart():
+    """The CUDA runtime torch already loaded (for strided host->device copies)."""
+    import torch  # noqa: F401  (loads libcudart)
+    for name in ("libcudart.so.13", "libcudart.so"):
+        try:
+            lib = ctypes.CDLL(name)
+            lib.cudaMemcpy2DAsync.restype = ctypes.c_int
+            return lib
+        except OSError:
+            continue
+    raise RuntimeError("libcudart not found")
 
 
 def _traffic():
