@@ -130,7 +130,8 @@ struct PfCfg {
     static constexpr int kOffQ = 0;                           // [2] Q tiles
     static constexpr int kOffK = kOffQ + 2 * kQBytes;         // [2] stages
     static constexpr int kOffV = kOffK + 2 * kKVBytes;        // [2] stages
-    static constexpr int kOffRole = kOffV + 2 * kKVBytes;     // [2][128] uint8
+    static constexpr int kOffMask = kOffV + 2 * kKVBytes;     // [2] TileMasks
+    static constexpr int kOffRole = kOffMask + 2 * 256;       // [2][128] uint8
     static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
     static constexpr int kOffList = kOffSeg + 2 * kBN * 4;    // [kMaxKTiles] int32
     static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
@@ -139,6 +140,21 @@ struct PfCfg {
     static constexpr int kBytes = kOffMisc + 32 * 4;
     static constexpr size_t kSmem = 1024 + kBytes;
 };
+
+// Column masks of one 128-key tile (bit c of word w = key 32 w + c of the
+// tile): keys that are not body rows (nb), Nexus keys (nx), and the keys of
+// each distinct segment among the body keys (bm) and among the Nexus keys
+// (nm, used by the causal-segments reading).  With them a row's visibility
+// mask costs a few word operations.  More than four distinct segments in
+// one tile (not produced by valid layouts of reasonable segment length)
+// sets `fallback` and the rule is evaluated per key instead.
+struct TileMasks {
+    uint32_t nb[4], nx[4];
+    int32_t nbody, nnex, fallback, pad;
+    int32_t bseg[4], nseg[4];
+    uint32_t bm[4][4], nm[4][4];
+};
+static_assert(sizeof(TileMasks) <= 256, "tile masks");
 
 __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, int sq,
                                         int mode) {
@@ -173,6 +189,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint8_t *Qs = smem + C::kOffQ;
     uint8_t *Ks = smem + C::kOffK;
     uint8_t *Vs = smem + C::kOffV;
+    TileMasks *tmasks = reinterpret_cast<TileMasks *>(smem + C::kOffMask);
     uint8_t *meta_role = smem + C::kOffRole;
     int32_t *meta_seg = reinterpret_cast<int32_t *>(smem + C::kOffSeg);
     int32_t *list = reinterpret_cast<int32_t *>(smem + C::kOffList);
@@ -309,21 +326,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (i >= 2 && !mbar_wait(&kv_empty[st], ((i >> 1) - 1) & 1, p.status, abort_flag))
                 break;
             const int kt = list[i] >> 2;
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int c = lane * 4 + u;
-                const int q = kt * kBN + c;
-                uint8_t ro = 255;  // rows past the sequence
-                int32_t sg = 0;
-                if (q < klen) {
-                    ro = p.role[kstart + q];
-                    sg = p.seg[kstart + q];
-                }
-                meta_role[st * kBN + c] = ro;
-                meta_seg[st * kBN + c] = sg;
-            }
+            // K/V copies first; the key metadata is built while they are in flight
             if (lane == 0) {
-                mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
+                mbar_expect_tx(&kv_full[st], 2 * C::kKVBytes);
                 const int row = kstart + kt * kBN;
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh) {
@@ -332,9 +337,104 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), &tmV, &kv_full[st],
                                 hh * 64, kvh, row, layer);
                 }
-            } else {
-                mbar_arrive(&kv_full[st]);
             }
+            // Roles / segments of the tile's keys (lane = key within each
+            // 32-key word; 255 marks rows past the sequence) and their masks:
+            // needed only where a query tile is cut by the mask.
+            if ((list[i] & 3) == 0) {
+                mbar_arrive(&kv_full[st]);
+                continue;
+            }
+            int ro[4], sg[4];
+            uint32_t bst[4], nst[4];
+            int pro = 255, psg = 0;
+            TileMasks &tm = tmasks[st];
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const int c = w * 32 + lane;
+                const int q = kt * kBN + c;
+                ro[w] = 255;
+                sg[w] = 0;
+                if (q < klen) {
+                    ro[w] = p.role[kstart + q];
+                    sg[w] = p.seg[kstart + q];
+                }
+                meta_role[st * kBN + c] = (uint8_t)ro[w];
+                meta_seg[st * kBN + c] = sg[w];
+                const bool isb = ro[w] == SONIC_ROLE_BODY, isn = ro[w] == SONIC_ROLE_NEXUS;
+                const uint32_t nbw = __ballot_sync(0xffffffffu, ro[w] != 255 && !isb);
+                const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
+                // previous key's role/segment (lane 0: last key of the previous word)
+                int r_up = __shfl_up_sync(0xffffffffu, ro[w], 1);
+                int s_up = __shfl_up_sync(0xffffffffu, sg[w], 1);
+                if (lane == 0) {
+                    r_up = pro;
+                    s_up = psg;
+                }
+                bst[w] = __ballot_sync(0xffffffffu, isb && !(r_up == SONIC_ROLE_BODY && s_up == sg[w]));
+                nst[w] = __ballot_sync(0xffffffffu, isn && !(r_up == SONIC_ROLE_NEXUS && s_up == sg[w]));
+                pro = __shfl_sync(0xffffffffu, ro[w], 31);
+                psg = __shfl_sync(0xffffffffu, sg[w], 31);
+                if (lane == 0) {
+                    tm.nb[w] = nbw;
+                    tm.nx[w] = nxw;
+                }
+            }
+            // distinct segments of body runs and Nexus runs (in key order)
+            int nb_n = 0, nn_n = 0, fb = 0;
+            int bsv[4] = {0, 0, 0, 0}, nsv[4] = {0, 0, 0, 0};
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                uint32_t m = bst[w];
+                while (m) {
+                    const int bl = __ffs(m) - 1;
+                    m &= m - 1;
+                    const int v = __shfl_sync(0xffffffffu, sg[w], bl);
+                    bool seen = false;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) seen |= (k < nb_n && bsv[k] == v);
+                    if (!seen) {
+                        if (nb_n < 4) bsv[nb_n++] = v; else fb = 1;
+                    }
+                }
+                m = nst[w];
+                while (m) {
+                    const int bl = __ffs(m) - 1;
+                    m &= m - 1;
+                    const int v = __shfl_sync(0xffffffffu, sg[w], bl);
+                    bool seen = false;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) seen |= (k < nn_n && nsv[k] == v);
+                    if (!seen) {
+                        if (nn_n < 4) nsv[nn_n++] = v; else fb = 1;
+                    }
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const uint32_t bmw = __ballot_sync(
+                        0xffffffffu, k < nb_n && ro[w] == SONIC_ROLE_BODY && sg[w] == bsv[k]);
+                    const uint32_t nmw = __ballot_sync(
+                        0xffffffffu, k < nn_n && ro[w] == SONIC_ROLE_NEXUS && sg[w] == nsv[k]);
+                    if (lane == 0) {
+                        tm.bm[k][w] = bmw;
+                        tm.nm[k][w] = nmw;
+                    }
+                }
+            if (lane == 0) {
+                tm.nbody = nb_n;
+                tm.nnex = nn_n;
+                tm.fallback = fb;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    tm.bseg[k] = bsv[k];
+                    tm.nseg[k] = nsv[k];
+                }
+            }
+            __syncwarp();
+            mbar_arrive(&kv_full[st]);  // 32 arrivals + the copies' bytes end the phase
         }
         if (lane == 0 && *abort_flag) {
             // let issued copies land before the block exits
@@ -451,25 +551,66 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][e]),
                                        __uint_as_float(sr[c][e + 1]));
             } else {
+                // the whole mask record in independent 16-byte loads
+                const uint4 *tv = reinterpret_cast<const uint4 *>(tmasks + st);
+                const uint4 nb = tv[0], nx = tv[1], hd = tv[2], bsg = tv[3], nsg = tv[4];
+                uint4 bm[4], nm[4];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const uint8_t *mr = meta_role + st * kBN + c * 32;
-                    const int32_t *ms = meta_seg + st * kBN + c * 32;
-                    uint32_t bits = 0;
-#pragma unroll 4
-                    for (int e = 0; e < 32; ++e) {
-                        const int rq = mr[e];
-                        const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp, sp, rq,
-                                                            ms[e], p.nexus_mode);
-                        bits |= (v ? 1u : 0u) << e;
+                for (int k = 0; k < 4; ++k) {
+                    bm[k] = tv[5 + k];
+                    nm[k] = tv[9 + k];
+                }
+                if (!hd.z) {
+                    // causal prefix (keys at or before this row), body keys of this
+                    // row's segment, and the Nexus keys a Nexus row sees
+                    const int nvis = pos - kt * kBN + 1;
+                    const int nbody = (int)hd.x, nnex = (int)hd.y;
+                    const int bs4[4] = {(int)bsg.x, (int)bsg.y, (int)bsg.z, (int)bsg.w};
+                    const int ns4[4] = {(int)nsg.x, (int)nsg.y, (int)nsg.z, (int)nsg.w};
+                    uint4 bw = make_uint4(0u, 0u, 0u, 0u), xw = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        if (k < nbody && bs4[k] == sp) {
+                            bw.x |= bm[k].x; bw.y |= bm[k].y; bw.z |= bm[k].z; bw.w |= bm[k].w;
+                        }
+                        if (rp == SONIC_ROLE_NEXUS && p.nexus_mode != SONIC_NEXUS_FULL &&
+                            k < nnex && ns4[k] <= sp) {
+                            xw.x |= nm[k].x; xw.y |= nm[k].y; xw.z |= nm[k].z; xw.w |= nm[k].w;
+                        }
                     }
-                    mbits[c] = bits;
+                    if (rp == SONIC_ROLE_NEXUS && p.nexus_mode == SONIC_NEXUS_FULL) xw = nx;
+                    const uint32_t nbw[4] = {nb.x, nb.y, nb.z, nb.w};
+                    const uint32_t bww[4] = {bw.x, bw.y, bw.z, bw.w};
+                    const uint32_t xww[4] = {xw.x, xw.y, xw.z, xw.w};
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        if (!((bits >> e) & 1)) sr[c][e] = __float_as_uint(-INFINITY);
-                        mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][e]));
+                    for (int w = 0; w < 4; ++w) {
+                        const int nw = min(max(nvis - 32 * w, 0), 32);
+                        const uint32_t cw = nw >= 32 ? 0xffffffffu : ((1u << nw) - 1u);
+                        mbits[w] = (cw & (nbw[w] | bww[w])) | xww[w];
+                    }
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const uint8_t *mr = meta_role + st * kBN + c * 32;
+                        const int32_t *ms = meta_seg + st * kBN + c * 32;
+                        uint32_t bits = 0;
+#pragma unroll 4
+                        for (int e = 0; e < 32; ++e) {
+                            const int rq = mr[e];
+                            const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp,
+                                                                sp, rq, ms[e], p.nexus_mode);
+                            bits |= (v ? 1u : 0u) << e;
+                        }
+                        mbits[c] = bits;
                     }
                 }
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        if (!((mbits[c] >> e) & 1)) sr[c][e] = __float_as_uint(-INFINITY);
+                        mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][e]));
+                    }
             }
             const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
             float alpha = 1.f, m_new = m_used;
