@@ -24,7 +24,6 @@ Reported:
 from __future__ import annotations
 
 import argparse
-import ctypes
 import json
 import math
 import os
@@ -330,8 +329,8 @@ def run_gpu(args, rank: int, world: int):
     # decode O).  Steps are pipelined over three streams, as a server would
     # run them: inputs of step k+1 and outputs of step k-1 move while step k
     # computes (Q/O double-buffered); the K/V rows land in one contiguous copy
-    # and are appended into their cache rows by device-to-device strided
-    # copies just before the step that reads them.
+    # and are appended into their cache rows by indexed device copies just
+    # before the step that reads them.
     pin = lambda t: t.cpu().pin_memory()
     hQ, hqd = pin(g.Qp), pin(g.qd)
     hOp, hOd = torch.empty_like(hQ).pin_memory(), torch.empty_like(hqd).pin_memory()
@@ -348,32 +347,20 @@ def run_gpu(args, rank: int, world: int):
     h2d = (hQ.numel() + hqd.numel() + newK.numel() + newV.numel() + hdecK.numel() +
            hdecV.numel()) * 2
     d2h = (hOp.numel() + hOd.numel()) * 2
-    rb = lay.row_bytes
-    cuda_rt = _cudart()
-    dpitch = lay.T_ret * rb
     s_in, s_out = torch.cuda.Stream(device), torch.cuda.Stream(device)
 
-    def copy2d_d2d(dst, src, spitch, width, height):
-        rc = cuda_rt.cudaMemcpy2DAsync(ctypes.c_void_p(dst), ctypes.c_size_t(dpitch),
-                                       ctypes.c_void_p(src), ctypes.c_size_t(spitch),
-                                       ctypes.c_size_t(width), ctypes.c_size_t(height), 3,
-                                       ctypes.c_void_p(stream.cuda_stream))
-        if rc != 0:
-            raise RuntimeError(f"cudaMemcpy2DAsync failed: {rc}")
+    # cache rows the new tokens go to (indexed copies on the compute stream)
+    pre_rows = torch.as_tensor(np.concatenate(
+        [np.arange(lay.k_start_pre[b] + lay.ret_pre[b],
+                   lay.k_start_pre[b] + lay.ret_pre[b] + lay.q_len[b])
+         for b in range(lay.n_pre)]), device=device).long()
+    dec_rows_t = torch.as_tensor(dec_rows, device=device).long()
 
     def append_rows():
-        for b in range(lay.n_pre):
-            r0, n, qs = (int(lay.k_start_pre[b] + lay.ret_pre[b]), int(lay.q_len[b]),
-                         int(lay.q_start[b]))
-            copy2d_d2d(g.Kret.data_ptr() + r0 * rb, stK.data_ptr() + qs * rb, lay.T_q * rb,
-                       n * rb, lay.NL)
-            copy2d_d2d(g.Vret.data_ptr() + r0 * rb, stV.data_ptr() + qs * rb, lay.T_q * rb,
-                       n * rb, lay.NL)
-        for i, r in enumerate(dec_rows):
-            copy2d_d2d(g.Kret.data_ptr() + int(r) * rb, stdK.data_ptr() + i * rb,
-                       lay.n_dec * rb, rb, lay.NL)
-            copy2d_d2d(g.Vret.data_ptr() + int(r) * rb, stdV.data_ptr() + i * rb,
-                       lay.n_dec * rb, rb, lay.NL)
+        g.Kret.index_copy_(1, pre_rows, stK)
+        g.Vret.index_copy_(1, pre_rows, stV)
+        g.Kret.index_copy_(1, dec_rows_t, stdK)
+        g.Vret.index_copy_(1, dec_rows_t, stdV)
 
     def e2e_run(nsteps):
         ev_in = [ev() for _ in range(nsteps)]
@@ -471,19 +458,6 @@ def run_gpu(args, rank: int, world: int):
         "clocks": clk,
     }
     return out, lay
-
-
-def _cudart():
-    """The CUDA runtime torch already loaded (for strided host->device copies)."""
-    import torch  # noqa: F401  (loads libcudart)
-    for name in ("libcudart.so.13", "libcudart.so"):
-        try:
-            lib = ctypes.CDLL(name)
-            lib.cudaMemcpy2DAsync.restype = ctypes.c_int
-            return lib
-        except OSError:
-            continue
-    raise RuntimeError("libcudart not found")
 
 
 def _traffic():
