@@ -91,6 +91,22 @@ typedef enum {
     SONIC_NEXUS_CAUSAL_SEGMENTS = 1
 } sonic_nexus_vis_t;
 
+/* Order in which sonic_attn_prefill walks a sequence's keys.
+ * AS_GIVEN: the key rows as laid out (S_aug order).
+ * RETAINED_FIRST: the library first copies each sequence's keys (K and V of
+ * every layer, role, segment) into its workspace as [system prompt, Nexus and
+ * current-turn rows | history bodies], each part in S_aug order and the
+ * bodies starting on a 128-row boundary; the mask still compares S_aug
+ * positions.  Every query row then sees one prefix of the retained part plus
+ * (for body and Nexus rows) the body of its own segment, so far fewer key
+ * tiles are visited and cut by the mask when all rows of S_aug are queried.
+ * Results equal AS_GIVEN up to floating-point summation order.  The copy
+ * costs workspace: see sonic_prefill_workspace_size. */
+typedef enum {
+    SONIC_KEYS_AS_GIVEN = 0,
+    SONIC_KEYS_RETAINED_FIRST = 1
+} sonic_key_order_t;
+
 /* ------------------------------------------------------------------------- */
 /* Compaction                                                                */
 /* ------------------------------------------------------------------------- */
@@ -159,7 +175,8 @@ typedef struct {
                                     query i is key position k_len[b] - q_len[b] + i
                                     (the last q_len rows: bottom-right aligned)         */
     int32_t max_q_len;           /* host: >= every q_len[b]; sizes the launch grid      */
-    int32_t max_k_len;           /* host: >= every k_len[b], at most 262144             */
+    int32_t max_k_len;           /* host: >= every k_len[b], at most 262144 (262016
+                                    with key_order RETAINED_FIRST)                      */
     int32_t total_q_rows;        /* rows per layer of Q and O                           */
     int32_t total_k_rows;        /* rows per layer of K and V (and of role, seg_id)     */
     int64_t q_layer_stride;      /* elements between layers of Q                        */
@@ -172,6 +189,7 @@ typedef struct {
     int32_t *status;             /* device int32 or NULL                                */
     void *workspace;             /* device, sonic_prefill_workspace_size() bytes        */
     size_t workspace_bytes;
+    int32_t key_order;           /* sonic_key_order_t                                   */
 } sonic_prefill_args;
 
 /*
@@ -186,12 +204,25 @@ typedef struct {
  * Whole 128x128 key tiles the mask hides are skipped; the rule is applied per
  * element only on tiles it cuts.  Q, K, V, O are bf16; every row stride and
  * base pointer must be 16-byte aligned.  role and seg_id are indexed like the
- * key rows of one layer (shared by all layers).
+ * key rows of one layer (shared by all layers); role 255 marks a row that is
+ * no key (padding).  key_order picks the order the key tiles are cut in
+ * (sonic_key_order_t).  A sequence with q_len[b] > k_len[b] or k_len[b] >
+ * max_k_len is refused with SONIC_ERR_INVALID_ARGUMENT in *status.
  */
 SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
                                   const int32_t *seg_id, const uint8_t *role, uint16_t *O,
                                   const sonic_prefill_args *args, sonic_stream_t stream);
 
+/*
+ * Workspace bytes for sonic_attn_prefill with these arguments (0 for an empty
+ * batch).  AS_GIVEN: 32 bytes per 128-key tile, batch * ceil(max_k_len / 128)
+ * tiles.  RETAINED_FIRST adds, for R = min(batch * (align128(max_k_len) + 128),
+ * total_k_rows + 256 * batch) rows: 13 bytes of metadata per row and a K and
+ * a V copy of R rows for every layer (2 * n_layers * R * n_heads_kv *
+ * head_dim * 2 bytes).  Sequence b takes align128(k_len[b]) + 128 of the R
+ * rows; sequences that share key rows can need more than R, which the GPU
+ * reports as SONIC_ERR_WORKSPACE in *status.
+ */
 SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
 
 /*
@@ -205,7 +236,9 @@ SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
  * fixed 1 MiB array compiled into the library (every GPU that loads the
  * library holds it until the process exits).  It allocates nothing.
  *  - Limit: batch * ceil(max_k_len / 128) <= 32768; larger calls return
- *    SONIC_ERR_WORKSPACE before launching anything.
+ *    SONIC_ERR_WORKSPACE before launching anything.  Only key_order AS_GIVEN
+ *    is served (RETAINED_FIRST copies K and V into the workspace):
+ *    SONIC_ERR_UNSUPPORTED otherwise.
  *  - The first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress, with that device current) and caches it; make
  *    that first call before any stream capture.

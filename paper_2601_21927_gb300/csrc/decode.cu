@@ -553,10 +553,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             const int jj = (r & 63) >> 3;
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
-                const float pr = ex2(sv[g] - m[g]);
-                l[g] = l[g] * alpha[g] + pr;
-                *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) =
-                    __float2bfloat16_rn(pr);
+                // the row sum adds the rounded probability P.V multiplies by
+                const __nv_bfloat16 pr = __float2bfloat16_rn(ex2(sv[g] - m[g]));
+                l[g] = l[g] * alpha[g] + __bfloat162float(pr);
+                *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) = pr;
             }
             if (!valid) {
                 // V rows past the keys: zero, so 0 * garbage cannot reach O

@@ -19,6 +19,8 @@
 // classified from precomputed per-tile summaries (which roles and segment
 // numbers occur in it) as hidden (skipped entirely), fully visible (no mask
 // work) or cut by the mask.  The two tiles' softmax and MMAs interleave.
+#include <algorithm>
+
 #include "sonic_dev.cuh"
 #include "sonic_host.h"
 
@@ -39,22 +41,28 @@ struct TileSum {
     int32_t bseg_max;
     int32_t nseg_min;  // segment range of the Nexus rows
     int32_t nseg_max;
-    int32_t n_rows;    // rows of the tile inside the sequence
-    int32_t pad0, pad1;
+    int32_t n_rows;    // valid key rows in the tile (a prefix of its 128 rows)
+    int32_t pos_min;   // S_aug position range of the valid rows
+    int32_t pos_max;
 };
 
+// Key rows with role 255 are padding (no key): they count as invalid.
+// `pos` gives each key row's S_aug position (NULL: the row index itself).
 __global__ void __launch_bounds__(128)
 tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
-                    const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
-                    TileSum *__restrict__ out, int max_k_tiles) {
+                    const int32_t *__restrict__ pos, const int32_t *__restrict__ k_start,
+                    const int32_t *__restrict__ k_len, TileSum *__restrict__ out,
+                    int max_k_tiles) {
     const int t = blockIdx.x, b = blockIdx.y;
     const int len = k_len[b];
     if (t * kBN >= len && t > 0) return;
     const int r = t * kBN + threadIdx.x;
     int flags = 0, bmin = INT_MAX, bmax = INT_MIN, nmin = INT_MAX, nmax = INT_MIN, n = 0;
-    if (r < len) {
-        const int ro = role[k_start[b] + r];
+    int pmin = INT_MAX, pmax = INT_MIN;
+    const int ro = r < len ? role[k_start[b] + r] : 255;
+    if (ro != 255) {
         const int s = seg[k_start[b] + r];
+        pmin = pmax = pos ? pos[k_start[b] + r] : r;
         n = 1;
         if (ro == SONIC_ROLE_BODY) {
             flags = 1;
@@ -74,8 +82,10 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
         nmin = min(nmin, __shfl_xor_sync(0xffffffffu, nmin, o));
         nmax = max(nmax, __shfl_xor_sync(0xffffffffu, nmax, o));
         n += __shfl_xor_sync(0xffffffffu, n, o);
+        pmin = min(pmin, __shfl_xor_sync(0xffffffffu, pmin, o));
+        pmax = max(pmax, __shfl_xor_sync(0xffffffffu, pmax, o));
     }
-    __shared__ int sh[4][6];
+    __shared__ int sh[4][8];
     const int w = threadIdx.x >> 5;
     if ((threadIdx.x & 31) == 0) {
         sh[w][0] = flags;
@@ -84,6 +94,8 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
         sh[w][3] = nmin;
         sh[w][4] = nmax;
         sh[w][5] = n;
+        sh[w][6] = pmin;
+        sh[w][7] = pmax;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -94,6 +106,8 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
         ts.nseg_min = INT_MAX;
         ts.nseg_max = INT_MIN;
         ts.n_rows = 0;
+        ts.pos_min = INT_MAX;
+        ts.pos_max = INT_MIN;
         for (int i = 0; i < 4; ++i) {
             ts.flags |= sh[i][0];
             ts.bseg_min = min(ts.bseg_min, sh[i][1]);
@@ -101,20 +115,28 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
             ts.nseg_min = min(ts.nseg_min, sh[i][3]);
             ts.nseg_max = max(ts.nseg_max, sh[i][4]);
             ts.n_rows += sh[i][5];
+            ts.pos_min = min(ts.pos_min, sh[i][6]);
+            ts.pos_max = max(ts.pos_max, sh[i][7]);
         }
         out[(int64_t)b * max_k_tiles + t] = ts;
     }
 }
 
 struct PfParams {
+    // query side: the sequences as given (S_aug order)
     const int32_t *k_start, *k_len, *q_start, *q_len;
     const uint8_t *role;
     const int32_t *seg;
+    // key side: the same arrays, or their retained-first permutation
+    const int32_t *key_start, *key_len;
+    const uint8_t *key_role;
+    const int32_t *key_seg;
+    const int32_t *key_pos;  // S_aug position of each key row; NULL: the row index
     uint16_t *O;
     float *lse;
     int32_t *status;
     const TileSum *sums;
-    int max_k_tiles;
+    int max_k_tiles, max_k_len;
     int B, Hq, G;
     int64_t o_ls;
     int total_q_rows;
@@ -133,7 +155,8 @@ struct PfCfg {
     static constexpr int kOffMask = kOffV + 2 * kKVBytes;     // [2] TileMasks
     static constexpr int kOffRole = kOffMask + 2 * 256;       // [2][128] uint8
     static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
-    static constexpr int kOffList = kOffSeg + 2 * kBN * 4;    // [kMaxKTiles] int32
+    static constexpr int kOffPos = kOffSeg + 2 * kBN * 4;     // [2][128] int32
+    static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [kMaxKTiles] int32
     static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
     static constexpr int kNumBars = 16;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 32 ints
@@ -144,17 +167,38 @@ struct PfCfg {
 // Column masks of one 128-key tile (bit c of word w = key 32 w + c of the
 // tile): keys that are not body rows (nb), Nexus keys (nx), and the keys of
 // each distinct segment among the body keys (bm) and among the Nexus keys
-// (nm, used by the causal-segments reading).  With them a row's visibility
-// mask costs a few word operations.  More than four distinct segments in
-// one tile (not produced by valid layouts of reasonable segment length)
-// sets `fallback` and the rule is evaluated per key instead.
+// (nm, used by the causal-segments reading); and the valid keys as runs of
+// consecutive S_aug positions (a tile's valid keys are a prefix of its rows
+// with increasing positions, so the keys at or before a position form a
+// prefix too, whose length the runs give).  With them a row's visibility
+// mask costs a few word operations.  More than four distinct segments or
+// position runs in one tile set `fallback`: the rule is then evaluated per
+// key instead.
 struct TileMasks {
     uint32_t nb[4], nx[4];
-    int32_t nbody, nnex, fallback, pad;
+    int32_t nbody, nnex, fallback, nrun;
     int32_t bseg[4], nseg[4];
     uint32_t bm[4][4], nm[4][4];
+    // the valid keys as runs of consecutive S_aug positions, in column order
+    int32_t rpos[4], rlen[4];
 };
 static_assert(sizeof(TileMasks) <= 256, "tile masks");
+
+// Column of the n-th (from 0) set bit of a 128-bit mask, or -1.
+__device__ __forceinline__ int nth_set_bit(const uint32_t m[4], int n) {
+    int col = -1;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const int c = __popc(m[w]);
+        if (col < 0 && n < c) {
+            uint32_t x = m[w];
+            for (int i = 0; i < n; ++i) x &= x - 1;
+            col = w * 32 + __ffs(x) - 1;
+        }
+        if (col < 0) n -= c;
+    }
+    return col;
+}
 
 __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, int sq,
                                         int mode) {
@@ -178,7 +222,7 @@ constexpr float kRescaleThreshold = 8.0f;
 // TMEM (512 columns): S/P of tile 0 at 0, of tile 1 at 128, O of tile 0 at
 // 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns
 // of its S block and feeds O += P V straight from tensor memory.
-template <int D>
+template <int D, bool kLse>
 __global__ void __launch_bounds__(kPfThreads, 1)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const PfParams p) {
@@ -192,6 +236,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     TileMasks *tmasks = reinterpret_cast<TileMasks *>(smem + C::kOffMask);
     uint8_t *meta_role = smem + C::kOffRole;
     int32_t *meta_seg = reinterpret_cast<int32_t *>(smem + C::kOffSeg);
+    int32_t *meta_pos = reinterpret_cast<int32_t *>(smem + C::kOffPos);
     int32_t *list = reinterpret_cast<int32_t *>(smem + C::kOffList);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
     uint64_t *q_full = bars + 0;
@@ -210,12 +255,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
     const int klen = p.k_len[b], qlen = p.q_len[b];
     if (qt * 2 * kBM >= qlen || timed_out(p.status)) return;
-    if (qlen > klen || klen > p.max_k_tiles * kBN) {
+    // key side (kk*): the rows the tiles are cut from; k*: the S_aug sequence
+    const int kklen = p.key_len[b];
+    if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
         // the host-side bounds were wrong for this sequence: refuse it
         if (threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
         return;
     }
-    const int kstart = p.k_start[b];
+    const int kstart = p.k_start[b], kkstart = p.key_start[b];
     const int kvh = h / p.G;
     const int pbase = klen - qlen + qt * 2 * kBM;  // position of query row 0 of tile 0
     const bool tile1 = qt * 2 * kBM + kBM < qlen;   // tile 1 has rows
@@ -240,7 +287,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
     // ------------------------------------------------ key tiles to visit
     // list entry: (tile << 2) | (tile 0 needs the mask) | (tile 1 needs it) << 1
-    const int n_kt = (klen + kBN - 1) / kBN;
+    const int n_kt = (kklen + kBN - 1) / kBN;
     int n_list = 0;
     for (int c0 = 0; c0 < n_kt; c0 += kPfThreads) {
         const int t = c0 + tid;
@@ -248,7 +295,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         bool keep = false;
         if (t < n_kt) {
             const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
-            const int k0 = t * kBN, k1 = k0 + ts.n_rows - 1;
+            const int k0 = ts.pos_min, k1 = ts.pos_max;  // S_aug positions of the keys
             const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
             for (int qi = 0; qi < 2; ++qi) {
                 const int p0 = pbase + qi * kBM;
@@ -329,7 +376,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // K/V copies first; the key metadata is built while they are in flight
             if (lane == 0) {
                 mbar_expect_tx(&kv_full[st], 2 * C::kKVBytes);
-                const int row = kstart + kt * kBN;
+                const int row = kkstart + kt * kBN;
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh) {
                     tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), &tmK, &kv_full[st],
@@ -338,16 +385,16 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                 hh * 64, kvh, row, layer);
                 }
             }
-            // Roles / segments of the tile's keys (lane = key within each
-            // 32-key word; 255 marks rows past the sequence) and their masks:
-            // needed only where a query tile is cut by the mask.
+            // Roles / segments / S_aug positions of the tile's keys (lane = key
+            // within each 32-key word; role 255 marks padding and rows past the
+            // sequence) and their masks: needed only where a query tile is cut.
             if ((list[i] & 3) == 0) {
                 mbar_arrive(&kv_full[st]);
                 continue;
             }
-            int ro[4], sg[4];
-            uint32_t bst[4], nst[4];
-            int pro = 255, psg = 0;
+            int ro[4], sg[4], ps[4];
+            uint32_t bst[4], nst[4], rst[4];
+            int pro = 255, psg = 0, pps = INT_MIN, n_valid = 0;
             TileMasks &tm = tmasks[st];
 #pragma unroll
             for (int w = 0; w < 4; ++w) {
@@ -355,32 +402,45 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const int q = kt * kBN + c;
                 ro[w] = 255;
                 sg[w] = 0;
-                if (q < klen) {
-                    ro[w] = p.role[kstart + q];
-                    sg[w] = p.seg[kstart + q];
+                ps[w] = INT_MAX;
+                if (q < kklen) {
+                    ro[w] = p.key_role[kkstart + q];
+                    if (ro[w] != 255) {
+                        sg[w] = p.key_seg[kkstart + q];
+                        ps[w] = p.key_pos != nullptr ? p.key_pos[kkstart + q] : q;
+                    }
                 }
                 meta_role[st * kBN + c] = (uint8_t)ro[w];
                 meta_seg[st * kBN + c] = sg[w];
+                meta_pos[st * kBN + c] = ps[w];
+                const bool valid = ro[w] != 255;
                 const bool isb = ro[w] == SONIC_ROLE_BODY, isn = ro[w] == SONIC_ROLE_NEXUS;
-                const uint32_t nbw = __ballot_sync(0xffffffffu, ro[w] != 255 && !isb);
+                const uint32_t nbw = __ballot_sync(0xffffffffu, valid && !isb);
                 const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
-                // previous key's role/segment (lane 0: last key of the previous word)
+                n_valid += __popc(__ballot_sync(0xffffffffu, valid));
+                // previous key's role/segment/position (lane 0: last key of the
+                // previous word)
                 int r_up = __shfl_up_sync(0xffffffffu, ro[w], 1);
                 int s_up = __shfl_up_sync(0xffffffffu, sg[w], 1);
+                int p_up = __shfl_up_sync(0xffffffffu, ps[w], 1);
                 if (lane == 0) {
                     r_up = pro;
                     s_up = psg;
+                    p_up = pps;
                 }
                 bst[w] = __ballot_sync(0xffffffffu, isb && !(r_up == SONIC_ROLE_BODY && s_up == sg[w]));
                 nst[w] = __ballot_sync(0xffffffffu, isn && !(r_up == SONIC_ROLE_NEXUS && s_up == sg[w]));
+                rst[w] = __ballot_sync(0xffffffffu, valid && p_up != ps[w] - 1);
                 pro = __shfl_sync(0xffffffffu, ro[w], 31);
                 psg = __shfl_sync(0xffffffffu, sg[w], 31);
+                pps = __shfl_sync(0xffffffffu, ps[w], 31);
                 if (lane == 0) {
                     tm.nb[w] = nbw;
                     tm.nx[w] = nxw;
                 }
             }
-            // distinct segments of body runs and Nexus runs (in key order)
+            // distinct segments of body runs and Nexus runs, and the position
+            // runs (all in key order)
             int nb_n = 0, nn_n = 0, fb = 0;
             int bsv[4] = {0, 0, 0, 0}, nsv[4] = {0, 0, 0, 0};
 #pragma unroll
@@ -426,12 +486,21 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (lane == 0) {
                 tm.nbody = nb_n;
                 tm.nnex = nn_n;
-                tm.fallback = fb;
+                tm.nrun = __popc(rst[0]) + __popc(rst[1]) + __popc(rst[2]) + __popc(rst[3]);
+                tm.fallback = fb | (tm.nrun > 4);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     tm.bseg[k] = bsv[k];
                     tm.nseg[k] = nsv[k];
                 }
+            }
+            // position run k (lane k < 4): from the k-th run start to the next
+            // one (or to the last valid key); the start's position from smem
+            __syncwarp();
+            if (lane < 4) {
+                const int c0 = nth_set_bit(rst, lane), c1 = nth_set_bit(rst, lane + 1);
+                tm.rpos[lane] = c0 < 0 ? 0 : meta_pos[st * kBN + c0];
+                tm.rlen[lane] = c0 < 0 ? 0 : (c1 < 0 ? n_valid : c1) - c0;
             }
             __syncwarp();
             mbar_arrive(&kv_full[st]);  // 32 arrivals + the copies' bytes end the phase
@@ -516,7 +585,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
         const uint32_t tS = tmem + lane_base + qi * kBN;
         const uint32_t tO = tmem + lane_base + 256 + qi * 128;
-        float m_used = -INFINITY, l = 0.f;
+        // l: sum of the rounded probabilities (normalises O); l_lse: of the
+        // unrounded ones, for the log-sum-exp output (kLse: lse requested)
+        float m_used = -INFINITY, l = 0.f, l_lse = 0.f;
         bool ok = true;
         // the next list entry is read one tile ahead: shared memory is busy
         // feeding the tensor cores, so a load on the critical path is slow
@@ -561,9 +632,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     nm[k] = tv[9 + k];
                 }
                 if (!hd.z) {
-                    // causal prefix (keys at or before this row), body keys of this
-                    // row's segment, and the Nexus keys a Nexus row sees
-                    const int nvis = pos - kt * kBN + 1;
+                    // causal prefix (keys at or before this row: a prefix of the
+                    // tile's columns, counted over the position runs), body keys of
+                    // this row's segment, and the Nexus keys a Nexus row sees
+                    const uint4 rp4 = tv[13], rl4 = tv[14];
+                    const int nvis = min(max(pos - (int)rp4.x + 1, 0), (int)rl4.x) +
+                                     min(max(pos - (int)rp4.y + 1, 0), (int)rl4.y) +
+                                     min(max(pos - (int)rp4.z + 1, 0), (int)rl4.z) +
+                                     min(max(pos - (int)rp4.w + 1, 0), (int)rl4.w);
                     const int nbody = (int)hd.x, nnex = (int)hd.y;
                     const int bs4[4] = {(int)bsg.x, (int)bsg.y, (int)bsg.z, (int)bsg.w};
                     const int ns4[4] = {(int)nsg.x, (int)nsg.y, (int)nsg.z, (int)nsg.w};
@@ -593,12 +669,13 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     for (int c = 0; c < 4; ++c) {
                         const uint8_t *mr = meta_role + st * kBN + c * 32;
                         const int32_t *ms = meta_seg + st * kBN + c * 32;
+                        const int32_t *mp = meta_pos + st * kBN + c * 32;
                         uint32_t bits = 0;
 #pragma unroll 4
                         for (int e = 0; e < 32; ++e) {
                             const int rq = mr[e];
-                            const bool v = rq != 255 && visible(pos, kt * kBN + c * 32 + e, rp,
-                                                                sp, rq, ms[e], p.nexus_mode);
+                            const bool v = rq != 255 &&
+                                           visible(pos, mp[e], rp, sp, rq, ms[e], p.nexus_mode);
                             bits |= (v ? 1u : 0u) << e;
                         }
                         mbits[c] = bits;
@@ -625,6 +702,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
             const float2 nm2 = make_float2(-mref, -mref);
             float2 rs2a = make_float2(0.f, 0.f), rs2b = make_float2(0.f, 0.f);
+            float2 rs2x = make_float2(0.f, 0.f);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 uint32_t pk[16];
@@ -633,16 +711,25 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     const float2 x = __ffma2_rn(
                         make_float2(__uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1])), sc2,
                         nm2);
-                    const float2 ev = make_float2(ex2(x.x), ex2(x.y));
+                    const float2 eu = make_float2(ex2(x.x), ex2(x.y));
+                    if (kLse) rs2x = __fadd2_rn(rs2x, eu);
+                    const uint32_t pr = pack_bf16x2(eu.x, eu.y);
+                    pk[e >> 1] = pr;
+                    // the row sum adds the rounded probabilities P.V multiplies
+                    // by, so O is a weighted mean of V rows with weights summing
+                    // to one (rounding moves weight between keys, it does not
+                    // scale the output)
+                    const float2 ev = make_float2(__uint_as_float(pr << 16),
+                                                  __uint_as_float(pr & 0xffff0000u));
                     if ((e >> 1) & 1)
                         rs2b = __fadd2_rn(rs2b, ev);
                     else
                         rs2a = __fadd2_rn(rs2a, ev);
-                    pk[e >> 1] = pack_bf16x2(ev.x, ev.y);
                 }
                 tmem_st16(tS + c * 16, pk);
             }
             l = l * alpha + ((rs2a.x + rs2a.y) + (rs2b.x + rs2b.y));
+            if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
             // O rescale (PV of the previous tile is complete: S of this tile was
             // issued after it, and S is done)
             if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
@@ -661,7 +748,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tmem_st_wait();
             // Rows of V past the sequence end: zero them so 0 * garbage cannot
             // reach the accumulator (tile 0's warps; its PV is issued first).
-            if (qi == 0 && kt * kBN + kBN > klen && kt * kBN + r >= klen) {
+            if (qi == 0 && kt * kBN + kBN > kklen && kt * kBN + r >= kklen) {
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh) {
                     uint4 *vr = reinterpret_cast<uint4 *>(Vs + st * C::kKVBytes +
@@ -700,14 +787,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     }
                 }
             }
-            if (row_ok && p.lse != nullptr)
+            if (kLse && row_ok)
                 p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] =
-                    l > 0.f ? (m_used + __log2f(l)) * kLn2f : -INFINITY;
+                    l_lse > 0.f ? (m_used + __log2f(l_lse)) * kLn2f : -INFINITY;
         } else if (row_ok && n_list == 0) {
             const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
             uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
             for (int d = 0; d < D; ++d) orow[d] = 0;
-            if (p.lse != nullptr)
+            if (kLse)
                 p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = -INFINITY;
         }
     }
@@ -717,12 +804,177 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
+// ---------------------------------------------------------------- key order
+// Retained-first order.  Sequence b's keys are rewritten into rows
+// [key_start[b], key_start[b] + span_b) of the workspace, span_b =
+// align128(k_len[b]) + 128: first its retained keys (every role but body, in
+// S_aug order), padded to a 128-row boundary, then its body keys (S_aug
+// order), then padding to the end of the span.  Padding rows have role 255,
+// position INT_MAX and source -1 (their K/V rows are zeroed).  key_start has
+// B + 1 entries; the last is the number of rows written (every one of them
+// gets a source index, so the copy kernel reads no unwritten entry).
+constexpr int kOrderThreads = 1024;
+
+__device__ __forceinline__ int span_of(int len) { return (len + kBN - 1) / kBN * kBN + kBN; }
+
+// A k_len outside [0, max_k_len] is refused: the sequence gets no keys.
+__device__ __forceinline__ int checked_len(int len, int max_len) {
+    return (len < 0 || len > max_len) ? 0 : len;
+}
+
+__global__ void __launch_bounds__(kOrderThreads)
+key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
+                 const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len, int B,
+                 int max_k_len, int64_t capacity, int32_t *__restrict__ key_start,
+                 int32_t *__restrict__ key_len, uint8_t *__restrict__ o_role,
+                 int32_t *__restrict__ o_seg, int32_t *__restrict__ o_pos,
+                 int32_t *__restrict__ o_src, int32_t *__restrict__ status) {
+    const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __shared__ int sh[2][32];
+    __shared__ long long sh_base;
+    __shared__ int sh_r;
+    // start of this sequence's span: the spans of the sequences before it
+    long long base = 0;
+    for (int i = tid; i < b; i += kOrderThreads) base += span_of(checked_len(k_len[i], max_k_len));
+    if (tid == 0) {
+        sh_base = 0;
+        sh_r = 0;
+    }
+    __syncthreads();
+    if (base) atomicAdd(reinterpret_cast<unsigned long long *>(&sh_base), (unsigned long long)base);
+    const int len_in = k_len[b];
+    const int len = checked_len(len_in, max_k_len);
+    if (tid == 0 && len != len_in) set_status(status, SONIC_ERR_INVALID_ARGUMENT);
+    const int ks = k_start[b];
+    int cnt = 0;
+    for (int i = tid; i < len; i += kOrderThreads) cnt += role[ks + i] != SONIC_ROLE_BODY;
+    cnt = __reduce_add_sync(0xffffffffu, cnt);
+    if (lane == 0 && cnt) atomicAdd(&sh_r, cnt);
+    __syncthreads();
+    const long long start = sh_base;
+    const int R = sh_r, span = span_of(len);
+    if (b == B - 1 && tid == 0) key_start[B] = (int32_t)min(start + span, (long long)capacity);
+    if (start + span > capacity) {
+        // the spans overflow the workspace (sequences that share key rows can
+        // sum to more than total_k_rows): this sequence gets no keys, and the
+        // rows of its span that exist become padding
+        for (long long i = start + tid; i < capacity; i += kOrderThreads) {
+            o_role[i] = 255;
+            o_seg[i] = 0;
+            o_pos[i] = INT_MAX;
+            o_src[i] = -1;
+        }
+        if (tid == 0) {
+            set_status(status, SONIC_ERR_WORKSPACE);
+            key_start[b] = 0;
+            key_len[b] = 0;
+        }
+        return;
+    }
+    const int body0 = (R + kBN - 1) / kBN * kBN;
+    int kept = 0, bodies = 0;
+    for (int c0 = 0; c0 < len; c0 += kOrderThreads) {
+        const int i = c0 + tid;
+        const bool valid = i < len;
+        const int r = valid ? role[ks + i] : SONIC_ROLE_BODY;
+        const bool keep = valid && r != SONIC_ROLE_BODY, body = valid && r == SONIC_ROLE_BODY;
+        const unsigned bk = __ballot_sync(0xffffffffu, keep), bb = __ballot_sync(0xffffffffu, body);
+        if (lane == 0) {
+            sh[0][warp] = __popc(bk);
+            sh[1][warp] = __popc(bb);
+        }
+        __syncthreads();
+        int pk = 0, pb = 0, tk = 0, tb = 0;
+        for (int w = 0; w < kOrderThreads / 32; ++w) {
+            if (w < warp) {
+                pk += sh[0][w];
+                pb += sh[1][w];
+            }
+            tk += sh[0][w];
+            tb += sh[1][w];
+        }
+        const unsigned below = (1u << lane) - 1u;
+        if (valid) {
+            const int dst = keep ? kept + pk + __popc(bk & below) : body0 + bodies + pb + __popc(bb & below);
+            const int64_t o = start + dst;
+            o_role[o] = (uint8_t)r;
+            o_seg[o] = seg[ks + i];
+            o_pos[o] = i;
+            o_src[o] = ks + i;
+        }
+        kept += tk;
+        bodies += tb;
+        __syncthreads();
+    }
+    // padding: between the retained keys and the bodies, and after the bodies
+    const int lp = body0 + (len - R);
+    for (int i = tid; i < span; i += kOrderThreads) {
+        if ((i >= R && i < body0) || i >= lp) {
+            o_role[start + i] = 255;
+            o_seg[start + i] = 0;
+            o_pos[start + i] = INT_MAX;
+            o_src[start + i] = -1;
+        }
+    }
+    if (tid == 0) {
+        key_start[b] = (int32_t)start;
+        key_len[b] = lp;
+    }
+}
+
+// K and V rows of every layer into the retained-first order (warp per row;
+// rows with source -1 are zeroed).
+constexpr int kPermThreads = 256;
+
+__device__ __forceinline__ int4 ld_nc(const void *ptr) {
+    int4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(ptr));
+    return v;
+}
+
+__global__ void __launch_bounds__(kPermThreads)
+kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
+                  uint8_t *__restrict__ Kp, uint8_t *__restrict__ Vp,
+                  const int32_t *__restrict__ src, const int32_t *__restrict__ key_start, int B,
+                  int64_t row_bytes, int64_t in_layer_bytes, int64_t out_layer_bytes) {
+    const int layer = blockIdx.y >> 1;
+    const bool is_v = blockIdx.y & 1;
+    const uint8_t *in = (is_v ? V : K) + (int64_t)layer * in_layer_bytes;
+    uint8_t *out = (is_v ? Vp : Kp) + (int64_t)layer * out_layer_bytes;
+    const int64_t n_rows = key_start[B];
+    const int lane = threadIdx.x & 31;
+    const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int cpr = (int)(row_bytes >> 4);
+    for (int64_t r = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < n_rows;
+         r += n_warps) {
+        const int32_t s = src[r];
+        const uint8_t *pi = in + (int64_t)s * row_bytes;
+        uint8_t *po = out + r * row_bytes;
+        for (int c0 = lane; c0 < cpr; c0 += 32 * 4) {
+            int4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int c = c0 + 32 * u;
+                v[u] = make_int4(0, 0, 0, 0);
+                if (c < cpr && s >= 0) v[u] = ld_nc(pi + ((int64_t)c << 4));
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < cpr) *reinterpret_cast<int4 *>(po + ((int64_t)c << 4)) = v[u];
+            }
+        }
+    }
+}
+
 template <int D>
 cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
                            const PfParams &p, dim3 grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
-    auto kern = prefill_kernel<D>;
+    auto kern = p.lse != nullptr ? prefill_kernel<D, true> : prefill_kernel<D, false>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -731,7 +983,41 @@ cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const C
 }
 
 int max_k_tiles_of(const sonic_prefill_args *a) {
-    return (a->max_k_len + kBN - 1) / kBN;
+    const int t = (a->max_k_len + kBN - 1) / kBN;
+    return a->key_order == SONIC_KEYS_RETAINED_FIRST ? t + 1 : t;
+}
+
+// Workspace: tile summaries; with the retained-first order also the
+// permuted key metadata and the permuted K and V of every layer.
+struct PfWorkspace {
+    size_t sums, key_start, key_len, role, seg, pos, src, kp, vp, total;
+    int64_t rows;  // rows of the permuted K/V per layer
+};
+
+PfWorkspace workspace_layout(const sonic_prefill_args *a) {
+    PfWorkspace w{};
+    size_t off = round_up((size_t)a->batch * max_k_tiles_of(a) * sizeof(TileSum), 256);
+    if (a->key_order == SONIC_KEYS_RETAINED_FIRST) {
+        const int64_t span = (int64_t)((a->max_k_len + kBN - 1) / kBN) * kBN + kBN;
+        w.rows = std::min<int64_t>((int64_t)a->batch * span,
+                                   (int64_t)a->total_k_rows + (int64_t)2 * kBN * a->batch);
+        auto take = [&](size_t bytes) {
+            const size_t o = off;
+            off += round_up(bytes, 256);
+            return o;
+        };
+        w.key_start = take((size_t)(a->batch + 1) * 4);
+        w.key_len = take((size_t)a->batch * 4);
+        w.role = take((size_t)w.rows);
+        w.seg = take((size_t)w.rows * 4);
+        w.pos = take((size_t)w.rows * 4);
+        w.src = take((size_t)w.rows * 4);
+        const size_t layer = (size_t)w.rows * a->n_heads_kv * a->head_dim * 2;
+        w.kp = take(layer * a->n_layers);
+        w.vp = take(layer * a->n_layers);
+    }
+    w.total = off;
+    return w;
 }
 
 }  // namespace
@@ -741,7 +1027,10 @@ using namespace sonic;
 
 extern "C" size_t sonic_prefill_workspace_size(const sonic_prefill_args *a) {
     if (a == nullptr || a->batch <= 0 || a->max_k_len <= 0) return 0;
-    return round_up((size_t)a->batch * max_k_tiles_of(a) * sizeof(TileSum), 256);
+    if (a->key_order == SONIC_KEYS_RETAINED_FIRST &&
+        (a->n_layers < 1 || a->n_heads_kv < 1 || a->head_dim < 1 || a->total_k_rows < 0))
+        return 0;
+    return workspace_layout(a).total;
 }
 
 extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K,
@@ -764,6 +1053,9 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     if (D != 64 && D != 128) return SONIC_ERR_UNSUPPORTED;
     if (a->nexus_vis != SONIC_NEXUS_FULL && a->nexus_vis != SONIC_NEXUS_CAUSAL_SEGMENTS)
         return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->key_order != SONIC_KEYS_AS_GIVEN && a->key_order != SONIC_KEYS_RETAINED_FIRST)
+        return SONIC_ERR_INVALID_ARGUMENT;
+    const bool reorder = a->key_order == SONIC_KEYS_RETAINED_FIRST;
     if (a->max_k_len < a->max_q_len || a->total_k_rows == 0 || a->total_q_rows == 0)
         return SONIC_ERR_INVALID_ARGUMENT;
     if (max_k_tiles_of(a) > kMaxKTiles) return SONIC_ERR_UNSUPPORTED;
@@ -776,6 +1068,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         return SONIC_ERR_INVALID_ARGUMENT;
     const size_t need = sonic_prefill_workspace_size(a);
     if (a->workspace == nullptr || a->workspace_bytes < need) return SONIC_ERR_WORKSPACE;
+    if (reorder && workspace_layout(a).rows > (int64_t)0x7fffffff - kBN)
+        return SONIC_ERR_UNSUPPORTED;
     const long long qtiles = (a->max_q_len + 2 * kBM - 1) / (2 * kBM);
     if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_q > 65535 || qtiles > 0x7fffffff)
         return SONIC_ERR_UNSUPPORTED;
@@ -788,13 +1082,20 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     const uint64_t qd[4] = {(uint64_t)D, (uint64_t)a->n_heads_q, (uint64_t)a->total_q_rows,
                             (uint64_t)a->n_layers};
     const uint64_t qs[3] = {(uint64_t)D * 2, qrow * 2, q_layer};
-    const uint64_t kd[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_k_rows,
+    const PfWorkspace ws = workspace_layout(a);
+    uint8_t *wsb = static_cast<uint8_t *>(a->workspace);
+    // K/V rows the tiles are cut from: the inputs, or their permuted copies
+    const void *Kt = reorder ? (const void *)(wsb + ws.kp) : (const void *)K;
+    const void *Vt = reorder ? (const void *)(wsb + ws.vp) : (const void *)V;
+    const uint64_t kt_rows = reorder ? (uint64_t)ws.rows : (uint64_t)a->total_k_rows;
+    const uint64_t kt_layer = reorder ? (uint64_t)ws.rows * krow * 2 : k_layer;
+    const uint64_t kd[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, kt_rows,
                             (uint64_t)a->n_layers};
-    const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, k_layer};
+    const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, kt_layer};
     const uint32_t box[4] = {64, 1, 128, 1};
     CUtensorMap tq, tk, tv;
-    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, box) || !make_tmap_bf16_4d(&tk, K, kd, ks, box) ||
-        !make_tmap_bf16_4d(&tv, V, kd, ks, box))
+    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, box) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
+        !make_tmap_bf16_4d(&tv, Vt, kd, ks, box))
         return SONIC_ERR_INVALID_ARGUMENT;
 
     PfParams p{};
@@ -804,11 +1105,24 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.q_len = a->q_len;
     p.role = role;
     p.seg = seg_id;
+    p.key_start = a->k_start;
+    p.key_len = a->k_len;
+    p.key_role = role;
+    p.key_seg = seg_id;
+    p.key_pos = nullptr;
+    if (reorder) {
+        p.key_start = reinterpret_cast<const int32_t *>(wsb + ws.key_start);
+        p.key_len = reinterpret_cast<const int32_t *>(wsb + ws.key_len);
+        p.key_role = wsb + ws.role;
+        p.key_seg = reinterpret_cast<const int32_t *>(wsb + ws.seg);
+        p.key_pos = reinterpret_cast<const int32_t *>(wsb + ws.pos);
+    }
     p.O = O;
     p.lse = a->lse;
     p.status = a->status;
     p.sums = static_cast<const TileSum *>(a->workspace);
     p.max_k_tiles = max_k_tiles_of(a);
+    p.max_k_len = a->max_k_len;
     p.B = a->batch;
     p.Hq = a->n_heads_q;
     p.G = a->n_heads_q / a->n_heads_kv;
@@ -818,8 +1132,24 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.scale_log2 = scale * kLog2ef;
     p.nexus_mode = a->nexus_vis;
 
+    if (reorder) {
+        key_order_kernel<<<a->batch, kOrderThreads, 0, stream>>>(
+            role, seg_id, a->k_start, a->k_len, a->batch, a->max_k_len, ws.rows,
+            reinterpret_cast<int32_t *>(wsb + ws.key_start),
+            reinterpret_cast<int32_t *>(wsb + ws.key_len), wsb + ws.role,
+            reinterpret_cast<int32_t *>(wsb + ws.seg), reinterpret_cast<int32_t *>(wsb + ws.pos),
+            reinterpret_cast<int32_t *>(wsb + ws.src), a->status);
+        const int sms = device_sm_count();
+        const int per_slice = std::max(1, (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers));
+        kv_permute_kernel<<<dim3(per_slice, 2 * a->n_layers), kPermThreads, 0, stream>>>(
+            reinterpret_cast<const uint8_t *>(K), reinterpret_cast<const uint8_t *>(V),
+            wsb + ws.kp, wsb + ws.vp, reinterpret_cast<const int32_t *>(wsb + ws.src),
+            reinterpret_cast<const int32_t *>(wsb + ws.key_start), a->batch, (int64_t)krow * 2,
+            (int64_t)k_layer, (int64_t)kt_layer);
+    }
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
-        role, seg_id, a->k_start, a->k_len, static_cast<TileSum *>(a->workspace), p.max_k_tiles);
+        p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
+        static_cast<TileSum *>(a->workspace), p.max_k_tiles);
     dim3 grid((unsigned)qtiles, a->n_heads_q, a->batch * a->n_layers);
     cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
                                : launch_prefill<64>(tq, tk, tv, p, grid, stream);

@@ -55,6 +55,8 @@ extern "C" sonic_status_t sonic_attn_prefill_static(const uint16_t *Q, const uin
                                                     const sonic_prefill_args *args,
                                                     sonic_stream_t stream) {
     if (args == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
+    // the retained-first order copies K and V into the workspace: not here
+    if (args->key_order != SONIC_KEYS_AS_GIVEN) return SONIC_ERR_UNSUPPORTED;
     sonic_prefill_args a = *args;
     a.workspace = nullptr;
     a.workspace_bytes = 0;

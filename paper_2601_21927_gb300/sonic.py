@@ -25,6 +25,7 @@ from . import _build
 
 ROLE_SYS, ROLE_BODY, ROLE_NEXUS, ROLE_CURR = 0, 1, 2, 3
 NEXUS_FULL, NEXUS_CAUSAL_SEGMENTS = 0, 1
+KEYS_AS_GIVEN, KEYS_RETAINED_FIRST = 0, 1
 
 STATUS = {0: "SONIC_OK", 1: "SONIC_ERR_INVALID_ARGUMENT", 2: "SONIC_ERR_UNSUPPORTED",
           3: "SONIC_ERR_WORKSPACE", 4: "SONIC_ERR_CAPACITY", 5: "SONIC_ERR_DEVICE_TIMEOUT",
@@ -54,7 +55,8 @@ class sonic_prefill_args(ctypes.Structure):
                 ("q_len", _P), ("max_q_len", _i32), ("max_k_len", _i32), ("total_q_rows", _i32),
                 ("total_k_rows", _i32), ("q_layer_stride", _i64), ("kv_layer_stride", _i64),
                 ("o_layer_stride", _i64), ("softmax_scale", _f32), ("nexus_vis", _i32),
-                ("lse", _P), ("status", _P), ("workspace", _P), ("workspace_bytes", _sz)]
+                ("lse", _P), ("status", _P), ("workspace", _P), ("workspace_bytes", _sz),
+                ("key_order", _i32)]
 
 
 class sonic_decode_args(ctypes.Structure):
@@ -177,7 +179,7 @@ def sonic_attn_prefill(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, seg_id
                        role: torch.Tensor, O: torch.Tensor, *, k_start, k_len, q_start, q_len,
                        max_q_len: int, max_k_len: int, softmax_scale: float = 0.0,
                        nexus_vis: int = NEXUS_FULL, lse=None, status=None, workspace=None,
-                       stream=None):
+                       key_order: int = KEYS_AS_GIVEN, stream=None):
     """Masked prefill.  Q, O: [n_layers, Tq, Hq, D] bf16; K, V: [n_layers, Tk, Hkv, D] bf16."""
     lib = load()
     nl, tq, hq, d = Q.shape
@@ -191,6 +193,7 @@ def sonic_attn_prefill(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, seg_id
     a.q_layer_stride, a.kv_layer_stride, a.o_layer_stride = Q.stride(0), K.stride(0), O.stride(0)
     a.softmax_scale, a.nexus_vis = softmax_scale, nexus_vis
     a.lse, a.status = _ptr(lse), _ptr(status)
+    a.key_order = key_order
     need = lib.sonic_prefill_workspace_size(ctypes.byref(a))
     ws = _workspace(need, Q.device, workspace)
     a.workspace, a.workspace_bytes = _ptr(ws), need

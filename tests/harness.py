@@ -43,11 +43,13 @@ def check_close(got: np.ndarray, want: np.ndarray, what: str):
 
 def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed: int = 0,
                 nexus_vis: int = sonic.NEXUS_FULL, n_layers: int = 1, with_lse: bool = True,
-                K=None, V=None, Q=None):
+                K=None, V=None, Q=None, key_order: int = sonic.KEYS_AS_GIVEN,
+                expect_status: int = 0, k_start=None, total_k_rows=None):
     """Prefill of the last q_len[b] rows of every sequence (all rows if None).
     Returns a dict with the device tensors and the query layout."""
-    role, seg, k_start, k_len = meta(batch)
-    T = batch.total
+    role, seg, k_start_b, k_len = meta(batch)
+    k_start = k_start_b if k_start is None else i32(k_start)
+    T = batch.total if total_k_rows is None else total_k_rows
     if q_len is None:
         q_len = batch.k_len.copy()
     q_len = np.asarray(q_len, dtype=np.int32)
@@ -64,9 +66,9 @@ def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed
     sonic.sonic_attn_prefill(Q, K, V, seg, role, O, k_start=k_start, k_len=k_len,
                              q_start=i32(q_start), q_len=i32(q_len),
                              max_q_len=int(q_len.max()), max_k_len=int(batch.k_len.max()),
-                             nexus_vis=nexus_vis, lse=lse, status=status)
+                             nexus_vis=nexus_vis, lse=lse, status=status, key_order=key_order)
     torch.cuda.synchronize()
-    assert sonic.read_status(status) == 0
+    assert sonic.read_status(status) == expect_status
     return dict(K=K, V=V, Q=Q, O=O, lse=lse, q_len=q_len, q_start=q_start)
 
 

@@ -82,6 +82,12 @@ def test_host_validation_rejects_before_launch():
     p.nexus_vis = 0
     assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 3  # workspace
     assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256
+    p.key_order = 7
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 1
+    # the fixed-scratch entry point serves only the as-given key order
+    p.key_order = sonic.KEYS_RETAINED_FIRST
+    assert lib.sonic_attn_prefill_static(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 2
+    p.key_order = sonic.KEYS_AS_GIVEN
 
     d = sonic.sonic_decode_args()
     d.batch, d.n_layers, d.n_heads_q, d.n_heads_kv, d.head_dim = 2, 1, 40, 2, 128
@@ -101,3 +107,31 @@ def test_python_binding_has_no_cpu_path():
         if f.endswith(".py"):
             t = open(os.path.join(ROOT, "paper_2601_21927_gb300", f)).read()
             assert "oracle" not in re.findall(r"^\s*(?:import|from)\s+(\w+)", t, re.M), f
+
+
+def test_retained_first_workspace_size():
+    """Workspace of the retained-first order: tile summaries of one extra tile
+    per sequence, 13 bytes of metadata per permuted row, and a K and a V copy
+    of every layer; each part rounded up to 256 bytes."""
+    lib = sonic.load()
+    p = sonic.sonic_prefill_args()
+    p.batch, p.n_layers, p.n_heads_q, p.n_heads_kv, p.head_dim = 2, 3, 8, 4, 128
+    p.max_q_len, p.max_k_len, p.total_q_rows, p.total_k_rows = 300, 300, 600, 600
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256  # 2 * 3 tiles * 32 B
+    p.key_order = sonic.KEYS_RETAINED_FIRST
+
+    def r256(x):
+        return (x + 255) // 256 * 256
+
+    def expect(rows):
+        return (r256(2 * 4 * 32) + r256(3 * 4) + r256(2 * 4) + r256(rows) + 3 * r256(4 * rows)
+                + 2 * r256(3 * rows * 4 * 128 * 2))
+
+    # spans of 384 + 128 rows per sequence, below total_k_rows + 256 per sequence
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == expect(1024)
+    p.total_k_rows = 300  # two sequences sharing rows: capped at 300 + 512
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == expect(812)
+    p.max_k_len = 2047 * 128 + 1  # one extra tile past the 2048-tile list
+    p.total_k_rows = p.max_k_len
+    p.k_start = p.k_len = p.q_start = p.q_len = 16
+    assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 2

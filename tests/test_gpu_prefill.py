@@ -10,8 +10,11 @@ from tests import harness as H
 pytestmark = pytest.mark.gpu
 
 
-def _all_rows(batch, hq, hkv, D, mode=sonic.NEXUS_FULL, seed=0):
-    res = H.run_prefill(batch, hq, hkv, D, seed=seed, nexus_vis=mode)
+ORDERS = [sonic.KEYS_AS_GIVEN, sonic.KEYS_RETAINED_FIRST]
+
+
+def _all_rows(batch, hq, hkv, D, mode=sonic.NEXUS_FULL, seed=0, order=sonic.KEYS_AS_GIVEN):
+    res = H.run_prefill(batch, hq, hkv, D, seed=seed, nexus_vis=mode, key_order=order)
     for b in range(batch.B):
         n = int(batch.k_len[b])
         O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, np.arange(n), nexus_vis=mode)
@@ -19,27 +22,100 @@ def _all_rows(batch, hq, hkv, D, mode=sonic.NEXUS_FULL, seed=0):
         np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
 
 
-def test_tiny_reference_all_rows():
+@pytest.mark.parametrize("order", ORDERS)
+def test_tiny_reference_all_rows(order):
     batch, hd = inputs.tiny_ref()
-    _all_rows(batch, hd.hq, hd.hkv, hd.d)
+    _all_rows(batch, hd.hq, hd.hkv, hd.d, order=order)
 
 
+@pytest.mark.parametrize("order", ORDERS)
 @pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
-def test_random_dialogues_multi_tile(mode):
+def test_random_dialogues_multi_tile(mode, order):
     rng = np.random.default_rng(11)
     ds = [inputs.random_dialogue(rng, max_segments=6, max_body=120, max_nexus=40, max_sys=90,
                                  max_curr=150) for _ in range(4)]
     ds.append(inputs.Dialogue(5, [(300, 0), (1, 1), (0, 70)], 1))  # K_i = 0, tiny pieces
-    _all_rows(inputs.Batch(ds), 4, 2, 128, mode=mode, seed=5)
+    _all_rows(inputs.Batch(ds), 4, 2, 128, mode=mode, seed=5, order=order)
 
 
-def test_head_dim_64_and_gqa_ratios():
+@pytest.mark.parametrize("order", ORDERS)
+def test_head_dim_64_and_gqa_ratios(order):
     rng = np.random.default_rng(3)
     ds = [inputs.random_dialogue(rng, max_segments=4, max_body=200, max_nexus=30) for _ in range(3)]
-    _all_rows(inputs.Batch(ds), 6, 2, 64, seed=9)
+    _all_rows(inputs.Batch(ds), 6, 2, 64, seed=9, order=order)
 
 
-def test_current_turn_over_compacted_cache():
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+def test_retained_first_many_runs_per_tile(mode):
+    """Short segments: a 128-key tile of the retained part holds more than four
+    runs of consecutive positions (Nexus groups of 3-6 tokens), and a body tile
+    more than four segments, so both take the per-key mask path."""
+    ds = [inputs.Dialogue(30, [(20, 5)] * 40, 100),
+          inputs.Dialogue(3, [(9, 3), (7, 6), (11, 4)] * 12, 37),
+          inputs.Dialogue(128, [(128, 128)] * 3, 128)]  # tile-aligned everything
+    _all_rows(inputs.Batch(ds), 4, 1, 128, mode=mode, seed=13, order=sonic.KEYS_RETAINED_FIRST)
+
+
+@pytest.mark.parametrize("order", ORDERS)
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+def test_uniform_scores_count_visible_keys(mode, order):
+    """Q = 0 makes every visible score 0 and every probability exactly 1, so
+    the GPU's lse is ln |vis(p)| up to fp32 rounding; one key missing or extra
+    in any row moves it by about 1 / |vis(p)|.  An exact check of the mask on
+    every row, both readings and both key orders."""
+    rng = np.random.default_rng(23)
+    ds = [inputs.random_dialogue(rng, max_segments=6, max_body=150, max_nexus=40, max_sys=90,
+                                 max_curr=150) for _ in range(4)]
+    ds += [inputs.Dialogue(30, [(20, 5)] * 40, 100), inputs.Dialogue(0, [(300, 0), (1, 1)], 2)]
+    batch = inputs.Batch(ds)
+    Q = torch.zeros((1, batch.total, 4, 128), dtype=torch.bfloat16, device=H.dev())
+    res = H.run_prefill(batch, 4, 2, 128, seed=29, nexus_vis=mode, key_order=order, Q=Q)
+    for b in range(batch.B):
+        n = int(batch.k_len[b])
+        O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, np.arange(n), nexus_vis=mode)
+        np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-5, err_msg=f"seq {b}")
+        H.check_close(got, O, f"seq {b}")
+
+
+def test_retained_first_sequences_sharing_key_rows():
+    """Two sequences over the same key rows (a shared history, different query
+    blocks): each gets its own span of the permuted copy.  The key tensor has
+    2 * 560 rows (the second half unused), so the workspace bound of
+    total_k_rows + 256 rows per sequence holds both spans of 768 rows."""
+    d = inputs.Dialogue(50, [(120, 40), (200, 60)], 90)
+    batch = inputs.Batch([d, d])
+    kl = int(batch.k_len[0])
+    res = H.run_prefill(batch, 4, 2, 128, seed=17, key_order=sonic.KEYS_RETAINED_FIRST,
+                        k_start=[0, 0], total_k_rows=2 * kl)
+    shared = inputs.Batch([d])
+    for b in range(2):
+        # both sequences read key rows [0, kl) of the same K, V, role, seg
+        O, lse, got, got_lse = H.oracle_prefill_rows(
+            shared, dict(res, q_len=res["q_len"][b:b + 1], q_start=res["q_start"][b:b + 1]),
+            0, np.arange(kl))
+        H.check_close(got, O, f"seq {b}")
+
+
+def test_retained_first_workspace_overflow_is_reported():
+    """Three sequences sharing 1,100 key rows need more permuted rows than the
+    workspace bound (total_k_rows + 256 per sequence): the GPU reports
+    SONIC_ERR_WORKSPACE in the status word, sequences that fit still run."""
+    d = inputs.Dialogue(100, [(400, 100)] * 2, 0)
+    batch = inputs.Batch([d, d, d])
+    res = H.run_prefill(batch, 2, 1, 128, seed=19, key_order=sonic.KEYS_RETAINED_FIRST,
+                        k_start=[0, 0, 0], total_k_rows=int(batch.k_len[0]),
+                        expect_status=3, with_lse=False)
+    # sequence 0 fits (its span starts at row 0); later ones are left as zeros
+    O, _, got, _ = H.oracle_prefill_rows(
+        inputs.Batch([d]), dict(res, q_len=res["q_len"][:1], q_start=res["q_start"][:1]), 0,
+        np.arange(0, int(batch.k_len[0]), 7))
+    H.check_close(got, O, "seq 0")
+    n = int(batch.k_len[0])
+    assert (res["O"][0, n:].float() == 0).all()
+
+
+@pytest.mark.parametrize("order", ORDERS)
+def test_current_turn_over_compacted_cache(order):
     """Turn-by-turn form: queries = the current turn, keys = retained cache +
     current turn (bottom-right aligned)."""
     full = [inputs.Dialogue(40, [(200, 30), (150, 20), (90, 45)], 333),
@@ -47,17 +123,18 @@ def test_current_turn_over_compacted_cache():
     ret = inputs.Batch([inputs.Dialogue(d.sys_len, [(0, k) for _, k in d.segments], d.curr_len)
                         for d in full])
     q_len = [d.curr_len for d in full]
-    res = H.run_prefill(ret, 8, 2, 128, q_len=q_len, seed=21)
+    res = H.run_prefill(ret, 8, 2, 128, q_len=q_len, seed=21, key_order=order)
     for b in range(ret.B):
         O, lse, got, got_lse = H.oracle_prefill_rows(ret, res, b, np.arange(q_len[b]))
         H.check_close(got, O, f"seq {b}")
 
 
-def test_masked_prefill_workload_sampled_rows():
+@pytest.mark.parametrize("order", ORDERS)
+def test_masked_prefill_workload_sampled_rows(order):
     """Batch 8, 32/8 heads, D = 128, L = 5632, every row (full mask); rows
     sampled across tiles, segment edges and the ragged end."""
     batch, hd = inputs.masked_prefill()
-    res = H.run_prefill(batch, hd.hq, hd.hkv, hd.d, seed=31)
+    res = H.run_prefill(batch, hd.hq, hd.hkv, hd.d, seed=31, key_order=order)
     L = int(batch.k_len[0])
     rows = np.unique(np.r_[0, 127, 128, 511, 512, 767, 799, 800, 2000, 4000, 5119, 5120, L - 1])
     for b in (0, 5):
