@@ -701,7 +701,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // probabilities, written as bf16 pairs over the S columns
             const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
             const float2 nm2 = make_float2(-mref, -mref);
-            float2 rs2a = make_float2(0.f, 0.f), rs2b = make_float2(0.f, 0.f);
+            float ls[4] = {0.f, 0.f, 0.f, 0.f};
             float2 rs2x = make_float2(0.f, 0.f);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
@@ -719,16 +719,11 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // by, so O is a weighted mean of V rows with weights summing
                     // to one (rounding moves weight between keys, it does not
                     // scale the output)
-                    const float2 ev = make_float2(__uint_as_float(pr << 16),
-                                                  __uint_as_float(pr & 0xffff0000u));
-                    if ((e >> 1) & 1)
-                        rs2b = __fadd2_rn(rs2b, ev);
-                    else
-                        rs2a = __fadd2_rn(rs2a, ev);
+                    add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
                 }
                 tmem_st16(tS + c * 16, pk);
             }
-            l = l * alpha + ((rs2a.x + rs2a.y) + (rs2b.x + rs2b.y));
+            l = l * alpha + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
             if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
             // O rescale (PV of the previous tile is complete: S of this tile was
             // issued after it, and S is done)
