@@ -284,9 +284,13 @@ typedef struct {
  * lens[b] - 1 of K_ret / V_ret (the new token's own row included) are all
  * visible:  O[l, b, h] = sum_t softmax_t(scale <q[l,b,h], K[t, h/G]>) V[t, h/G].
  * The keys are split into chunks of chunk_len; each (layer, sequence, KV
- * head, chunk) block produces a partial (max, sum, accumulator) in the
- * workspace, and a second kernel merges them by log-sum-exp.  lens[b] = 0
- * gives zeros (and lse = -inf).  bf16 in/out, fp32 arithmetic.
+ * head, chunk) unit produces a partial (max, sum, accumulator) in the
+ * workspace, and a second kernel merges them by log-sum-exp (a sequence that
+ * fits one chunk is written directly).  At head_dim 128 one persistent block
+ * per SM claims units from a counter in the workspace (zeroed on `stream`
+ * before the launch), so the workspace is never empty there and concurrent
+ * calls need workspaces of their own.  lens[b] = 0 gives zeros (and
+ * lse = -inf).  bf16 in/out, fp32 arithmetic.
  */
 SONIC_API sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
                                  const uint16_t *V_ret, const int32_t *lens, uint16_t *O,

@@ -321,6 +321,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
 // memory; a running maximum that rises by less than 2^8 does not trigger an
 // O rescale.  S^T and P are double buffered so S^T of the next tile overlaps
 // the softmax and P.V of the current one.
+//
+// The kernel is persistent: one block per SM claims units (key chunk, KV
+// head, sequence, layer) from a global counter (so ragged units balance over
+// the SMs) and works through them as one continuous stream of key tiles: the
+// K/V ring and the tensor pipe stay busy across unit boundaries (the next
+// unit's q is staged and its first S^T issued while the current unit
+// finishes).  q and the O^T accumulator are double buffered by unit.  Short
+// sequences (a few tiles per unit) would otherwise spend most of a block's
+// life on set-up and on the first copies.
 // ---------------------------------------------------------------------------
 constexpr int kTcKeys = 128;
 constexpr int kTcStages = 3;
@@ -332,82 +341,142 @@ struct TcCfg {
     static constexpr int D = 128;
     static constexpr int kTileBytes = kTcKeys * D * 2;           // K or V tile: 32 KB
     static constexpr int kStageBytes = 2 * kTileBytes;           // 64 KB
-    static constexpr int kOffQ = kTcStages * kStageBytes;        // q, 16 x 128 bf16, swizzled
+    static constexpr int kQBufs = 2;                             // q of this unit and the next
+    static constexpr int kOffQ = kTcStages * kStageBytes;        // q [2], 16 x 128 bf16, swizzled
     static constexpr int kQBytes = kTcN * D * 2;                 // 4 KB
-    static constexpr int kOffP = kOffQ + kQBytes;                // P, [2][16 x 128 keys] bf16
+    static constexpr int kOffP = kOffQ + kQBufs * kQBytes;       // P, [2][16 x 128 keys] bf16
     static constexpr int kPBytes = kTcN * kTcKeys * 2;           // 4 KB
     static constexpr int kOffRed = kOffP + 2 * kPBytes;          // [2][4][16] float
     static constexpr int kOffL = kOffRed + 2 * 4 * kTcN * 4;     // [4][16] float
     static constexpr int kOffBar = kOffL + 4 * kTcN * 4;
-    static constexpr int kNumBars = 2 * kTcStages + 2 + 5;
+    static constexpr int kNumBars = 2 * kTcStages + 24;  // the pointers carved out below
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
-    static constexpr size_t kSmem = 1024 + kOffMisc + 16;
+    static constexpr int kSeqCache = 1024;                       // sequences whose lens/kv_start
+    static constexpr int kOffSeq = kOffMisc + 128;               // are cached: [2][1024] int32
+    static constexpr size_t kSmem = 1024 + kOffSeq + 2 * kSeqCache * 4;
 };
+constexpr int kUnitSlots = 4;  // claimed-unit queue between the producer and the others
+
+// Unit u: (key chunk, KV head, sequence, layer), KV head fastest.  A unit whose
+// chunk starts past the sequence's end has no keys.
+struct TcUnit {
+    int u, kvh, chunk, b, layer, nkeys, ntiles, row0, len;
+};
+
+// The indices of unit w.u and its tile count (from w.nkeys).
+__device__ __forceinline__ void tc_coords(const DecParams &p, int units_x, TcUnit &w) {
+    const int x = w.u % units_x, y = w.u / units_x;
+    w.kvh = x % p.Hkv;
+    w.chunk = x / p.Hkv;
+    w.b = y % p.B;
+    w.layer = y / p.B;
+    w.ntiles = (w.nkeys + kTcKeys - 1) / kTcKeys;
+}
+
+// seq_len / seq_start: the sequences' lengths and first rows cached in shared
+// memory (B <= kSeqCache), or NULL to read them from global memory.
+__device__ __forceinline__ bool tc_unit(const DecParams &p, int units_x, int u, TcUnit &w,
+                                        const int32_t *seq_len, const int32_t *seq_start) {
+    const int x = u % units_x, y = u / units_x;
+    w.u = u;
+    w.kvh = x % p.Hkv;
+    w.chunk = x / p.Hkv;
+    w.b = y % p.B;
+    w.layer = y / p.B;
+    int len = seq_len != nullptr ? seq_len[w.b] : p.lens[w.b];
+    len = min(max(len, 0), p.max_chunks * p.chunk_len);
+    const int key0 = w.chunk * p.chunk_len;
+    w.len = len;
+    w.nkeys = max(min(p.chunk_len, len - key0), 0);
+    w.ntiles = (w.nkeys + kTcKeys - 1) / kTcKeys;
+    w.row0 = (seq_start != nullptr ? seq_start[w.b] : p.kv_start[w.b]) + key0;
+    return w.nkeys > 0;
+}
 
 template <int GT>
 __global__ void __launch_bounds__(kTcThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                 const DecParams p) {
+                 const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK16,
+                 const __grid_constant__ CUtensorMap tmV16, const DecParams p, int units_x,
+                 int n_units, int *unit_counter) {
     constexpr int D = 128;
     using C = TcCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t *q_s = smem + C::kOffQ;
-    uint8_t *P_s = smem + C::kOffP;
+    uint8_t *q_s = smem + C::kOffQ;  // [2]
+    uint8_t *P_s = smem + C::kOffP;  // [2]
     float *red = reinterpret_cast<float *>(smem + C::kOffRed);
     float *lred = reinterpret_cast<float *>(smem + C::kOffL);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
-    uint64_t *full = bars;                    // [stages]
-    uint64_t *empty = bars + kTcStages;       // [stages]
-    uint64_t *s_full = bars + 2 * kTcStages;  // [2]
-    uint64_t *p_full = s_full + 2;
-    uint64_t *o_done = p_full + 1;
+    uint64_t *full = bars;                    // [stages] K/V tile landed
+    uint64_t *empty = bars + kTcStages;       // [stages] its P.V is done
+    uint64_t *s_full = bars + 2 * kTcStages;  // [2] per global tile
+    uint64_t *p_full = s_full + 2;            // [2] per global tile: its P written (128 threads)
+    uint64_t *o_done = p_full + 2;            // a P.V done
     uint64_t *mma_idle = o_done + 1;
-    uint64_t *sm_sync = mma_idle + 1;  // the 128 softmax threads, once per tile + epilogue
-    uint64_t *o_last = sm_sync + 1;    // completes once, after the last P.V
+    uint64_t *sm_sync = mma_idle + 1;  // the 128 softmax threads, once per tile
+    uint64_t *ep_sync = sm_sync + 1;   // the 128 softmax threads, once per unit
+    uint64_t *q_full = ep_sync + 1;    // [2] per unit: q staged
+    uint64_t *q_empty = q_full + 2;    // [2] per unit: its last S^T done
+    uint64_t *o_last = q_empty + 2;    // [2] per unit: its last P.V done
+    uint64_t *o_free = o_last + 2;     // [2] per unit: its O^T read out (128 threads)
+    uint64_t *uq_full = o_free + 2;    // [kUnitSlots] a claimed unit is in its slot
+    uint64_t *uq_empty = uq_full + kUnitSlots;  // [kUnitSlots] the issuer and 4 warps read it
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
+    // [kUnitSlots][4]: unit index (-1: no more), its keys, first key row, sequence length
+    volatile int32_t *unit_q = misc + 4;
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 1);
 
-    const int kvh = blockIdx.x % p.Hkv, chunk = blockIdx.x / p.Hkv;
-    const int b = blockIdx.y % p.B, layer = blockIdx.y / p.B;
-    int len = p.lens[b];
-    if (len > p.max_chunks * p.chunk_len) {
-        if (threadIdx.x == 0 && blockIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
-        len = p.max_chunks * p.chunk_len;
-    }
-    const int key0 = chunk * p.chunk_len;
-    if (key0 >= len || timed_out(p.status)) return;
-    const int nkeys = min(p.chunk_len, len - key0);
-    const int ntiles = (nkeys + kTcKeys - 1) / kTcKeys;
     const int G = p.G;
-    const int row0 = p.kv_start[b] + key0;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-    // q of the G heads (rows >= G zero) in the 128-byte-swizzled K-major layout;
-    // both P buffers zeroed (their rows >= G stay zero).
-    const uint16_t *qp = p.q + layer * p.q_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G) * D;
-    for (int i = tid; i < kTcN * (D / 8); i += blockDim.x) {
-        const int g = i / (D / 8), c = i % (D / 8);
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (g < G) v = *reinterpret_cast<const uint4 *>(qp + g * D + c * 8);
-        *reinterpret_cast<uint4 *>(q_s + (c >> 3) * (kTcN * 128) + g * 128 +
-                                   (((c & 7) ^ (g & 7)) << 4)) = v;
+    if (timed_out(p.status)) return;
+    if (tid == 0) {
+        // a sequence longer than the plan allows is clipped, and reported
+        for (int b = blockIdx.x; b < p.B; b += gridDim.x)
+            if (p.lens[b] > p.max_chunks * p.chunk_len) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
     }
+
+    // The P buffers zeroed (rows >= GT stay zero), and the K/V ring: rows a
+    // partial tile does not load keep older, finite data, which P = 0 cancels.
     for (int i = tid; i < 2 * C::kPBytes / 16; i += blockDim.x)
         reinterpret_cast<uint4 *>(P_s)[i] = make_uint4(0, 0, 0, 0);
+    for (int i = tid; i < kTcStages * C::kStageBytes / 16; i += blockDim.x)
+        reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0, 0, 0, 0);
+    // the sequences' lengths and first rows, for claiming units without
+    // global loads on the producer's path
+    int32_t *seq_len = nullptr, *seq_start = nullptr;
+    if (p.B <= C::kSeqCache) {
+        seq_len = reinterpret_cast<int32_t *>(smem + C::kOffSeq);
+        seq_start = seq_len + C::kSeqCache;
+        for (int b = tid; b < p.B; b += blockDim.x) {
+            seq_len[b] = p.lens[b];
+            seq_start[b] = p.kv_start[b];
+        }
+    }
     if (tid == 0) {
         for (int s = 0; s < kTcStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(&s_full[0], 1);
-        mbar_init(&s_full[1], 1);
-        mbar_init(p_full, 128);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&p_full[i], 128);
+            mbar_init(&o_last[i], 1);
+            mbar_init(&o_free[i], 128);
+        }
+        for (int i = 0; i < C::kQBufs; ++i) {
+            mbar_init(&q_full[i], 1);
+            mbar_init(&q_empty[i], 1);
+        }
+        for (int i = 0; i < kUnitSlots; ++i) {
+            mbar_init(&uq_full[i], 1);
+            mbar_init(&uq_empty[i], 5);
+        }
         mbar_init(o_done, 1);
         mbar_init(mma_idle, 1);
         mbar_init(sm_sync, 128);
-        mbar_init(o_last, 1);
+        mbar_init(ep_sync, 128);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -420,78 +489,202 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
+    // TMEM: S^T [2] at columns 0 / 16, O^T [2] at 32 / 48
     const uint32_t tS = tmem, tO = tmem + 32;
+    // The k-th claimed unit (w.u = -1: none left, or a wait gave up), from
+    // shared memory: the consumers never touch global memory for it.  Each
+    // reader (the issuer, lane 0 of each softmax warp) frees the slot.
+    auto read_unit = [&](int k, TcUnit &w) -> bool {
+        const int slot = k & (kUnitSlots - 1);
+        w.u = -1;
+        if (!mbar_wait(&uq_full[slot], (k / kUnitSlots) & 1, p.status, abort_flag)) return false;
+        const volatile int32_t *q = unit_q + slot * 4;
+        w.u = q[0];
+        w.nkeys = q[1];
+        w.row0 = q[2];
+        w.len = q[3];
+        mbar_arrive(&uq_empty[slot]);
+        return w.u >= 0;
+    };
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             tma_prefetch_desc(&tmK);
             tma_prefetch_desc(&tmV);
-            int t = 0;
-            for (; t < ntiles; ++t) {
-                const int s = t % kTcStages;
-                if (t >= kTcStages &&
-                    !mbar_wait(&empty[s], ((t / kTcStages) - 1) & 1, p.status, abort_flag))
-                    break;
-                mbar_arrive_expect_tx(&full[s], C::kStageBytes);
-                uint8_t *kd = smem + s * C::kStageBytes;
-                uint8_t *vd = kd + C::kTileBytes;
-                const int r = row0 + t * kTcKeys;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], hh * 64, kvh, r, layer);
-                    tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], hh * 64, kvh, r, layer);
+        }
+        // Lane 0 claims units from the counter, publishes each in the unit
+        // queue and streams its q (one TMA box of 16 heads: rows past the
+        // group's G heads are other heads' q or zeros, whose S^T columns the
+        // softmax never reads) and its K/V tiles.  The claim of unit k + 1 is
+        // sent before unit k's copies are queued; its answer is needed only
+        // after them.
+        if (lane == 0) {
+            tma_prefetch_desc(&tmQ);
+            int T = 0;
+            int pending = atomicAdd(unit_counter, 1);
+            for (int k = 0;; ++k) {
+                const int slot = k & (kUnitSlots - 1);
+                bool ok = k < kUnitSlots ||
+                          mbar_wait(&uq_empty[slot], ((k / kUnitSlots) - 1) & 1, p.status, abort_flag);
+                int u = -1;
+                TcUnit w;
+                if (ok) {
+                    u = pending;
+                    while (u < n_units && !tc_unit(p, units_x, u, w, seq_len, seq_start))
+                        u = atomicAdd(unit_counter, 1);
+                    if (u >= n_units) u = -1;
                 }
+                volatile int32_t *q = unit_q + slot * 4;
+                q[0] = u;
+                q[1] = w.nkeys;
+                q[2] = w.row0;
+                q[3] = w.len;
+                mbar_arrive(&uq_full[slot]);  // release: the slot is written
+                if (u < 0) break;
+                pending = atomicAdd(unit_counter, 1);
+                // q into buffer k & 1 once the S^T MMAs of unit k - 2 no longer read it
+                const int qb = k & 1;
+                if (k >= 2 && !mbar_wait(&q_empty[qb], ((k >> 1) - 1) & 1, p.status, abort_flag))
+                    break;
+                mbar_arrive_expect_tx(&q_full[qb], C::kQBytes);
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh)
+                    tma_load_4d(q_s + qb * C::kQBytes + hh * (kTcN * 128), &tmQ, &q_full[qb],
+                                hh * 64, w.kvh * G, w.b, w.layer);
+                for (int t = 0; t < w.ntiles; ++t, ++T) {
+                    const int s = T % kTcStages;
+                    if (T >= kTcStages &&
+                        !mbar_wait(&empty[s], ((T / kTcStages) - 1) & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t *kd = smem + s * C::kStageBytes;
+                    uint8_t *vd = kd + C::kTileBytes;
+                    const int r = w.row0 + t * kTcKeys;
+                    const int rem = w.nkeys - t * kTcKeys;
+                    if (rem >= kTcKeys) {
+                        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+#pragma unroll
+                        for (int hh = 0; hh < 2; ++hh) {
+                            tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], hh * 64, w.kvh,
+                                        r, w.layer);
+                            tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], hh * 64, w.kvh,
+                                        r, w.layer);
+                        }
+                    } else {
+                        // a unit's last, partial tile: only its rows, in 16-row boxes
+                        // (the rows past them keep older data; the softmax masks
+                        // their scores and zeroes their V rows)
+                        const int nb = (rem + 15) / 16;
+                        mbar_arrive_expect_tx(&full[s], nb * 4 * (16 * 128));
+                        for (int j = 0; j < nb; ++j)
+#pragma unroll
+                            for (int hh = 0; hh < 2; ++hh) {
+                                tma_load_4d(kd + hh * (kTcKeys * 128) + j * (16 * 128), &tmK16,
+                                            &full[s], hh * 64, w.kvh, r + 16 * j, w.layer);
+                                tma_load_4d(vd + hh * (kTcKeys * 128) + j * (16 * 128), &tmV16,
+                                            &full[s], hh * 64, w.kvh, r + 16 * j, w.layer);
+                            }
+                    }
+                }
+                if (!ok) break;
             }
-            if (*abort_flag)
-                for (int u = max(0, t - kTcStages); u < t; ++u)
+            if (*abort_flag) {
+                for (int u = max(0, T - kTcStages); u < T; ++u)
                     mbar_wait(&full[u % kTcStages], (u / kTcStages) & 1, p.status, abort_flag);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kTcKeys, kTcN, 0, 0);
             constexpr uint32_t idPV = idesc_bf16_f32(D, kTcN, 0, 1);
-            const uint32_t base = smem_u32(smem), q_addr = smem_u32(q_s), p_addr = smem_u32(P_s);
-            auto issue_s = [&](int t) {
-                const uint32_t k_addr = base + (t % kTcStages) * C::kStageBytes;
+            const uint32_t base = smem_u32(smem), q_base = smem_u32(q_s), p_addr = smem_u32(P_s);
+            // S^T of global tile T (unit number k, its tile t) from q buffer k % 2
+            auto issue_s = [&](int T, int k, int t, int nt) -> bool {
+                if (t == 0 &&
+                    !mbar_wait(&q_full[k % C::kQBufs], (k / C::kQBufs) & 1, p.status, abort_flag))
+                    return false;
+                if (!mbar_wait(&full[T % kTcStages], (T / kTcStages) & 1, p.status, abort_flag))
+                    return false;
+                tc_fence_after();
+                const uint32_t k_addr = base + (T % kTcStages) * C::kStageBytes;
+                const uint32_t q_addr = q_base + (k % C::kQBufs) * C::kQBytes;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint64_t a = smem_desc_sw128(
                         k_addr + (kk >> 2) * (kTcKeys * 128) + (kk & 3) * 32, 16, 1024);
                     const uint64_t bd =
                         smem_desc_sw128(q_addr + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
-                    tc_mma_ss(tS + (t & 1) * kTcN, a, bd, idS, kk > 0 ? 1u : 0u);
+                    tc_mma_ss(tS + (T & 1) * kTcN, a, bd, idS, kk > 0 ? 1u : 0u);
                 }
-                tc_commit(&s_full[t & 1]);
+                tc_commit(&s_full[T & 1]);
+                if (t == nt - 1) tc_commit(&q_empty[k % C::kQBufs]);
+                return true;
             };
-            bool ok = mbar_wait(&full[0], 0, p.status, abort_flag);
+            TcUnit w, nx;
+            int T = 0, k = 0;
+            bool ok = read_unit(0, w);
             if (ok) {
-                tc_fence_after();
-                issue_s(0);
+                tc_coords(p, units_x, w);
+                ok = issue_s(0, 0, 0, w.ntiles);
             }
-            for (int t = 0; ok && t < ntiles; ++t) {
-                if (t + 1 < ntiles) {
-                    const int s1 = (t + 1) % kTcStages;
-                    if (!mbar_wait(&full[s1], ((t + 1) / kTcStages) & 1, p.status, abort_flag))
+            for (bool more = true; ok && more; ++k) {
+                bool has_next = false;
+                for (int t = 0; ok && t < w.ntiles; ++t, ++T) {
+                    // The next tile: this unit's, or the next unit's first (read
+                    // only now: the producer publishes it after queueing all of this
+                    // unit's copies).  Its S^T goes before this tile's P.V when its
+                    // K tile (and q) are already in; otherwise after, so that a late
+                    // copy never holds back the P.V that frees a stage.
+                    int nk = k, nt1 = t + 1, nnt = w.ntiles;
+                    bool next_tile = t + 1 < w.ntiles;
+                    if (!next_tile) {
+                        has_next = read_unit(k + 1, nx);
+                        if (has_next) {
+                            tc_coords(p, units_x, nx);
+                            next_tile = true;
+                            nk = k + 1;
+                            nt1 = 0;
+                            nnt = nx.ntiles;
+                        }
+                    }
+                    bool s_issued = false;
+                    if (next_tile &&
+                        mbar_test(&full[(T + 1) % kTcStages], ((T + 1) / kTcStages) & 1) &&
+                        (nt1 > 0 || mbar_test(&q_full[nk & 1], (nk >> 1) & 1))) {
+                        ok = issue_s(T + 1, nk, nt1, nnt);
+                        s_issued = true;
+                    }
+                    if (!ok || !mbar_wait(&p_full[T & 1], (T >> 1) & 1, p.status, abort_flag)) {
+                        ok = false;
                         break;
+                    }
+                    // O^T buffer k & 1: unit k - 2's epilogue has read it out
+                    if (t == 0 && k >= 2 &&
+                        !mbar_wait(&o_free[k & 1], ((k >> 1) - 1) & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
                     tc_fence_after();
-                    issue_s(t + 1);
-                }
-                if (!mbar_wait(p_full, t & 1, p.status, abort_flag)) break;
-                tc_fence_after();
-                const uint32_t v_addr = base + (t % kTcStages) * C::kStageBytes + C::kTileBytes;
-                const uint32_t pb = p_addr + (t & 1) * C::kPBytes;
+                    const uint32_t v_addr = base + (T % kTcStages) * C::kStageBytes + C::kTileBytes;
+                    const uint32_t pb = p_addr + (T & 1) * C::kPBytes;
 #pragma unroll
-                for (int kk = 0; kk < kTcKeys / 16; ++kk) {
-                    const uint64_t a = smem_desc_sw128(v_addr + kk * (16 * 128), kTcKeys * 128, 1024);
-                    const uint64_t bd =
-                        smem_desc_sw128(pb + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
-                    tc_mma_ss(tO, a, bd, idPV, (t > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < kTcKeys / 16; ++kk) {
+                        const uint64_t a =
+                            smem_desc_sw128(v_addr + kk * (16 * 128), kTcKeys * 128, 1024);
+                        const uint64_t bd =
+                            smem_desc_sw128(pb + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
+                        tc_mma_ss(tO + (k & 1) * kTcN, a, bd, idPV, (t > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc_commit(o_done);
+                    tc_commit(&empty[T % kTcStages]);
+                    if (t == w.ntiles - 1) tc_commit(&o_last[k & 1]);
+                    if (next_tile && !s_issued) ok = issue_s(T + 1, nk, nt1, nnt);
                 }
-                tc_commit(o_done);
-                tc_commit(&empty[t % kTcStages]);
-                if (t == ntiles - 1) tc_commit(o_last);
+                more = has_next;
+                w = nx;
             }
             tc_commit(mma_idle);
             mbar_wait(mma_idle, 0, p.status, abort_flag);
@@ -501,96 +694,13 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;  // key row of the tile, and d row of O^T
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-        float m[GT], l[GT];
-#pragma unroll
-        for (int g = 0; g < GT; ++g) {
-            m[g] = -INFINITY;
-            l[g] = 0.f;
-        }
-        bool ok = true;
-        for (int t = 0; t < ntiles; ++t) {
-            if (!mbar_wait(&s_full[t & 1], (t >> 1) & 1, p.status, abort_flag)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            uint32_t sr[16];
-            tmem_ld16(tS + lane_base + (t & 1) * kTcN, sr);
-            tmem_ld_wait();
-            reg_fence16(sr);
-            const bool valid = t * kTcKeys + r < nkeys;
-            float sv[GT];
-            float *rd = red + (t & 1) * 4 * kTcN;
-#pragma unroll
-            for (int g = 0; g < GT; ++g) {
-                sv[g] = valid ? __uint_as_float(sr[g]) * p.scale_log2 : -INFINITY;
-                const float wm = warp_max(sv[g]);
-                if (lane == 0) rd[quarter * kTcN + g] = wm;
-            }
-            // all four warps' maxima visible (bounded: a wait that gives up ends the loop)
-            mbar_arrive(sm_sync);
-            if (!mbar_wait(sm_sync, t & 1, p.status, abort_flag)) {
-                ok = false;
-                break;
-            }
-            float alpha[GT];
-            bool resc = false;
-#pragma unroll
-            for (int g = 0; g < GT; ++g) {
-                const float mt = fmaxf(fmaxf(rd[g], rd[kTcN + g]),
-                                       fmaxf(rd[2 * kTcN + g], rd[3 * kTcN + g]));
-                alpha[g] = 1.f;
-                if (t == 0) {
-                    m[g] = mt;
-                } else if (mt > m[g] + kTcRescale) {
-                    alpha[g] = ex2(m[g] - mt);
-                    m[g] = mt;
-                    resc = true;
-                }
-            }
-            // P^T column r (this key) in the swizzled K-major P buffer
-            uint8_t *pb = P_s + (t & 1) * C::kPBytes + (r >> 6) * (kTcN * 128) + (r & 7) * 2;
-            const int jj = (r & 63) >> 3;
-#pragma unroll
-            for (int g = 0; g < GT; ++g) {
-                // the row sum adds the rounded probability P.V multiplies by
-                const __nv_bfloat16 pr = __float2bfloat16_rn(ex2(sv[g] - m[g]));
-                l[g] = l[g] * alpha[g] + __bfloat162float(pr);
-                *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) = pr;
-            }
-            if (!valid) {
-                // V rows past the keys: zero, so 0 * garbage cannot reach O
-                uint8_t *vrow = smem + (t % kTcStages) * C::kStageBytes + C::kTileBytes + r * 128;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-                    for (int u = 0; u < 8; ++u)
-                        reinterpret_cast<uint4 *>(vrow + hh * (kTcKeys * 128))[u] =
-                            make_uint4(0, 0, 0, 0);
-            }
-            if (resc) {  // block-uniform
-                if (!mbar_wait(o_done, (t - 1) & 1, p.status, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                uint32_t o[16];
-                tmem_ld16(tO + lane_base, o);
-                tmem_ld_wait();
-                reg_fence16(o);
-#pragma unroll
-                for (int g = 0; g < GT; ++g) o[g] = __float_as_uint(__uint_as_float(o[g]) * alpha[g]);
-                tmem_st16(tO + lane_base, o);
-                tmem_st_wait();
-            }
-            fence_proxy_async_smem();
-            tc_fence_before();
-            mbar_arrive(p_full);
-        }
-        // ------------------------------------------------------------ epilogue
-        // o_done may still be two phases behind here (S of a tile is issued before
-        // the previous tile's P.V), so the end of the last P.V has its own barrier.
-        if (ok && mbar_wait(o_last, 0, p.status, abort_flag)) {
+        // Unit epilogue: normalise O^T of unit k and write it (or its partial).
+        // It runs one tile into the next unit, when the unit's last P.V is long
+        // done, so the move from one unit to the next costs no pipeline drain.
+        auto epilogue = [&](const TcUnit &w, int k, const float (&m)[GT],
+                            const float (&l)[GT]) -> bool {
+            const uint32_t tOk = tO + (k & 1) * kTcN;
+            if (!mbar_wait(&o_last[k & 1], (k >> 1) & 1, p.status, abort_flag)) return false;
             tc_fence_after();
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
@@ -599,26 +709,33 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
                 if (lane == 0) lred[quarter * kTcN + g] = v;
             }
-            mbar_arrive(sm_sync);
-            if (mbar_wait(sm_sync, ntiles & 1, p.status, abort_flag)) {
+            mbar_arrive(ep_sync);
+            if (!mbar_wait(ep_sync, k & 1, p.status, abort_flag)) return false;
             uint32_t o[16];
-            tmem_ld16(tO + lane_base, o);
+            tmem_ld16(tOk + lane_base, o);
             tmem_ld_wait();
             reg_fence16(o);
-            const int n_chunks = (len + p.chunk_len - 1) / p.chunk_len;
-            const int64_t unit0 = ((int64_t)layer * p.B + b) * p.Hq + (int64_t)kvh * G;
+            float Lg[GT];
+#pragma unroll
+            for (int g = 0; g < GT; ++g)
+                Lg[g] = lred[g] + lred[kTcN + g] + lred[2 * kTcN + g] + lred[3 * kTcN + g];
+            // O^T of this unit is in registers and lred read: the buffers are free
+            tc_fence_before();
+            mbar_arrive(&o_free[k & 1]);
+            const int n_chunks = (w.len + p.chunk_len - 1) / p.chunk_len;
+            const int64_t unit0 = ((int64_t)w.layer * p.B + w.b) * p.Hq + (int64_t)w.kvh * G;
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
                 if (g >= G) break;
-                const float L = lred[g] + lred[kTcN + g] + lred[2 * kTcN + g] + lred[3 * kTcN + g];
+                const float L = Lg[g];
                 const float a = __uint_as_float(o[g]);
                 if (n_chunks == 1) {
                     uint16_t *op =
-                        p.O + layer * p.o_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G + g) * D;
+                        p.O + w.layer * p.o_ls + ((int64_t)w.b * p.Hq + (int64_t)w.kvh * G + g) * D;
                     op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
                     if (r == 0 && p.lse != nullptr) p.lse[unit0 + g] = (m[g] + __log2f(L)) * kLn2;
                 } else {
-                    const int64_t slot = (unit0 + g) * p.max_chunks + chunk;
+                    const int64_t slot = (unit0 + g) * p.max_chunks + w.chunk;
                     p.part_acc[slot * D + r] = a;
                     if (r == 0) {
                         p.part_ml[slot * 2 + 0] = m[g];
@@ -626,8 +743,127 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                     }
                 }
             }
+            return true;
+        };
+        bool ok = true, pend = false;  // pend: unit kp still owes its epilogue
+        int T = 0, kp = 0;
+        TcUnit wp;
+        float mp[GT], lp[GT];
+        for (int k = 0; ok; ++k) {
+            TcUnit w;
+            if (lane == 0) read_unit(k, w);
+            w.u = __shfl_sync(0xffffffffu, w.u, 0);
+            if (w.u < 0) break;
+            w.nkeys = __shfl_sync(0xffffffffu, w.nkeys, 0);
+            w.row0 = __shfl_sync(0xffffffffu, w.row0, 0);
+            w.len = __shfl_sync(0xffffffffu, w.len, 0);
+            tc_coords(p, units_x, w);
+            const uint32_t tOk = tO + (k & 1) * kTcN;
+            float m[GT], l[GT];
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                m[g] = -INFINITY;
+                l[g] = 0.f;
             }
+            for (int t = 0; t < w.ntiles; ++t, ++T) {
+                if (!mbar_wait(&s_full[T & 1], (T >> 1) & 1, p.status, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                uint32_t sr[16];
+                tmem_ld16(tS + lane_base + (T & 1) * kTcN, sr);
+                tmem_ld_wait();
+                reg_fence16(sr);
+                const bool valid = t * kTcKeys + r < w.nkeys;
+                float sv[GT];
+                float *rd = red + (T & 1) * 4 * kTcN;
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    sv[g] = valid ? __uint_as_float(sr[g]) * p.scale_log2 : -INFINITY;
+                    const float wm = warp_max(sv[g]);
+                    if (lane == 0) rd[quarter * kTcN + g] = wm;
+                }
+                // all four warps' maxima visible (bounded: a wait that gives up ends the loop)
+                mbar_arrive(sm_sync);
+                if (!mbar_wait(sm_sync, T & 1, p.status, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                float alpha[GT];
+                bool resc = false;
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    const float mt = fmaxf(fmaxf(rd[g], rd[kTcN + g]),
+                                           fmaxf(rd[2 * kTcN + g], rd[3 * kTcN + g]));
+                    alpha[g] = 1.f;
+                    if (t == 0) {
+                        m[g] = mt;
+                    } else if (mt > m[g] + kTcRescale) {
+                        alpha[g] = ex2(m[g] - mt);
+                        m[g] = mt;
+                        resc = true;
+                    }
+                }
+                // P^T column r (this key) in the swizzled K-major P buffer
+                uint8_t *pb = P_s + (T & 1) * C::kPBytes + (r >> 6) * (kTcN * 128) + (r & 7) * 2;
+                const int jj = (r & 63) >> 3;
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    // the row sum adds the rounded probability P.V multiplies by
+                    const __nv_bfloat16 pr = __float2bfloat16_rn(ex2(sv[g] - m[g]));
+                    l[g] = l[g] * alpha[g] + __bfloat162float(pr);
+                    *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) = pr;
+                }
+                if (!valid && r < ((w.nkeys - t * kTcKeys + 15) & ~15)) {
+                    // rows a partial tile loaded past the unit's keys (another
+                    // sequence's, or junk): zero their V, so 0 * garbage cannot
+                    // reach O
+                    uint8_t *vrow =
+                        smem + (T % kTcStages) * C::kStageBytes + C::kTileBytes + r * 128;
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                        for (int u = 0; u < 8; ++u)
+                            reinterpret_cast<uint4 *>(vrow + hh * (kTcKeys * 128))[u] =
+                                make_uint4(0, 0, 0, 0);
+                }
+                if (resc) {  // block-uniform
+                    if (!mbar_wait(o_done, (T - 1) & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint32_t o[16];
+                    tmem_ld16(tOk + lane_base, o);
+                    tmem_ld_wait();
+                    reg_fence16(o);
+#pragma unroll
+                    for (int g = 0; g < GT; ++g)
+                        o[g] = __float_as_uint(__uint_as_float(o[g]) * alpha[g]);
+                    tmem_st16(tOk + lane_base, o);
+                    tmem_st_wait();
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(&p_full[T & 1]);
+                if (t == 0 && pend) {
+                    ok = epilogue(wp, kp, mp, lp);
+                    pend = false;
+                    if (!ok) break;
+                }
+            }
+            if (!ok) break;
+            wp = w;
+            kp = k;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                mp[g] = m[g];
+                lp[g] = l[g];
+            }
+            pend = true;
         }
+        if (ok && pend) epilogue(wp, kp, mp, lp);
     }
     tc_fence_before();
     __syncthreads();
@@ -691,7 +927,7 @@ int g_template(int G) {
 
 struct Plan {
     int chunk_len, max_chunks;
-    size_t ws_acc, ws_ml;
+    size_t ws_acc, ws_ml, ws_cnt;  // partial accumulators, partial (max, sum), unit counter
 };
 
 Plan make_plan(const sonic_decode_args *a) {
@@ -716,6 +952,7 @@ Plan make_plan(const sonic_decode_args *a) {
         pl.ws_acc = round_up(units_q * pl.max_chunks * a->head_dim * sizeof(float), 256);
         pl.ws_ml = round_up(units_q * pl.max_chunks * 2 * sizeof(float), 256);
     }
+    if (a->head_dim == 128) pl.ws_cnt = 256;  // the persistent kernel's unit counter
     return pl;
 }
 
@@ -732,8 +969,14 @@ cudaError_t launch_split(const CUtensorMap &tk, const CUtensorMap &tv, const Dec
     return cudaGetLastError();
 }
 
+// Persistent launch: one block per SM (the stage ring takes most of shared
+// memory); the blocks claim units from a counter zeroed on the stream first.
+struct TcMaps {
+    CUtensorMap k, v, q, k16, v16;
+};
+
 template <int GT>
-cudaError_t launch_tc(const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p, dim3 grid,
+cudaError_t launch_tc(const TcMaps &m, const DecParams &p, int units_x, int n_units, int *counter,
                       cudaStream_t stream) {
     constexpr size_t smem = TcCfg::kSmem;
     static_assert(smem <= 232448, "decode shared memory");
@@ -741,19 +984,24 @@ cudaError_t launch_tc(const CUtensorMap &tk, const CUtensorMap &tv, const DecPar
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kTcThreads, smem, stream>>>(tk, tv, p);
+    e = cudaMemsetAsync(counter, 0, sizeof(int), stream);
+    if (e != cudaSuccess) return e;
+    const int sms = device_sm_count();
+    const int blocks = n_units < sms ? n_units : sms;
+    kern<<<blocks, kTcThreads, smem, stream>>>(m.k, m.v, m.q, m.k16, m.v16, p, units_x, n_units,
+                                               counter);
     return cudaGetLastError();
 }
 
-cudaError_t dispatch_tc(int GT, const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
-                        dim3 grid, cudaStream_t s) {
+cudaError_t dispatch_tc(int GT, const TcMaps &m, const DecParams &p, int units_x, int n_units,
+                        int *counter, cudaStream_t s) {
     switch (GT) {
-        case 1: return launch_tc<1>(tk, tv, p, grid, s);
-        case 2: return launch_tc<2>(tk, tv, p, grid, s);
-        case 4: return launch_tc<4>(tk, tv, p, grid, s);
-        case 7: return launch_tc<7>(tk, tv, p, grid, s);
-        case 8: return launch_tc<8>(tk, tv, p, grid, s);
-        case 16: return launch_tc<16>(tk, tv, p, grid, s);
+        case 1: return launch_tc<1>(m, p, units_x, n_units, counter, s);
+        case 2: return launch_tc<2>(m, p, units_x, n_units, counter, s);
+        case 4: return launch_tc<4>(m, p, units_x, n_units, counter, s);
+        case 7: return launch_tc<7>(m, p, units_x, n_units, counter, s);
+        case 8: return launch_tc<8>(m, p, units_x, n_units, counter, s);
+        case 16: return launch_tc<16>(m, p, units_x, n_units, counter, s);
     }
     return cudaErrorInvalidValue;
 }
@@ -782,7 +1030,7 @@ extern "C" size_t sonic_decode_workspace_size(const sonic_decode_args *a) {
         a->head_dim < 1)
         return 0;
     Plan pl = make_plan(a);
-    return pl.ws_acc + pl.ws_ml;
+    return pl.ws_acc + pl.ws_ml + pl.ws_cnt;
 }
 
 extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
@@ -817,11 +1065,12 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
         return SONIC_OK;
     }
     Plan pl = make_plan(a);
-    const size_t need = pl.ws_acc + pl.ws_ml;
+    const size_t need = pl.ws_acc + pl.ws_ml + pl.ws_cnt;
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
-    if ((long long)a->batch * a->n_layers > 65535 ||
-        (long long)pl.max_chunks * a->n_heads_kv > 0x7fffffffLL)
+    const long long units_x = (long long)pl.max_chunks * a->n_heads_kv;
+    if ((D == 64 && (long long)a->batch * a->n_layers > 65535) || units_x > 0x7fffffffLL ||
+        units_x * a->batch * a->n_layers > 0x7fffffffLL)
         return SONIC_ERR_UNSUPPORTED;
 
     const uint64_t row_elems = (uint64_t)a->n_heads_kv * D;
@@ -832,9 +1081,26 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const uint64_t strides[3] = {(uint64_t)D * 2, row_elems * 2, layer_bytes};
     const uint32_t box[4] = {64, 1, (uint32_t)(D == 128 ? kTcKeys : kTileKeys), 1};
     CUtensorMap tk, tv;
+    TcMaps tm{};
     if (!make_tmap_bf16_4d(&tk, K_ret, dims, strides, box) ||
         !make_tmap_bf16_4d(&tv, V_ret, dims, strides, box))
         return SONIC_ERR_INVALID_ARGUMENT;
+    if (D == 128) {
+        tm.k = tk;
+        tm.v = tv;
+        const uint32_t box16[4] = {64, 1, 16, 1};
+        if (!make_tmap_bf16_4d(&tm.k16, K_ret, dims, strides, box16) ||
+            !make_tmap_bf16_4d(&tm.v16, V_ret, dims, strides, box16))
+            return SONIC_ERR_INVALID_ARGUMENT;
+        // q as (D, head, sequence, layer): one box = 16 heads of one sequence
+        const uint64_t qdims[4] = {(uint64_t)D, (uint64_t)a->n_heads_q, (uint64_t)a->batch,
+                                   (uint64_t)a->n_layers};
+        const uint64_t qstr[3] = {(uint64_t)D * 2, (uint64_t)a->n_heads_q * D * 2,
+                                  a->n_layers > 1 ? (uint64_t)a->q_layer_stride * 2
+                                                  : (uint64_t)a->batch * a->n_heads_q * D * 2};
+        const uint32_t qbox[4] = {64, (uint32_t)kTcN, 1, 1};
+        if (!make_tmap_bf16_4d(&tm.q, q, qdims, qstr, qbox)) return SONIC_ERR_INVALID_ARGUMENT;
+    }
 
     DecParams p{};
     p.q = q;
@@ -856,8 +1122,10 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
     p.scale_log2 = scale * kLog2e;
 
-    dim3 grid(pl.max_chunks * a->n_heads_kv, a->batch * a->n_layers);
-    cudaError_t e = (D == 128) ? dispatch_tc(GT, tk, tv, p, grid, stream)
+    dim3 grid((unsigned)units_x, a->batch * a->n_layers);
+    int *counter = reinterpret_cast<int *>(static_cast<char *>(a->workspace) + pl.ws_acc + pl.ws_ml);
+    cudaError_t e = (D == 128) ? dispatch_tc(GT, tm, p, (int)units_x,
+                                             (int)(units_x * a->batch * a->n_layers), counter, stream)
                                : dispatch_g<64>(GT, tk, tv, p, grid, stream);
     if (e != cudaSuccess) return SONIC_ERR_CUDA;
     const long long units = (long long)a->n_layers * a->batch * a->n_heads_q;
