@@ -326,11 +326,11 @@ def run_gpu(args, rank: int, world: int):
     # ---------------- end to end: host buffers through the public calls
     # Every step copies its inputs from pinned host memory (new-turn Q, decode
     # q, the new tokens' K/V rows) and reads its outputs back (prefill O,
-    # decode O).  Steps are pipelined over three streams, as a server would
-    # run them: inputs of step k+1 and outputs of step k-1 move while step k
-    # computes (Q/O double-buffered); the K/V rows land in one contiguous copy
-    # and are appended into their cache rows by indexed device copies just
-    # before the step that reads them.
+    # decode O).  Steps are pipelined over a compute stream and a copy stream,
+    # as a server would run them: outputs of step k-1 and then inputs of step
+    # k+1 move while step k computes (Q/O double-buffered); the K/V rows land in
+    # one contiguous copy and are appended into their cache rows by indexed
+    # device copies just before the step that reads them.
     pin = lambda t: t.cpu().pin_memory()
     hQ, hqd = pin(g.Qp), pin(g.qd)
     hOp, hOd = torch.empty_like(hQ).pin_memory(), torch.empty_like(hqd).pin_memory()
@@ -347,7 +347,7 @@ def run_gpu(args, rank: int, world: int):
     h2d = (hQ.numel() + hqd.numel() + newK.numel() + newV.numel() + hdecK.numel() +
            hdecV.numel()) * 2
     d2h = (hOp.numel() + hOd.numel()) * 2
-    s_in, s_out = torch.cuda.Stream(device), torch.cuda.Stream(device)
+    s_io = torch.cuda.Stream(device)
 
     # cache rows the new tokens go to (indexed copies on the compute stream)
     pre_rows = torch.as_tensor(np.concatenate(
@@ -363,27 +363,44 @@ def run_gpu(args, rank: int, world: int):
         g.Vret.index_copy_(1, dec_rows_t, stdV)
 
     def e2e_run(nsteps):
+        # One copy stream carries both directions, one after the other: on this
+        # host link concurrent host->device and device->host copies slow each
+        # other down far more than running them back to back.  Per step k it
+        # reads back step k-1's outputs, then writes step k+1's inputs.
         ev_in = [ev() for _ in range(nsteps)]
         ev_app = [ev() for _ in range(nsteps)]
         ev_comp = [ev() for _ in range(nsteps)]
         ev_out = [ev() for _ in range(nsteps)]
         start, end = ev(), ev()
         start.record(stream)
-        s_in.wait_event(start)
-        for k in range(nsteps):
-            Qp, qd, Op, Od = sets[k % 2]
-            with torch.cuda.stream(s_in):
+        s_io.wait_event(start)
+
+        def inputs_in(k):
+            Qp, qd = sets[k % 2][0], sets[k % 2][1]
+            with torch.cuda.stream(s_io):
                 if k >= 2:
-                    s_in.wait_event(ev_comp[k - 2])  # set k%2 no longer read
+                    s_io.wait_event(ev_comp[k - 2])  # set k%2 no longer read
                 if k >= 1:
-                    s_in.wait_event(ev_app[k - 1])   # staging buffers consumed
+                    s_io.wait_event(ev_app[k - 1])   # staging buffers consumed
                 Qp.copy_(hQ, non_blocking=True)
                 qd.copy_(hqd, non_blocking=True)
                 stK.copy_(newK, non_blocking=True)
                 stV.copy_(newV, non_blocking=True)
                 stdK.copy_(hdecK, non_blocking=True)
                 stdV.copy_(hdecV, non_blocking=True)
-                ev_in[k].record(s_in)
+                ev_in[k].record(s_io)
+
+        def outputs_out(k):
+            Op, Od = sets[k % 2][2], sets[k % 2][3]
+            with torch.cuda.stream(s_io):
+                s_io.wait_event(ev_comp[k])
+                hOp.copy_(Op, non_blocking=True)
+                hOd.copy_(Od, non_blocking=True)
+                ev_out[k].record(s_io)
+
+        inputs_in(0)
+        for k in range(nsteps):
+            Qp, qd, Op, Od = sets[k % 2]
             with torch.cuda.stream(stream):
                 stream.wait_event(ev_in[k])
                 if k >= 2:
@@ -393,13 +410,12 @@ def run_gpu(args, rank: int, world: int):
                 g.Qp, g.qd, g.Op, g.Od = Qp, qd, Op, Od
                 g.step(stream)
                 ev_comp[k].record(stream)
-            with torch.cuda.stream(s_out):
-                s_out.wait_event(ev_comp[k])
-                hOp.copy_(Op, non_blocking=True)
-                hOd.copy_(Od, non_blocking=True)
-                ev_out[k].record(s_out)
-        s_out.wait_event(ev_out[nsteps - 1])
-        end.record(s_out)
+            if k >= 1:
+                outputs_out(k - 1)
+            if k + 1 < nsteps:
+                inputs_in(k + 1)
+        outputs_out(nsteps - 1)
+        end.record(s_io)
         return start, end
 
     e2e_run(max(2, args.warmup // 2))
