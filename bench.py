@@ -521,6 +521,217 @@ def oracle_sample(lay: Layout, n_rows: int = 512, threads: int = None):
     return flops / dt / 1e12, dt, threads, desc
 
 
+# ---------------------------------------------------------------------------
+# Further workloads (`--extra NAME`): one JSON line each, outside the
+# benchmark contract line.  Every rate counts algorithmic work only.
+# ---------------------------------------------------------------------------
+
+def _ev_time(fn, reps=5, warm=2):
+    import torch
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def _visible_pairs(role, seg, rows, mode):
+    """Visible (query, key) pairs of the Sec. 3.2 mask for query positions
+    `rows` of one sequence (host bookkeeping for the flop count)."""
+    pos = np.arange(len(role))
+    n = 0
+    for p in rows:
+        body = role == 1
+        nex = (role[p] == 2) & (role == 2)
+        nexv = True if mode == 0 else (seg <= seg[p])
+        v = np.where(body, (seg == seg[p]) & (pos <= p), np.where(nex, nexv, pos <= p))
+        n += int(v.sum())
+    return n
+
+
+def extra_masked_prefill():
+    """Masked prefill of a whole S_aug (Sec. 3.2): batch 8, 512 system tokens,
+    16 segments of 256 body + 32 Nexus tokens, a 512-token current turn (L =
+    5632), 32/8 heads, D = 128, one layer; every row a query, both key orders
+    and both Nexus readings; then the current turn's rows alone."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    batch, hd = inputs.masked_prefill()
+    d = batch.dialogues[0]
+    role, seg = d.arrays()
+    L = d.length
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    K = inputs.randn((1, batch.total, hd.hkv, hd.d), seed=1, device=dev)
+    V = inputs.randn((1, batch.total, hd.hkv, hd.d), seed=2, device=dev)
+    Q = inputs.randn((1, batch.total, hd.hq, hd.d), seed=3, device=dev)
+    O = torch.empty_like(Q)
+    r_, s_, ks, kl = t(batch.role), t(batch.seg), t(batch.k_start), t(batch.k_len)
+    res = {}
+    for mode in (0, 1):
+        flops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L), mode) * batch.B
+        for order, oname in ((0, "as_given"), (1, "retained_first")):
+            ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+                Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks, q_len=kl, max_q_len=L,
+                max_k_len=L, nexus_vis=mode, key_order=order))
+            res[f"all_rows_{'full' if mode == 0 else 'causal_segments'}_{oname}"] = {
+                "ms": round(ms, 3), "tflops": round(flops / ms / 1e9, 1)}
+    ql = np.full(batch.B, d.curr_len, np.int32)
+    qs = np.concatenate([[0], np.cumsum(ql)[:-1]]).astype(np.int32)
+    Qc = inputs.randn((1, int(ql.sum()), hd.hq, hd.d), seed=4, device=dev)
+    Oc = torch.empty_like(Qc)
+    flops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L - d.curr_len, L), 0) * batch.B
+    for order, oname in ((0, "as_given"), (1, "retained_first")):
+        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=t(qs), q_len=t(ql),
+            max_q_len=int(ql.max()), max_k_len=L, key_order=order))
+        res[f"current_rows_{oname}"] = {"ms": round(ms, 3), "tflops": round(flops / ms / 1e9, 1)}
+    return {"workload": "masked prefill, batch 8 x 5632 rows, 32/8 heads, D=128, 1 layer",
+            "results": res}
+
+
+def extra_decode():
+    """Decode over retained caches: Llama-3-8B-like (batch 16, 32 layers, 32/8
+    heads, 641 retained rows) and 64 long ragged dialogues with Nexus =
+    len/2 and len/5 (32 layers, 32/8 heads)."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    res = {}
+    for name, (b2, h2) in {"llama8b_641_rows": inputs.decode_llama8b(),
+                           "long_ragged_nexus_len_div_2": inputs.long_ragged(2),
+                           "long_ragged_nexus_len_div_5": inputs.long_ragged(5)}.items():
+        lens = np.array([x.recipe_retained + 1 for x in b2.dialogues], np.int32)
+        starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int32)
+        T = int(lens.sum())
+        K = inputs.randn((h2.n_layers, T, h2.hkv, h2.d), seed=7, device=dev)
+        V = inputs.randn((h2.n_layers, T, h2.hkv, h2.d), seed=8, device=dev)
+        q = inputs.randn((h2.n_layers, b2.B, h2.hq, h2.d), seed=9, device=dev)
+        O = torch.empty_like(q)
+        lt, st = t(lens), t(starts)
+        ms = _ev_time(lambda: sonic.sonic_attn_decode(q, K, V, lt, O, kv_start=st,
+                                                      max_len=int(lens.max())), reps=10)
+        by = (T * h2.hkv * h2.d * 2 * 2 + 2 * b2.B * h2.hq * h2.d * 2) * h2.n_layers
+        res[name] = {"ms": round(ms, 3), "gbs": round(by / ms / 1e6, 1), "gb": round(by / 1e9, 2)}
+        del K, V
+        torch.cuda.empty_cache()
+    return {"workload": "decode over retained caches", "results": res}
+
+
+def extra_context(n_layers: int = 8):
+    """Full-context vs SONIC decode at the mixed serving step's shapes: the 56
+    decoding dialogues (28/4 heads, D = 128; n_layers of 28 layers) decode one
+    token over (a) their whole dialogue without Nexus tokens -- system prompt,
+    every turn, the current turn: plain causal attention -- and (b) their
+    retained cache -- system prompt, Nexus tokens, current turn (Eq. 15).  The
+    same kernel serves both; the ratio is the decode-side mechanism behind
+    the paper's end-to-end speedup."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    ms_ = inputs.mixed_serving(seed=1)
+    h = ms_.heads
+    res = {}
+    full = np.array([d.sys_len + sum(b for b, _ in d.segments) + d.curr_len + 1
+                     for d in ms_.decode_hist], np.int64)
+    ret = np.array([d.recipe_retained + 1 for d in ms_.decode_hist], np.int64)
+    for name, lens in (("full_context", full), ("sonic_retained", ret)):
+        lens = lens.astype(np.int32)
+        starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int32)
+        T = int(lens.sum())
+        K = inputs.randn((n_layers, T, h.hkv, h.d), seed=7, device=dev)
+        V = inputs.randn((n_layers, T, h.hkv, h.d), seed=8, device=dev)
+        q = inputs.randn((n_layers, len(lens), h.hq, h.d), seed=9, device=dev)
+        O = torch.empty_like(q)
+        lt, st = t(lens), t(starts)
+        ms = _ev_time(lambda: sonic.sonic_attn_decode(q, K, V, lt, O, kv_start=st,
+                                                      max_len=int(lens.max())), reps=10)
+        by = (T * h.hkv * h.d * 2 * 2 + 2 * len(lens) * h.hq * h.d * 2) * n_layers
+        res[name] = {"rows": T, "ms": round(ms, 3), "gbs": round(by / ms / 1e6, 1),
+                     "kv_gb": round(T * h.hkv * h.d * 4 * n_layers / 1e9, 2)}
+        del K, V
+        torch.cuda.empty_cache()
+    res["speedup"] = round(res["full_context"]["ms"] / res["sonic_retained"]["ms"], 2)
+    return {"workload": f"56 decoding dialogues of the mixed serving step, {n_layers} layers, "
+                        "28/4 heads, D=128", "results": res}
+
+
+def extra_nexus_gen():
+    """Nexus generation with incremental compaction (Sec. 3.1, Table 3's
+    "Nexus Gen." step) at the masked-prefill shapes: batch 8, 32 layers, 32/8
+    heads, D = 128, 512 system tokens, 16 segments of 256 body + 32 Nexus.
+    Segment i: the 32 Nexus rows attend over [retained | body_i | Nexus_i]
+    (one prefill launch for the batch and all layers), then compaction drops
+    body_i.  Inputs of every segment step are staged beforehand; the timed
+    region is the 16 prefill and 16 compaction launches."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    batch, hd = inputs.masked_prefill()
+    d = batch.dialogues[0]
+    B, NL = batch.B, hd.n_layers
+    sysl, segs = d.sys_len, d.segments
+    steps = []
+    flops = comp_bytes = 0.0
+    for i, (nb, nk) in enumerate(segs, start=1):
+        r_len = sysl + sum(k for _, k in segs[:i - 1])
+        L = r_len + nb + nk
+        role = np.concatenate([np.zeros(sysl, np.uint8), np.full(r_len - sysl, 2, np.uint8),
+                               np.full(nb, 1, np.uint8), np.full(nk, 2, np.uint8)])
+        seg = np.concatenate([np.zeros(sysl, np.int32),
+                              np.repeat(np.arange(1, i, dtype=np.int32), [k for _, k in segs[:i - 1]]),
+                              np.full(nb + nk, i, np.int32)])
+        K = inputs.randn((NL, B * L, hd.hkv, hd.d), seed=100 + i, device=dev)
+        V = inputs.randn((NL, B * L, hd.hkv, hd.d), seed=200 + i, device=dev)
+        Q = inputs.randn((NL, B * nk, hd.hq, hd.d), seed=300 + i, device=dev)
+        O = torch.empty_like(Q)
+        ks = t(np.arange(B, dtype=np.int32) * L)
+        kl = t(np.full(B, L, np.int32))
+        qs = t(np.arange(B, dtype=np.int32) * nk)
+        ql = t(np.full(B, nk, np.int32))
+        R = r_len + nk
+        oK = torch.empty((NL, B * R, hd.hkv, hd.d), dtype=K.dtype, device=dev)
+        oV = torch.empty_like(oK)
+        off = torch.zeros(B + 1, dtype=torch.int32, device=dev)
+        steps.append(dict(K=K, V=V, Q=Q, O=O, ks=ks, kl=kl, qs=qs, ql=ql, L=L, nk=nk,
+                          role=t(np.tile(role, B)), seg=t(np.tile(seg, B)), oK=oK, oV=oV, off=off))
+        flops += 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L - nk, L), 0) * B * NL
+        comp_bytes += 2.0 * R * B * hd.hkv * hd.d * 2 * 2 * NL
+
+    def prefills():
+        for s in steps:
+            sonic.sonic_attn_prefill(s["Q"], s["K"], s["V"], s["seg"], s["role"], s["O"],
+                                     k_start=s["ks"], k_len=s["kl"], q_start=s["qs"],
+                                     q_len=s["ql"], max_q_len=s["nk"], max_k_len=s["L"])
+
+    def compactions():
+        for s in steps:
+            sonic.sonic_compact_kv(s["K"], s["V"], s["seg"], s["role"], s["oK"], s["oV"],
+                                   s["off"], k_start=s["ks"], k_len=s["kl"])
+
+    p_ms = _ev_time(prefills)
+    c_ms = _ev_time(compactions)
+    return {"workload": "Nexus generation: batch 8, 32 layers, 32/8 heads, D=128, "
+                        "16 segments of 256 body + 32 Nexus after 512 system tokens",
+            "results": {"prefill_ms_all_segments": round(p_ms, 3),
+                        "prefill_tflops": round(flops / p_ms / 1e9, 1),
+                        "compaction_ms_all_segments": round(c_ms, 3),
+                        "compaction_gbs": round(comp_bytes / c_ms / 1e6, 1),
+                        "ms_per_segment": round((p_ms + c_ms) / len(segs), 3)}}
+
+
+EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
+          "context": extra_context, "nexus_gen": extra_nexus_gen}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -531,9 +742,18 @@ def main():
     ap.add_argument("--only", choices=["compact", "prefill", "decode"], default=None,
                     help="time one phase alone (for profiler captures)")
     ap.add_argument("--layers", type=int, default=0, help="override the layer count")
+    ap.add_argument("--extra", choices=sorted(EXTRAS), default=None,
+                    help="time a further workload instead of the benchmark step")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
+
+    if args.extra:
+        if rank == 0:
+            out = EXTRAS[args.extra]()
+            out["extra"] = args.extra
+            print(json.dumps(out))
+        return
 
     if args.impl == "reference":
         if rank != 0:
