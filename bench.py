@@ -174,7 +174,7 @@ class GpuStep:
         self.outV = self.Vret[:, lay.T_dec:]
         # workspaces (caller-owned; sized once)
         self.ws_c = self.ws_p = self.ws_d = None
-        self.launches_per_step = 3 + 2 + 2
+        self.launches_per_step = 4 + 2 + 2
 
     def compact(self, stream=None):
         self.ws_c = self.sonic.sonic_compact_kv(

@@ -147,7 +147,8 @@ typedef struct {
  * (non-decreasing within a sequence, no body row in segment 0) and a
  * violation sets SONIC_ERR_LAYOUT.  If offsets[B] > out_capacity_rows the
  * call sets SONIC_ERR_CAPACITY and copies only rows below the capacity.
- * K/V/out pointers must be 16-byte aligned.
+ * K/V/out pointers must be 16-byte aligned.  B > 65535 or n_layers > 32767
+ * returns SONIC_ERR_UNSUPPORTED.
  */
 SONIC_API sonic_status_t sonic_compact_kv(const void *K, const void *V, const int32_t *seg_id,
                                 const uint8_t *role, void *out_K, void *out_V,

@@ -5,13 +5,17 @@
 // effective context is I_sys + Nexus state + current query): a row is kept
 // iff its role is not BODY; kept rows keep their order.
 //
-// Three launches, none of which needs a host round trip:
-//   keep_count    one block per sequence: number of kept rows (and a layout
-//                 check when segment numbers are given);
-//   keep_scatter  one block per sequence: its output offset (sum over
-//                 earlier sequences), then a block-wide prefix scan of the
-//                 keep flags built from warp-shuffle scans, writing the
-//                 source row of every output row (-1 in reserve rows);
+// Four launches, none of which needs a host round trip:
+//   keep_count    one block per (chunk, sequence), each sequence cut into
+//                 kChunks pieces: kept rows of the piece (and a layout check
+//                 when segment numbers are given);
+//   keep_bases    one block: per-sequence totals and their exclusive scan
+//                 (with the reserve rows) -> offsets, ret_len, capacity check;
+//   keep_scatter  one block per (chunk, sequence): its output base (the
+//                 sequence's offset plus the pieces before it), then a block
+//                 prefix scan of the keep flags from warp-shuffle scans,
+//                 writing the source row of every output row (-1 in reserve
+//                 rows);
 //   kv_gather     all layers, K and V: 16-byte vector copy of every kept row
 //                 to its output row, grid-stride over rows of each layer.
 #include "sonic_dev.cuh"
@@ -21,23 +25,33 @@ namespace sonic {
 namespace {
 
 constexpr int kScanThreads = 512;
+constexpr int kChunks = 64;  // pieces per sequence in the scans
+
+// Rows [*lo, *hi) of piece c of a sequence of len rows (32-row aligned pieces).
+__device__ __forceinline__ void piece(int32_t len, int c, int32_t *lo, int32_t *hi) {
+    const long long ch = (((long long)len + kChunks - 1) / kChunks + 31) & ~31LL;
+    *lo = (int32_t)min((long long)len, c * ch);
+    *hi = (int32_t)min((long long)len, (c + 1) * ch);
+}
 
 __global__ void __launch_bounds__(kScanThreads)
 keep_count_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                   const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
                   int32_t *__restrict__ counts, int32_t *status) {
-    const int b = blockIdx.x;
-    const int32_t start = k_start[b], len = k_len[b];
+    const int c = blockIdx.x, b = blockIdx.y;
+    const int32_t start = k_start[b];
+    int32_t lo, hi;
+    piece(k_len[b], c, &lo, &hi);
     int n = 0;
     bool bad = false;
-    for (int32_t t = threadIdx.x; t < len; t += blockDim.x) {
+    for (int32_t t = lo + threadIdx.x; t < hi; t += blockDim.x) {
         uint8_t r = role[start + t];
         n += (r != SONIC_ROLE_BODY);
         bad |= (r > SONIC_ROLE_CURR);
         if (seg != nullptr) {
-            int32_t s = seg[start + t];
-            bad |= (r == SONIC_ROLE_BODY && s <= 0);
-            if (t > 0) bad |= (s < seg[start + t - 1]);
+            int32_t sv = seg[start + t];
+            bad |= (r == SONIC_ROLE_BODY && sv <= 0);
+            if (t > 0) bad |= (sv < seg[start + t - 1]);
         }
     }
     // block reduction
@@ -50,9 +64,9 @@ keep_count_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ 
     if (bad) bad_any = 1;
     __syncthreads();
     if (threadIdx.x == 0) {
-        int s = 0;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
-        counts[b] = s;
+        int sum = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) sum += red[w];
+        counts[b * kChunks + c] = sum;
         if (bad_any) set_status(status, SONIC_ERR_LAYOUT);
     }
 }
@@ -68,52 +82,74 @@ __device__ __forceinline__ int warp_inclusive_scan(int v) {
     return v;
 }
 
+// Exclusive scan over the sequences of (kept rows + reserve): one block.
+__global__ void __launch_bounds__(kScanThreads)
+keep_bases_kernel(const int32_t *__restrict__ counts, const int32_t *__restrict__ reserve,
+                  int32_t B, int32_t capacity, long long *__restrict__ seq_base,
+                  int32_t *__restrict__ offsets, int32_t *__restrict__ ret_len,
+                  int32_t *status) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int kWarps = kScanThreads / 32;
+    __shared__ long long warp_tot[kWarps];
+    long long running = 0;
+    for (int32_t b0 = 0; b0 < B; b0 += blockDim.x) {
+        const int32_t b = b0 + tid;
+        long long v = 0;
+        int32_t kept = 0;
+        if (b < B) {
+            for (int c = 0; c < kChunks; ++c) kept += counts[b * kChunks + c];
+            v = (long long)kept + (reserve ? reserve[b] : 0);
+        }
+        // inclusive warp scan of v
+        long long incl = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            long long u = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += u;
+        }
+        if (lane == 31) warp_tot[warp] = incl;
+        __syncthreads();
+        long long wb = 0, tot = 0;
+        for (int w = 0; w < kWarps; ++w) {
+            if (w < warp) wb += warp_tot[w];
+            tot += warp_tot[w];
+        }
+        if (b < B) {
+            const long long base = running + wb + incl - v;
+            seq_base[b] = base;
+            offsets[b] = (int32_t)base;
+            if (ret_len) ret_len[b] = kept;
+        }
+        running += tot;
+        __syncthreads();
+    }
+    if (tid == 0) {
+        offsets[B] = (int32_t)running;
+        if (running > capacity || running > 0x7fffffffLL) set_status(status, SONIC_ERR_CAPACITY);
+    }
+}
+
 __global__ void __launch_bounds__(kScanThreads)
 keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                     const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
                     const int32_t *__restrict__ reserve, const int32_t *__restrict__ counts,
-                    int32_t B, int32_t capacity, int32_t *__restrict__ offsets,
-                    int32_t *__restrict__ ret_len, int32_t *__restrict__ src_idx,
-                    uint8_t *__restrict__ out_role, int32_t *__restrict__ out_seg,
-                    int32_t *status) {
-    const int b = blockIdx.x;
+                    const long long *__restrict__ seq_base, int32_t capacity,
+                    int32_t *__restrict__ src_idx, uint8_t *__restrict__ out_role,
+                    int32_t *__restrict__ out_seg) {
+    const int c = blockIdx.x, b = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     constexpr int kWarps = kScanThreads / 32;
     __shared__ int warp_tot[kWarps];
-    __shared__ long long base_sh;
-
-    // Output offset of this sequence: sum of (count + reserve) over b' < b.
-    long long part = 0;
-    for (int i = tid; i < b; i += blockDim.x)
-        part += (long long)counts[i] + (reserve ? reserve[i] : 0);
-    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-    __shared__ long long red[kWarps];
-    if (lane == 0) red[warp] = part;
-    __syncthreads();
-    if (tid == 0) {
-        long long s = 0;
-        for (int w = 0; w < kWarps; ++w) s += red[w];
-        base_sh = s;
-    }
-    __syncthreads();
-    const long long base = base_sh;
-    const int32_t count = counts[b];
-    const int32_t res = reserve ? reserve[b] : 0;
-    const long long end = base + count + res;
-    if (tid == 0) {
-        offsets[b] = (int32_t)base;
-        if (b == B - 1) offsets[B] = (int32_t)end;
-        if (ret_len) ret_len[b] = count;
-        if (end > capacity || end > 0x7fffffffLL) set_status(status, SONIC_ERR_CAPACITY);
-    }
-    if (src_idx == nullptr && out_role == nullptr && out_seg == nullptr) return;
-
-    // Block-wide exclusive scan of the keep flags, chunk by chunk.
+    // output base of this piece: the sequence's offset plus the earlier pieces
+    long long base = seq_base[b];
+    for (int i = 0; i < c; ++i) base += counts[b * kChunks + i];
     const int32_t start = k_start[b], len = k_len[b];
+    int32_t lo, hi;
+    piece(len, c, &lo, &hi);
     long long running = base;
-    for (int32_t c0 = 0; c0 < len; c0 += blockDim.x) {
+    for (int32_t c0 = lo; c0 < hi; c0 += blockDim.x) {
         const int32_t t = c0 + tid;
-        const int keep = (t < len) && (role[start + t] != SONIC_ROLE_BODY);
+        const int keep = (t < hi) && (role[start + t] != SONIC_ROLE_BODY);
         int incl = warp_inclusive_scan(keep);
         if (lane == 31) warp_tot[warp] = incl;
         __syncthreads();
@@ -132,13 +168,18 @@ keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
         running += chunk_tot;
         __syncthreads();
     }
-    // Reserve rows: no source.
-    for (int32_t r = tid; r < res; r += blockDim.x) {
-        const long long o = base + count + r;
-        if (o < capacity) {
-            if (src_idx) src_idx[o] = -1;
-            if (out_role) out_role[o] = SONIC_ROLE_BODY;
-            if (out_seg) out_seg[o] = -1;
+    // Reserve rows (piece 0 writes them): no source.
+    if (c == 0 && reserve != nullptr) {
+        long long kept = 0;
+        for (int i = 0; i < kChunks; ++i) kept += counts[b * kChunks + i];
+        const int32_t res = reserve[b];
+        for (int32_t r = tid; r < res; r += blockDim.x) {
+            const long long o = seq_base[b] + kept + r;
+            if (o < capacity) {
+                if (src_idx) src_idx[o] = -1;
+                if (out_role) out_role[o] = SONIC_ROLE_BODY;
+                if (out_seg) out_seg[o] = -1;
+            }
         }
     }
 }
@@ -211,7 +252,10 @@ using namespace sonic;
 
 extern "C" size_t sonic_compact_workspace_size(const sonic_compact_args *a) {
     if (a == nullptr || a->batch < 0) return 0;
-    size_t ws = round_up((size_t)a->batch * sizeof(int32_t), 256);
+    // per-piece counts, then per-sequence 64-bit bases, then (if the caller
+    // gives no src_idx) the source row of every output row
+    size_t ws = round_up((size_t)a->batch * kChunks * sizeof(int32_t), 256) +
+                round_up((size_t)a->batch * sizeof(long long), 256);
     if (a->src_idx == nullptr)
         ws += round_up((size_t)(a->out_capacity_rows > 0 ? a->out_capacity_rows : 0) *
                            sizeof(int32_t),
@@ -242,22 +286,27 @@ extern "C" sonic_status_t sonic_compact_kv(const void *K, const void *V, const i
         return SONIC_ERR_INVALID_ARGUMENT;
     if (!aligned16(K) || !aligned16(V) || !aligned16(out_K) || !aligned16(out_V))
         return SONIC_ERR_INVALID_ARGUMENT;
-    if (a->n_layers > 32767) return SONIC_ERR_UNSUPPORTED;
+    if (a->n_layers > 32767 || a->batch > 65535) return SONIC_ERR_UNSUPPORTED;
     const size_t need = sonic_compact_workspace_size(a);
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
 
-    int32_t *counts = static_cast<int32_t *>(a->workspace);
-    int32_t *src_idx = a->src_idx;
-    if (src_idx == nullptr)
-        src_idx = reinterpret_cast<int32_t *>(static_cast<char *>(a->workspace) +
-                                              round_up((size_t)a->batch * 4, 256));
+    char *ws = static_cast<char *>(a->workspace);
+    int32_t *counts = reinterpret_cast<int32_t *>(ws);
+    ws += round_up((size_t)a->batch * kChunks * sizeof(int32_t), 256);
+    long long *seq_base = reinterpret_cast<long long *>(ws);
+    ws += round_up((size_t)a->batch * sizeof(long long), 256);
+    int32_t *src_idx = a->src_idx != nullptr ? a->src_idx : reinterpret_cast<int32_t *>(ws);
 
-    keep_count_kernel<<<a->batch, kScanThreads, 0, stream>>>(role, seg_id, a->k_start, a->k_len,
-                                                            counts, a->status);
-    keep_scatter_kernel<<<a->batch, kScanThreads, 0, stream>>>(
-        role, seg_id, a->k_start, a->k_len, a->reserve, counts, a->batch, a->out_capacity_rows,
-        offsets, a->ret_len, src_idx, a->out_role, a->out_seg, a->status);
+    const dim3 pieces(kChunks, a->batch);
+    keep_count_kernel<<<pieces, kScanThreads, 0, stream>>>(role, seg_id, a->k_start, a->k_len,
+                                                          counts, a->status);
+    keep_bases_kernel<<<1, kScanThreads, 0, stream>>>(counts, a->reserve, a->batch,
+                                                      a->out_capacity_rows, seq_base, offsets,
+                                                      a->ret_len, a->status);
+    keep_scatter_kernel<<<pieces, kScanThreads, 0, stream>>>(
+        role, seg_id, a->k_start, a->k_len, a->reserve, counts, seq_base, a->out_capacity_rows,
+        src_idx, a->out_role, a->out_seg);
     const int sms = device_sm_count();
     // Enough blocks per (layer, K|V) to keep every SM busy with ~8 blocks.
     const int per_slice = (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers);

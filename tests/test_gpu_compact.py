@@ -120,3 +120,19 @@ def test_masked_prefill_workload_all_layers():
         for name, raw in (("oK", K), ("oV", V)):
             want = oracle.compact_copy(_bytes(raw[layer:layer + 1]), off, ret_len, src, int(off[-1]))
             assert np.array_equal(_bytes(r[name][layer:layer + 1]), want), f"{name} layer {layer}"
+
+
+def test_many_sequences_and_long_pieces():
+    """1,100 sequences (the base scan runs over more than one 512-wide block
+    pass) plus one sequence of about 70,000 rows (each of its 64 scan pieces
+    spans several 512-row passes), reserve rows on every sequence."""
+    rng = np.random.default_rng(8)
+    ds = [inputs.random_dialogue(rng, max_segments=3, max_body=40, max_nexus=6, max_sys=8,
+                                 max_curr=9) for _ in range(1100)]
+    ds.insert(517, inputs.Dialogue(33, [(700, 13), (1, 0), (0, 9)] * 99 + [(1500, 1)], 77))
+    batch = inputs.Batch(ds)
+    reserve = rng.integers(0, 5, batch.B)
+    K = inputs.randn((1, batch.total, 1, 64), seed=6, device=H.dev())
+    V = inputs.randn((1, batch.total, 1, 64), seed=7, device=H.dev())
+    r = _run(batch, K, V, reserve=reserve)
+    _check(batch, K, V, r, reserve=reserve)
