@@ -14,6 +14,9 @@ builds that file with gcc and marshals numpy arrays into it:
 * :func:`compact_copy`  -- byte copy of retained rows for all layers.
 * :func:`attn_masked`   -- masked softmax attention for selected query rows.
 * :func:`decode`        -- one decode step over a retained cache.
+* :func:`nexus_mass`    -- attention mass on Nexus keys per query row and head
+                           (the quantity behind A_nexus, Sec. 4.1 Eq. 9).
+* :func:`decode_nexus_mass` -- the same for one decode step.
 """
 from __future__ import annotations
 
@@ -73,6 +76,11 @@ class Oracle:
         lib.orc_attn_masked.restype = None
         lib.orc_decode.argtypes = [i64, i32, i32, i32, P, P, P, f64, P, P, P]
         lib.orc_decode.restype = None
+        lib.orc_nexus_mass.argtypes = [i64, i32, i32, i32, P, P, P, P, P, i64, f64,
+                                       ctypes.c_int, P, P]
+        lib.orc_nexus_mass.restype = None
+        lib.orc_decode_nexus_mass.argtypes = [i64, i32, i32, i32, P, P, P, f64, P, P]
+        lib.orc_decode_nexus_mass.restype = None
         self.lib = lib
         self.path = so_path
 
@@ -169,6 +177,43 @@ class Oracle:
                             _ptr(s_buf), _ptr(O), _ptr(lse))
         return O, lse
 
+    def nexus_mass(self, Q, K, role, seg, rows, scale=None, nexus_mode=NEXUS_FULL):
+        """Share of each query row's attention (per head) on visible Nexus keys.
+
+        Q: [n_rows, Hq, D]; K: [L, Hkv, D]; rows: positions of the queries.
+        Returns mass [n_rows, Hq] float64.
+        """
+        Q = _c(Q, np.float64)
+        K = _c(K, np.float64)
+        role = _c(role, np.uint8)
+        seg = _c(seg, np.int32)
+        rows = _c(rows, np.int64)
+        n_rows, Hq, D = Q.shape
+        L, Hkv, _ = K.shape
+        if scale is None:
+            scale = 1.0 / np.sqrt(D)
+        mass = np.zeros((n_rows, Hq), np.float64)
+        s_buf = np.zeros(max(L, 1), np.float64)
+        self.lib.orc_nexus_mass(L, Hq, Hkv, D, _ptr(Q), _ptr(K), _ptr(role), _ptr(seg),
+                                _ptr(rows), n_rows, float(scale), nexus_mode, _ptr(s_buf),
+                                _ptr(mass))
+        return mass
+
+    def decode_nexus_mass(self, q, K, role, scale=None):
+        """Decode form: q [Hq, D]; K [n, Hkv, D]; role [n]. Returns mass [Hq]."""
+        q = _c(q, np.float64)
+        K = _c(K, np.float64)
+        role = _c(role, np.uint8)
+        Hq, D = q.shape
+        n, Hkv, _ = K.shape
+        if scale is None:
+            scale = 1.0 / np.sqrt(D)
+        mass = np.zeros(Hq, np.float64)
+        s_buf = np.zeros(max(n, 1), np.float64)
+        self.lib.orc_decode_nexus_mass(n, Hq, Hkv, D, _ptr(q), _ptr(K), _ptr(role),
+                                       float(scale), _ptr(s_buf), _ptr(mass))
+        return mass
+
 
 def _ptr(a):
     return None if a is None else a.ctypes.data
@@ -209,3 +254,11 @@ def attn_masked(*a, **k):
 
 def decode(*a, **k):
     return default().decode(*a, **k)
+
+
+def nexus_mass(*a, **k):
+    return default().nexus_mass(*a, **k)
+
+
+def decode_nexus_mass(*a, **k):
+    return default().decode_nexus_mass(*a, **k)

@@ -250,3 +250,90 @@ void orc_decode(int64_t n, int32_t Hq, int32_t Hkv, int32_t D, const double *q,
             lse[h] = m + log(denom);
     }
 }
+
+/*
+ * Attention mass on Nexus keys: the per-row, per-head quantity behind
+ * A_nexus of the Nexus attention regularisation (Sec. 4.1, Eq. 9, "the
+ * average attention weight assigned to Nexus tokens by the current query").
+ * For each selected query row p and query head h, with the softmax of
+ * orc_attn_masked (scores s_q over the keys visible to p under the Sec. 3.2
+ * rule):
+ *   mass[p,h] = sum_{q visible, role[q] = NEXUS} e^{s_q}
+ *             / sum_{q visible} e^{s_q},
+ * 0 when p sees no key.  Same argument layout as orc_attn_masked; mass is
+ * [n_rows][Hq].
+ */
+void orc_nexus_mass(int64_t L, int32_t Hq, int32_t Hkv, int32_t D,
+                    const double *Q, const double *K, const uint8_t *role,
+                    const int32_t *seg, const int64_t *rows, int64_t n_rows,
+                    double scale, int nexus_mode, double *s_buf, double *mass)
+{
+    int32_t G = Hq / Hkv;
+    for (int64_t i = 0; i < n_rows; ++i) {
+        int64_t p = rows[i];
+        for (int32_t h = 0; h < Hq; ++h) {
+            int32_t hk = h / G;
+            const double *qv = Q + (i * Hq + h) * (int64_t)D;
+            double m = -INFINITY;
+            for (int64_t q = 0; q < L; ++q) {
+                if (!orc_visible(p, q, role, seg, nexus_mode)) {
+                    s_buf[q] = -INFINITY;
+                    continue;
+                }
+                const double *kv = K + (q * Hkv + hk) * (int64_t)D;
+                double s = 0.0;
+                for (int32_t d = 0; d < D; ++d)
+                    s += qv[d] * kv[d];
+                s *= scale;
+                s_buf[q] = s;
+                if (s > m)
+                    m = s;
+            }
+            double all = 0.0, nexus = 0.0;
+            for (int64_t q = 0; q < L; ++q) {
+                if (s_buf[q] == -INFINITY)
+                    continue;
+                double w = exp(s_buf[q] - m);
+                all += w;
+                if (role[q] == ORC_NEXUS)
+                    nexus += w;
+            }
+            mass[i * Hq + h] = all > 0.0 ? nexus / all : 0.0;
+        }
+    }
+}
+
+/*
+ * The same mass for one decode step (App. C): the new token's query q
+ * [Hq][D] sees every one of the n retained rows K [n][Hkv][D], whose roles
+ * are role[n]; mass is [Hq], 0 when n = 0.
+ */
+void orc_decode_nexus_mass(int64_t n, int32_t Hq, int32_t Hkv, int32_t D,
+                           const double *q, const double *K, const uint8_t *role,
+                           double scale, double *s_buf, double *mass)
+{
+    int32_t G = Hq / Hkv;
+    for (int32_t h = 0; h < Hq; ++h) {
+        int32_t hk = h / G;
+        const double *qv = q + (int64_t)h * D;
+        double m = -INFINITY;
+        for (int64_t t = 0; t < n; ++t) {
+            const double *kv = K + (t * Hkv + hk) * (int64_t)D;
+            double s = 0.0;
+            for (int32_t d = 0; d < D; ++d)
+                s += qv[d] * kv[d];
+            s *= scale;
+            s_buf[t] = s;
+            if (s > m)
+                m = s;
+        }
+        double all = 0.0, nexus = 0.0;
+        for (int64_t t = 0; t < n; ++t) {
+            double w = exp(s_buf[t] - m);
+            all += w;
+            if (role[t] == ORC_NEXUS)
+                nexus += w;
+        }
+        mass[h] = all > 0.0 ? nexus / all : 0.0;
+    }
+}

@@ -272,6 +272,67 @@ def test_decode_equals_unmasked_sdpa():
     assert (o0 == 0).all() and np.isneginf(l0).all()
 
 
+# ------------------------------------------- Nexus attention mass (Sec. 4.1, Eq. 9)
+
+def _sdpa_nexus_share(Q, K, role, add_mask):
+    """Share of the attention on Nexus keys through torch SDPA: with V the
+    indicator of a Nexus key (one value channel), the output is the mass."""
+    Vn = np.zeros((K.shape[0], K.shape[1], 1))
+    Vn[role == inputs.ROLE_NEXUS] = 1.0
+    return _sdpa(Q, K, Vn, add_mask, scale=1.0 / math.sqrt(Q.shape[2]))[:, :, 0]
+
+
+@pytest.mark.parametrize("mode", [oracle.NEXUS_FULL, oracle.NEXUS_CAUSAL_SEGMENTS])
+def test_nexus_mass_equals_sdpa_of_nexus_indicator(mode):
+    for i, d in enumerate(_dialogues()[:12]):
+        role, seg = d.arrays()
+        Q, K, _ = _qkv(d.length, 6, 2, 16, seed=60 + i)
+        mass = ORC().nexus_mass(Q, K, role, seg, np.arange(d.length), nexus_mode=mode)
+        want = _sdpa_nexus_share(Q, K, role, rule_mask(d, mode == oracle.NEXUS_CAUSAL_SEGMENTS))
+        np.testing.assert_allclose(mass, want, rtol=0, atol=1e-12)
+        assert ((mass >= 0) & (mass <= 1)).all()
+
+
+def test_nexus_mass_of_uniform_scores_counts_visible_nexus_keys():
+    """K = 0: every visible key gets the same weight, so the mass is the
+    share of Nexus keys among the keys the row sees."""
+    for d in _dialogues()[:12]:
+        role, seg = d.arrays()
+        Q, _, _ = _qkv(d.length, 2, 1, 8, seed=8)
+        K = np.zeros((d.length, 1, 8))
+        mass = ORC().nexus_mass(Q, K, role, seg, np.arange(d.length))
+        vis = rule_mask(d) == 0.0
+        nexus = role == inputs.ROLE_NEXUS
+        want = (vis & nexus[None, :]).sum(1) / vis.sum(1)
+        np.testing.assert_allclose(mass, np.repeat(want[:, None], 2, 1), rtol=0, atol=1e-14)
+
+
+def test_nexus_mass_zero_without_nexus_and_one_for_lone_nexus_rows():
+    d = inputs.Dialogue(5, [(7, 0), (4, 0)], 6)          # no Nexus at all
+    role, seg = d.arrays()
+    Q, K, _ = _qkv(d.length, 2, 1, 8, seed=4)
+    assert (ORC().nexus_mass(Q, K, role, seg, np.arange(d.length)) == 0).all()
+    d = inputs.Dialogue(0, [(0, 3)], 0)                  # only Nexus rows
+    role, seg = d.arrays()
+    Q, K, _ = _qkv(d.length, 2, 1, 8, seed=4)
+    assert (ORC().nexus_mass(Q, K, role, seg, np.arange(d.length)) == 1).all()
+
+
+def test_decode_nexus_mass_equals_sdpa_and_current_rows_of_prefill():
+    """Decode over a retained cache (system, Nexus, current rows): equal to
+    SDPA of the Nexus indicator, and to the prefill mass of the last current
+    row over the same cache (Sec. 3.2: it sees every retained row)."""
+    d = inputs.Dialogue(6, [(0, 4), (0, 5), (0, 3)], 7)  # a retained cache
+    role, seg = d.arrays()
+    Q, K, _ = _qkv(d.length, 8, 2, 16, seed=33)
+    m = ORC().decode_nexus_mass(Q[-1], K, role)
+    np.testing.assert_allclose(m, _sdpa_nexus_share(Q[-1:], K, role, np.zeros((1, d.length)))[0],
+                               rtol=0, atol=1e-12)
+    mp = ORC().nexus_mass(Q[-1:], K, role, seg, np.array([d.length - 1]))
+    np.testing.assert_allclose(m, mp[0], rtol=0, atol=1e-13)
+    assert (ORC().decode_nexus_mass(Q[-1], K[:0], role[:0]) == 0).all()
+
+
 # ------------------------------------------------------------ mutants
 
 _MUTANTS = {
@@ -289,6 +350,14 @@ _MUTANTS = {
                  "                s_buf[q] = s;"),
     # retention keeps the bodies
     "keep_bodies": ("if (role[row] != ORC_BODY) {", "if (role[row] != 255) {"),
+    # Nexus mass counts every retained role, not just Nexus keys
+    "mass_any_retained": ("if (role[q] == ORC_NEXUS)\n                    nexus += w;",
+                          "if (role[q] != ORC_BODY)\n                    nexus += w;"),
+    # Nexus mass of a decode step over the current-turn rows instead
+    "decode_mass_curr": ("if (role[t] == ORC_NEXUS)", "if (role[t] == ORC_CURR)"),
+    # Nexus mass ignores the mask (every key's weight in the denominator)
+    "mass_unmasked": ("            double all = 0.0, nexus = 0.0;\n            for (int64_t q = 0; q < L; ++q) {\n                if (s_buf[q] == -INFINITY)\n                    continue;",
+                      "            double all = 0.0, nexus = 0.0;\n            for (int64_t q = 0; q < L; ++q) {\n                if (s_buf[q] == -INFINITY)\n                    s_buf[q] = m;"),
 }
 
 
@@ -315,6 +384,18 @@ def _run_pins(orc):
         if ret_len[0] != d.recipe_retained:
             failed.append("retention")
             break
+    for i, d in enumerate(ds[:6]):
+        role, seg = d.arrays()
+        Q, K, _ = _qkv(d.length, 4, 2, 16, seed=40 + i)
+        mass = orc.nexus_mass(Q, K, role, seg, np.arange(d.length))
+        if not np.allclose(mass, _sdpa_nexus_share(Q, K, role, rule_mask(d)), rtol=0, atol=1e-12):
+            failed.append("nexus mass")
+            break
+    q, K, _ = _qkv(40, 4, 2, 16, seed=47, nq=1)
+    role = np.random.default_rng(3).choice([0, 2, 3], 40).astype(np.uint8)
+    if not np.allclose(orc.decode_nexus_mass(q[0], K, role),
+                       _sdpa_nexus_share(q, K, role, np.zeros((1, 40)))[0], rtol=0, atol=1e-12):
+        failed.append("decode nexus mass")
     return failed
 
 
@@ -326,7 +407,9 @@ def test_pins_pass_on_oracle():
 def test_pins_catch_planted_mistake(name, tmp_path):
     src = open(os.path.join(os.path.dirname(oracle.__file__), "sonic_oracle.c")).read()
     old, new = _MUTANTS[name]
-    assert src.count(old) == 1, f"mutation site for {name} not unique"
+    # the attention loops of orc_attn_masked and orc_nexus_mass share some
+    # sites: a mutation is planted in every copy of its site
+    assert src.count(old) >= 1, f"mutation site for {name} not found"
     mutant = tmp_path / f"mutant_{name}.c"
     mutant.write_text(src.replace(old, new))
     so = oracle.compile_source(str(mutant), str(tmp_path / f"mutant_{name}.so"))
