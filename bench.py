@@ -728,7 +728,44 @@ def extra_nexus_gen():
                         "ms_per_segment": round((p_ms + c_ms) / len(segs), 3)}}
 
 
+def extra_nexus_mass():
+    """Cost of the attention-mass output (Sec. 4.1 Eq. 9's A_nexus per row and
+    head) on the mixed serving step at 8 layers: its prefill and its decode
+    launch, each with and without the mass (same inputs, same outputs
+    otherwise)."""
+    import torch
+    dev = torch.device("cuda", 0)
+    lay = Layout(n_layers=8)
+    g = GpuStep(lay, dev)
+    sonic = g.sonic
+    mass_p = torch.empty((lay.NL, lay.T_q, lay.HQ), dtype=torch.float32, device=dev)
+    mass_d = torch.empty((lay.NL, lay.n_dec, lay.HQ), dtype=torch.float32, device=dev)
+
+    def prefill(m):
+        sonic.sonic_attn_prefill(
+            g.Qp, g.Kret, g.Vret, g.seg_ret, g.role_ret, g.Op, k_start=g.k_start_pre,
+            k_len=g.k_len_pre, q_start=g.q_start, q_len=g.q_len,
+            max_q_len=int(lay.q_len.max()), max_k_len=int(lay.k_len_pre.max()), nexus_mass=m)
+
+    def decode(m):
+        sonic.sonic_attn_decode(g.qd, g.Kret, g.Vret, g.dec_len, g.Od, kv_start=g.dec_start,
+                                max_len=int(lay.dec_len.max()), role=g.role_ret, nexus_mass=m)
+
+    res = {}
+    for name, fn, m in (("prefill", prefill, mass_p), ("decode", decode, mass_d)):
+        t0 = _ev_time(lambda: fn(None), reps=10)
+        t1 = _ev_time(lambda: fn(m), reps=10)
+        res[name] = {"ms": round(t0, 3), "ms_with_mass": round(t1, 3),
+                     "overhead_pct": round(100.0 * (t1 / t0 - 1.0), 1)}
+    pf = lay.prefill_flops()
+    res["prefill"]["tflops_with_mass"] = round(pf / res["prefill"]["ms_with_mass"] / 1e9, 1)
+    res["decode"]["gbs_with_mass"] = round(lay.decode_bytes() / res["decode"]["ms_with_mass"] / 1e6, 1)
+    return {"workload": "mixed serving step, 8 layers: prefill and decode with / without the "
+                        "attention mass on Nexus keys", "results": res}
+
+
 EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
+          "nexus_mass": extra_nexus_mass,
           "context": extra_context, "nexus_gen": extra_nexus_gen}
 
 

@@ -51,7 +51,7 @@
 extern "C" {
 #endif
 
-#define SONIC_ABI_VERSION 1
+#define SONIC_ABI_VERSION 2
 
 #if defined(__GNUC__)
 #define SONIC_API __attribute__((visibility("default")))
@@ -191,6 +191,8 @@ typedef struct {
     void *workspace;             /* device, sonic_prefill_workspace_size() bytes        */
     size_t workspace_bytes;
     int32_t key_order;           /* sonic_key_order_t                                   */
+    float *nexus_mass;           /* device [n_layers][total_q_rows][Hq] or NULL: share of
+                                    each row's attention on visible Nexus keys          */
 } sonic_prefill_args;
 
 /*
@@ -209,6 +211,12 @@ typedef struct {
  * no key (padding).  key_order picks the order the key tiles are cut in
  * (sonic_key_order_t).  A sequence with q_len[b] > k_len[b] or k_len[b] >
  * max_k_len is refused with SONIC_ERR_INVALID_ARGUMENT in *status.
+ * nexus_mass (optional) is the per-row, per-head quantity behind A_nexus of
+ * the Nexus attention regularisation (Sec. 4.1, Eq. 9):
+ *   nexus_mass[i, h] = sum_{q in vis, role[q] = NEXUS} softmax(s)_q
+ * (0 when nothing is visible), normalised like O, i.e. over the bf16-rounded
+ * probabilities the P.V product uses.  The paper's A_nexus is its mean over
+ * heads and current-turn rows, a reduction left to the caller.
  */
 SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
                                   const int32_t *seg_id, const uint8_t *role, uint16_t *O,
@@ -277,6 +285,10 @@ typedef struct {
     int32_t *status;             /* device int32 or NULL                                */
     void *workspace;             /* device, sonic_decode_workspace_size() bytes         */
     size_t workspace_bytes;
+    const uint8_t *role;         /* device [total_kv_rows] or NULL: role of each retained
+                                    row (needed for nexus_mass)                         */
+    float *nexus_mass;           /* device [n_layers][B][Hq] or NULL: share of the
+                                    attention on rows whose role is SONIC_ROLE_NEXUS    */
 } sonic_decode_args;
 
 /*
@@ -291,7 +303,12 @@ typedef struct {
  * per SM claims units from a counter in the workspace (zeroed on `stream`
  * before the launch), so the workspace is never empty there and concurrent
  * calls need workspaces of their own.  lens[b] = 0 gives zeros (and
- * lse = -inf).  bf16 in/out, fp32 arithmetic.
+ * lse = -inf).  bf16 in/out, fp32 arithmetic.  nexus_mass (optional, role
+ * then required, else SONIC_ERR_INVALID_ARGUMENT) is the decode form of the
+ * quantity behind A_nexus (Sec. 4.1, Eq. 9): the share of the new token's
+ * attention, per query head, on retained rows t with role[kv_start[b] + t]
+ * = SONIC_ROLE_NEXUS (0 when lens[b] = 0); it adds one float per (unit,
+ * chunk) to the workspace.
  */
 SONIC_API sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
                                  const uint16_t *V_ret, const int32_t *lens, uint16_t *O,

@@ -54,6 +54,11 @@ struct DecParams {
     float *lse;
     float *part_acc;  // [units][max_chunks][D]
     float *part_ml;   // [units][max_chunks][2]
+    // attention mass on Nexus keys (when nexus_mass is given): the role of
+    // every key row, the output, and the per-chunk partial sums
+    const uint8_t *role;
+    float *nexus_mass;
+    float *part_nx;   // [units][max_chunks]
     int32_t *status;
     int B, Hq, Hkv, G;
     int64_t q_ls, o_ls;
@@ -163,12 +168,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
     }
 
     // ------------------------------------------------------------ consumers
-    float m[GT], l[GT];
+    // n: the part of l on Nexus keys (only when the mass is requested)
+    const bool want_nx = p.nexus_mass != nullptr;
+    float m[GT], l[GT], n[GT];
     float2 acc[GT][C::kDpl / 2];
 #pragma unroll
     for (int g = 0; g < GT; ++g) {
         m[g] = -INFINITY;
         l[g] = 0.f;
+        n[g] = 0.f;
 #pragma unroll
         for (int e = 0; e < C::kDpl / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
     }
@@ -181,6 +189,8 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
             const uint8_t *Ks = smem + s * C::kStageBytes;
             const uint8_t *Vs = Ks + C::kTileBytes;
             const int valid = min(kTileKeys, nkeys - t * kTileKeys);
+            const bool isn = want_nx && lane < valid &&
+                             p.role[row0 + t * kTileKeys + lane] == SONIC_ROLE_NEXUS;
 
             // scores: lane owns key `lane` of the tile
             float2 dk[GT];
@@ -210,6 +220,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
                 const float alpha = ex2(m[g] - mn);
                 const float pr = ex2(sc - mn);
                 l[g] = l[g] * alpha + pr;
+                if (want_nx) n[g] = n[g] * alpha + (isn ? pr : 0.f);
 #pragma unroll
                 for (int e = 0; e < C::kDpl / 2; ++e) {
                     acc[g][e].x *= alpha;
@@ -260,7 +271,10 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
 #pragma unroll
         for (int g = 0; g < GT; ++g)
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
+            for (int o = 16; o > 0; o >>= 1) {
+                l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
+                if (want_nx) n[g] += __shfl_xor_sync(0xffffffffu, n[g], o);
+            }
     }
     __syncthreads();
     if (*abort_flag) return;
@@ -268,6 +282,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
     // ---------------------------------------------------- merge the 4 warps
     float *macc = reinterpret_cast<float *>(smem);  // [warps][GT][D] (stage memory is free now)
     float *mml = macc + kConsumerWarps * GT * D;    // [warps][GT][2]
+    float *mnx = mml + kConsumerWarps * GT * 2;     // [warps][GT]
     if (warp < kConsumerWarps) {
 #pragma unroll
         for (int g = 0; g < GT; ++g) {
@@ -278,6 +293,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
             if (lane == 0) {
                 mml[(warp * GT + g) * 2 + 0] = m[g];
                 mml[(warp * GT + g) * 2 + 1] = l[g];
+                mnx[warp * GT + g] = n[g];
             }
         }
     }
@@ -289,23 +305,26 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
         float M = -INFINITY;
 #pragma unroll
         for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, mml[(w * GT + g) * 2]);
-        float L = 0.f, a = 0.f;
+        float L = 0.f, a = 0.f, N = 0.f;
 #pragma unroll
         for (int w = 0; w < kConsumerWarps; ++w) {
             const float f = ex2(mml[(w * GT + g) * 2] - M);
             L += f * mml[(w * GT + g) * 2 + 1];
             a += f * macc[(w * GT + g) * D + d];
+            N += f * mnx[w * GT + g];
         }
         if (n_chunks == 1) {
             uint16_t *op = p.O + layer * p.o_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G + g) * D;
             op[d] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
             if (d == 0 && p.lse != nullptr) p.lse[unit0 + g] = (M + __log2f(L)) * kLn2;
+            if (d == 0 && want_nx) p.nexus_mass[unit0 + g] = N / L;
         } else {
             const int64_t slot = (unit0 + g) * p.max_chunks + chunk;
             p.part_acc[slot * D + d] = a;
             if (d == 0) {
                 p.part_ml[slot * 2 + 0] = M;
                 p.part_ml[slot * 2 + 1] = L;
+                if (want_nx) p.part_nx[slot] = N;
             }
         }
     }
@@ -348,7 +367,8 @@ struct TcCfg {
     static constexpr int kPBytes = kTcN * kTcKeys * 2;           // 4 KB
     static constexpr int kOffRed = kOffP + 2 * kPBytes;          // [2][4][16] float
     static constexpr int kOffL = kOffRed + 2 * 4 * kTcN * 4;     // [4][16] float
-    static constexpr int kOffBar = kOffL + 4 * kTcN * 4;
+    static constexpr int kOffN = kOffL + 4 * kTcN * 4;           // [4][16] float
+    static constexpr int kOffBar = kOffN + 4 * kTcN * 4;
     static constexpr int kNumBars = 2 * kTcStages + 24;  // the pointers carved out below
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kSeqCache = 1024;                       // sequences whose lens/kv_start
@@ -408,6 +428,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     uint8_t *P_s = smem + C::kOffP;  // [2]
     float *red = reinterpret_cast<float *>(smem + C::kOffRed);
     float *lred = reinterpret_cast<float *>(smem + C::kOffL);
+    float *nred = reinterpret_cast<float *>(smem + C::kOffN);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
     uint64_t *full = bars;                    // [stages] K/V tile landed
     uint64_t *empty = bars + kTcStages;       // [stages] its P.V is done
@@ -697,17 +718,24 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         // Unit epilogue: normalise O^T of unit k and write it (or its partial).
         // It runs one tile into the next unit, when the unit's last P.V is long
         // done, so the move from one unit to the next costs no pipeline drain.
-        auto epilogue = [&](const TcUnit &w, int k, const float (&m)[GT],
-                            const float (&l)[GT]) -> bool {
+        const bool want_nx = p.nexus_mass != nullptr;
+        auto epilogue = [&](const TcUnit &w, int k, const float (&m)[GT], const float (&l)[GT],
+                            const float (&n)[GT]) -> bool {
             const uint32_t tOk = tO + (k & 1) * kTcN;
             if (!mbar_wait(&o_last[k & 1], (k >> 1) & 1, p.status, abort_flag)) return false;
             tc_fence_after();
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
-                float v = l[g];
+                float v = l[g], vn = n[g];
 #pragma unroll
-                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                if (lane == 0) lred[quarter * kTcN + g] = v;
+                for (int o = 16; o > 0; o >>= 1) {
+                    v += __shfl_xor_sync(0xffffffffu, v, o);
+                    if (want_nx) vn += __shfl_xor_sync(0xffffffffu, vn, o);
+                }
+                if (lane == 0) {
+                    lred[quarter * kTcN + g] = v;
+                    nred[quarter * kTcN + g] = vn;
+                }
             }
             mbar_arrive(ep_sync);
             if (!mbar_wait(ep_sync, k & 1, p.status, abort_flag)) return false;
@@ -715,10 +743,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             tmem_ld16(tOk + lane_base, o);
             tmem_ld_wait();
             reg_fence16(o);
-            float Lg[GT];
+            float Lg[GT], Ng[GT];
 #pragma unroll
-            for (int g = 0; g < GT; ++g)
+            for (int g = 0; g < GT; ++g) {
                 Lg[g] = lred[g] + lred[kTcN + g] + lred[2 * kTcN + g] + lred[3 * kTcN + g];
+                Ng[g] = nred[g] + nred[kTcN + g] + nred[2 * kTcN + g] + nred[3 * kTcN + g];
+            }
             // O^T of this unit is in registers and lred read: the buffers are free
             tc_fence_before();
             mbar_arrive(&o_free[k & 1]);
@@ -734,12 +764,14 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                         p.O + w.layer * p.o_ls + ((int64_t)w.b * p.Hq + (int64_t)w.kvh * G + g) * D;
                     op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
                     if (r == 0 && p.lse != nullptr) p.lse[unit0 + g] = (m[g] + __log2f(L)) * kLn2;
+                    if (r == 0 && want_nx) p.nexus_mass[unit0 + g] = Ng[g] / L;
                 } else {
                     const int64_t slot = (unit0 + g) * p.max_chunks + w.chunk;
                     p.part_acc[slot * D + r] = a;
                     if (r == 0) {
                         p.part_ml[slot * 2 + 0] = m[g];
                         p.part_ml[slot * 2 + 1] = L;
+                        if (want_nx) p.part_nx[slot] = Ng[g];
                     }
                 }
             }
@@ -748,7 +780,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         bool ok = true, pend = false;  // pend: unit kp still owes its epilogue
         int T = 0, kp = 0;
         TcUnit wp;
-        float mp[GT], lp[GT];
+        float mp[GT], lp[GT], np[GT];
         for (int k = 0; ok; ++k) {
             TcUnit w;
             if (lane == 0) read_unit(k, w);
@@ -759,13 +791,18 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             w.len = __shfl_sync(0xffffffffu, w.len, 0);
             tc_coords(p, units_x, w);
             const uint32_t tOk = tO + (k & 1) * kTcN;
-            float m[GT], l[GT];
+            float m[GT], l[GT], n[GT];
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
                 m[g] = -INFINITY;
                 l[g] = 0.f;
+                n[g] = 0.f;
             }
             for (int t = 0; t < w.ntiles; ++t, ++T) {
+                // this key's role, loaded before the wait (kept rows only)
+                const bool in_unit = t * kTcKeys + r < w.nkeys;
+                int role_k = 255;
+                if (want_nx && in_unit) role_k = p.role[w.row0 + t * kTcKeys + r];
                 if (!mbar_wait(&s_full[T & 1], (T >> 1) & 1, p.status, abort_flag)) {
                     ok = false;
                     break;
@@ -775,7 +812,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 tmem_ld16(tS + lane_base + (T & 1) * kTcN, sr);
                 tmem_ld_wait();
                 reg_fence16(sr);
-                const bool valid = t * kTcKeys + r < w.nkeys;
+                const bool valid = in_unit;
+                const bool isn = role_k == SONIC_ROLE_NEXUS;
                 float sv[GT];
                 float *rd = red + (T & 1) * 4 * kTcN;
 #pragma unroll
@@ -813,6 +851,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                     // the row sum adds the rounded probability P.V multiplies by
                     const __nv_bfloat16 pr = __float2bfloat16_rn(ex2(sv[g] - m[g]));
                     l[g] = l[g] * alpha[g] + __bfloat162float(pr);
+                    if (want_nx) n[g] = n[g] * alpha[g] + (isn ? __bfloat162float(pr) : 0.f);
                     *reinterpret_cast<__nv_bfloat16 *>(pb + g * 128 + ((jj ^ (g & 7)) << 4)) = pr;
                 }
                 if (!valid && r < ((w.nkeys - t * kTcKeys + 15) & ~15)) {
@@ -848,7 +887,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 tc_fence_before();
                 mbar_arrive(&p_full[T & 1]);
                 if (t == 0 && pend) {
-                    ok = epilogue(wp, kp, mp, lp);
+                    ok = epilogue(wp, kp, mp, lp, np);
                     pend = false;
                     if (!ok) break;
                 }
@@ -860,10 +899,11 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             for (int g = 0; g < GT; ++g) {
                 mp[g] = m[g];
                 lp[g] = l[g];
+                np[g] = n[g];
             }
             pend = true;
         }
-        if (ok && pend) epilogue(wp, kp, mp, lp);
+        if (ok && pend) epilogue(wp, kp, mp, lp, np);
     }
     tc_fence_before();
     __syncthreads();
@@ -891,6 +931,7 @@ decode_combine_kernel(const DecParams p, int n_layers) {
 #pragma unroll
         for (int e = 0; e < kDpl; ++e) op[lane * kDpl + e] = 0;
         if (lane == 0 && p.lse != nullptr) p.lse[unit] = -INFINITY;
+        if (lane == 0 && p.nexus_mass != nullptr) p.nexus_mass[unit] = 0.f;
         return;
     }
     const float *ml = p.part_ml + unit * p.max_chunks * 2;
@@ -899,13 +940,14 @@ decode_combine_kernel(const DecParams p, int n_layers) {
     for (int c = lane; c < n_chunks; c += 32) M = fmaxf(M, ml[2 * c]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float L = 0.f;
+    float L = 0.f, N = 0.f;
     float a[kDpl];
 #pragma unroll
     for (int e = 0; e < kDpl; ++e) a[e] = 0.f;
     for (int c = 0; c < n_chunks; ++c) {
         const float f = ex2(ml[2 * c] - M);
         L += f * ml[2 * c + 1];
+        if (p.nexus_mass != nullptr) N += f * p.part_nx[unit * p.max_chunks + c];
 #pragma unroll
         for (int e = 0; e < kDpl; ++e) a[e] += f * ac[(int64_t)c * D + lane * kDpl + e];
     }
@@ -913,6 +955,22 @@ decode_combine_kernel(const DecParams p, int n_layers) {
     for (int e = 0; e < kDpl; ++e)
         op[lane * kDpl + e] = __bfloat16_as_ushort(__float2bfloat16_rn(a[e] / L));
     if (lane == 0 && p.lse != nullptr) p.lse[unit] = (M + __log2f(L)) * kLn2;
+    if (lane == 0 && p.nexus_mass != nullptr) p.nexus_mass[unit] = N / L;
+}
+
+// Every output of a call with no key rows at all: O = 0, lse = -inf, mass 0.
+__global__ void decode_empty_kernel(uint16_t *O, int64_t o_ls, float *lse, float *nexus_mass,
+                                    int n_layers, int64_t per_layer_units, int D) {
+    const int64_t n = (int64_t)n_layers * per_layer_units;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n * D;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t unit = i / D, layer = unit / per_layer_units;
+        O[layer * o_ls + (unit - layer * per_layer_units) * D + (i - unit * D)] = 0;
+        if (i - unit * D == 0) {
+            if (lse != nullptr) lse[unit] = -INFINITY;
+            if (nexus_mass != nullptr) nexus_mass[unit] = 0.f;
+        }
+    }
 }
 
 int g_template(int G) {
@@ -927,7 +985,9 @@ int g_template(int G) {
 
 struct Plan {
     int chunk_len, max_chunks;
-    size_t ws_acc, ws_ml, ws_cnt;  // partial accumulators, partial (max, sum), unit counter
+    // partial accumulators, partial (max, sum), partial Nexus sums, unit counter
+    size_t ws_acc, ws_ml, ws_nx, ws_cnt;
+    size_t total() const { return ws_acc + ws_ml + ws_nx + ws_cnt; }
 };
 
 Plan make_plan(const sonic_decode_args *a) {
@@ -951,6 +1011,8 @@ Plan make_plan(const sonic_decode_args *a) {
     if (pl.max_chunks > 1) {
         pl.ws_acc = round_up(units_q * pl.max_chunks * a->head_dim * sizeof(float), 256);
         pl.ws_ml = round_up(units_q * pl.max_chunks * 2 * sizeof(float), 256);
+        if (a->nexus_mass != nullptr)
+            pl.ws_nx = round_up(units_q * pl.max_chunks * sizeof(float), 256);
     }
     if (a->head_dim == 128) pl.ws_cnt = 256;  // the persistent kernel's unit counter
     return pl;
@@ -1030,7 +1092,7 @@ extern "C" size_t sonic_decode_workspace_size(const sonic_decode_args *a) {
         a->head_dim < 1)
         return 0;
     Plan pl = make_plan(a);
-    return pl.ws_acc + pl.ws_ml + pl.ws_cnt;
+    return pl.total();
 }
 
 extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_ret,
@@ -1052,20 +1114,22 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const int GT = g_template(G);
     if (GT == 0) return SONIC_ERR_UNSUPPORTED;
     if (a->chunk_len < 0) return SONIC_ERR_INVALID_ARGUMENT;
+    if (a->nexus_mass != nullptr && a->role == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
     if (!aligned16(K_ret) || !aligned16(V_ret) || !aligned16(q) || (a->q_layer_stride * 2) % 16)
         return SONIC_ERR_INVALID_ARGUMENT;
     if (a->n_layers > 1 && (a->kv_layer_stride <= 0 || (a->kv_layer_stride * 2) % 16 != 0))
         return SONIC_ERR_INVALID_ARGUMENT;
     if (a->total_kv_rows == 0 || a->max_len == 0) {
-        // nothing to attend: every output is zero
-        for (int l = 0; l < a->n_layers; ++l)
-            if (cudaMemsetAsync(O + l * a->o_layer_stride, 0,
-                                (size_t)a->batch * a->n_heads_q * D * 2, stream) != cudaSuccess)
-                return SONIC_ERR_CUDA;
-        return SONIC_OK;
+        // nothing to attend: every output is zero (lse -inf)
+        const long long units = (long long)a->batch * a->n_heads_q;
+        const long long n = units * a->n_layers * D;
+        const unsigned blocks = (unsigned)(n / 256 + 1 < 4096 ? n / 256 + 1 : 4096);
+        decode_empty_kernel<<<blocks, 256, 0, stream>>>(O, a->o_layer_stride, a->lse,
+                                                       a->nexus_mass, a->n_layers, units, D);
+        return cudaGetLastError() == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
     }
     Plan pl = make_plan(a);
-    const size_t need = pl.ws_acc + pl.ws_ml + pl.ws_cnt;
+    const size_t need = pl.total();
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
     const long long units_x = (long long)pl.max_chunks * a->n_heads_kv;
@@ -1110,6 +1174,10 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     p.lse = a->lse;
     p.part_acc = static_cast<float *>(a->workspace);
     p.part_ml = reinterpret_cast<float *>(static_cast<char *>(a->workspace) + pl.ws_acc);
+    p.part_nx =
+        reinterpret_cast<float *>(static_cast<char *>(a->workspace) + pl.ws_acc + pl.ws_ml);
+    p.role = a->role;
+    p.nexus_mass = a->nexus_mass;
     p.status = a->status;
     p.B = a->batch;
     p.Hq = a->n_heads_q;
@@ -1123,7 +1191,8 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     p.scale_log2 = scale * kLog2e;
 
     dim3 grid((unsigned)units_x, a->batch * a->n_layers);
-    int *counter = reinterpret_cast<int *>(static_cast<char *>(a->workspace) + pl.ws_acc + pl.ws_ml);
+    int *counter = reinterpret_cast<int *>(static_cast<char *>(a->workspace) + pl.ws_acc +
+                                           pl.ws_ml + pl.ws_nx);
     cudaError_t e = (D == 128) ? dispatch_tc(GT, tm, p, (int)units_x,
                                              (int)(units_x * a->batch * a->n_layers), counter, stream)
                                : dispatch_g<64>(GT, tk, tv, p, grid, stream);

@@ -134,6 +134,7 @@ struct PfParams {
     const int32_t *key_pos;  // S_aug position of each key row; NULL: the row index
     uint16_t *O;
     float *lse;
+    float *nexus_mass;
     int32_t *status;
     const TileSum *sums;
     int max_k_tiles, max_k_len;
@@ -222,11 +223,13 @@ constexpr float kRescaleThreshold = 8.0f;
 // TMEM (512 columns): S/P of tile 0 at 0, of tile 1 at 128, O of tile 0 at
 // 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns
 // of its S block and feeds O += P V straight from tensor memory.
-template <int D, bool kLse>
+// kOut: bit 0 writes the log-sum-exp, bit 1 the attention mass on Nexus keys.
+template <int D, int kOut>
 __global__ void __launch_bounds__(kPfThreads, 1)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const PfParams p) {
     using C = PfCfg<D>;
+    constexpr bool kLse = kOut & 1, kMass = kOut & 2;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -286,7 +289,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     __syncthreads();
 
     // ------------------------------------------------ key tiles to visit
-    // list entry: (tile << 2) | (tile 0 needs the mask) | (tile 1 needs it) << 1
+    // list entry: (tile << 4) | (Nexus keys: 0 none, 1 all, 2 some) << 2
+    //             | (tile 0 needs the mask) | (tile 1 needs it) << 1
     const int n_kt = (kklen + kBN - 1) / kBN;
     int n_list = 0;
     for (int c0 = 0; c0 < n_kt; c0 += kPfThreads) {
@@ -297,6 +301,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
             const int k0 = ts.pos_min, k1 = ts.pos_max;  // S_aug positions of the keys
             const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
+            entry = (kn ? ((kb || ko) ? 2 : 1) : 0) << 2;
             for (int qi = 0; qi < 2; ++qi) {
                 const int p0 = pbase + qi * kBM;
                 const int p1 = min(p0 + kBM - 1, klen - 1);
@@ -327,7 +332,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int w = 0; w < warp; ++w) base += misc[16 + w];
         int tot = 0;
         for (int w = 0; w < kPfThreads / 32; ++w) tot += misc[16 + w];
-        if (keep) list[base + __popc(bal & ((1u << lane) - 1u))] = (t << 2) | entry;
+        if (keep) list[base + __popc(bal & ((1u << lane) - 1u))] = (t << 4) | entry;
         n_list += tot;
         __syncthreads();
     }
@@ -372,7 +377,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const int st = i & 1;
             if (i >= 2 && !mbar_wait(&kv_empty[st], ((i >> 1) - 1) & 1, p.status, abort_flag))
                 break;
-            const int kt = list[i] >> 2;
+            const int kt = list[i] >> 4;
             // K/V copies first; the key metadata is built while they are in flight
             if (lane == 0) {
                 mbar_expect_tx(&kv_full[st], 2 * C::kKVBytes);
@@ -389,6 +394,18 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // within each 32-key word; role 255 marks padding and rows past the
             // sequence) and their masks: needed only where a query tile is cut.
             if ((list[i] & 3) == 0) {
+                if (kMass && ((list[i] >> 2) & 3) == 2) {
+                    // an uncut tile with some Nexus keys: their bits only
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        const int q = kt * kBN + w * 32 + lane;
+                        const bool isn =
+                            q < kklen && p.key_role[kkstart + q] == SONIC_ROLE_NEXUS;
+                        const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
+                        if (lane == 0) tmasks[st].nx[w] = nxw;
+                    }
+                    __syncwarp();
+                }
                 mbar_arrive(&kv_full[st]);
                 continue;
             }
@@ -588,17 +605,22 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // l: sum of the rounded probabilities (normalises O); l_lse: of the
         // unrounded ones, for the log-sum-exp output (kLse: lse requested)
         float m_used = -INFINITY, l = 0.f, l_lse = 0.f;
+        // ln: the part of l on Nexus keys (kMass)
+        float ln = 0.f;
         bool ok = true;
         // the next list entry is read one tile ahead: shared memory is busy
         // feeding the tensor cores, so a load on the critical path is slow
         int entry = n_list > 0 ? list[0] : 0;
         for (int j = 0; j < n_list; ++j) {
             const int st = j & 1;
-            const int kt = entry >> 2;
+            const int kt = entry >> 4;
             const bool cut = (entry >> qi) & 1;
+            const int nexus_keys = (entry >> 2) & 3;
             entry = j + 1 < n_list ? list[j + 1] : 0;
-            // the keys' roles/segments are read (and V rows zeroed) on cut tiles only
-            if ((cut && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) ||
+            // the keys' roles/segments are read (and V rows zeroed) on cut tiles
+            // only, and their Nexus bits on tiles with some Nexus keys
+            const bool need_meta = cut || (kMass && nexus_keys == 2);
+            if ((need_meta && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) ||
                 !mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
                 ok = false;
                 break;
@@ -703,6 +725,19 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const float2 nm2 = make_float2(-mref, -mref);
             float ls[4] = {0.f, 0.f, 0.f, 0.f};
             float2 rs2x = make_float2(0.f, 0.f);
+            float lsn[2] = {0.f, 0.f};
+            uint32_t nxb[4] = {0u, 0u, 0u, 0u};
+            if (kMass) {
+                if (nexus_keys == 1) {
+                    nxb[0] = nxb[1] = nxb[2] = nxb[3] = 0xffffffffu;
+                } else if (nexus_keys == 2) {
+                    const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
+                    nxb[0] = nx.x;
+                    nxb[1] = nx.y;
+                    nxb[2] = nx.z;
+                    nxb[3] = nx.w;
+                }
+            }
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 uint32_t pk[16];
@@ -720,11 +755,15 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // to one (rounding moves weight between keys, it does not
                     // scale the output)
                     add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
+                    if (kMass)
+                        add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << e),
+                                             nxb[c] & (2u << e));
                 }
                 tmem_st16(tS + c * 16, pk);
             }
             l = l * alpha + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
             if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
+            if (kMass) ln = ln * alpha + (lsn[0] + lsn[1]);
             // O rescale (PV of the previous tile is complete: S of this tile was
             // issued after it, and S is done)
             if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
@@ -785,12 +824,15 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (kLse && row_ok)
                 p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] =
                     l_lse > 0.f ? (m_used + __log2f(l_lse)) * kLn2f : -INFINITY;
+            if (kMass && row_ok)
+                p.nexus_mass[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = ln * inv;
         } else if (row_ok && n_list == 0) {
             const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
             uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
             for (int d = 0; d < D; ++d) orow[d] = 0;
             if (kLse)
                 p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = -INFINITY;
+            if (kMass) p.nexus_mass[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = 0.f;
         }
     }
     tc_fence_before();
@@ -969,7 +1011,11 @@ cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const C
                            const PfParams &p, dim3 grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
-    auto kern = p.lse != nullptr ? prefill_kernel<D, true> : prefill_kernel<D, false>;
+    const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
+    auto kern = out == 0   ? prefill_kernel<D, 0>
+                : out == 1 ? prefill_kernel<D, 1>
+                : out == 2 ? prefill_kernel<D, 2>
+                           : prefill_kernel<D, 3>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -1114,6 +1160,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     }
     p.O = O;
     p.lse = a->lse;
+    p.nexus_mass = a->nexus_mass;
     p.status = a->status;
     p.sums = static_cast<const TileSum *>(a->workspace);
     p.max_k_tiles = max_k_tiles_of(a);

@@ -348,6 +348,19 @@ __device__ __forceinline__ void add_bf16x2_to_f32(float &a, float &b, uint32_t p
         : "r"(pair));
 }
 
+// The same, each half added only where its selector is nonzero.
+__device__ __forceinline__ void add_bf16x2_to_f32_if(float &a, float &b, uint32_t pair,
+                                                     uint32_t sel_lo, uint32_t sel_hi) {
+    asm("{\n\t.reg .b16 lo, hi;\n\t.reg .pred pl, ph;\n\t"
+        "mov.b32 {lo, hi}, %2;\n\t"
+        "setp.ne.b32 pl, %3, 0;\n\t"
+        "setp.ne.b32 ph, %4, 0;\n\t"
+        "@pl add.rn.f32.bf16 %0, lo, %0;\n\t"
+        "@ph add.rn.f32.bf16 %1, hi, %1;\n\t}"
+        : "+f"(a), "+f"(b)
+        : "r"(pair), "r"(sel_lo), "r"(sel_hi));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     uint32_t u;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(u) : "f"(hi), "f"(lo));

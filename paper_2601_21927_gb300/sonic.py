@@ -56,7 +56,7 @@ class sonic_prefill_args(ctypes.Structure):
                 ("total_k_rows", _i32), ("q_layer_stride", _i64), ("kv_layer_stride", _i64),
                 ("o_layer_stride", _i64), ("softmax_scale", _f32), ("nexus_vis", _i32),
                 ("lse", _P), ("status", _P), ("workspace", _P), ("workspace_bytes", _sz),
-                ("key_order", _i32)]
+                ("key_order", _i32), ("nexus_mass", _P)]
 
 
 class sonic_decode_args(ctypes.Structure):
@@ -64,7 +64,7 @@ class sonic_decode_args(ctypes.Structure):
                 ("head_dim", _i32), ("kv_start", _P), ("max_len", _i32), ("total_kv_rows", _i32),
                 ("q_layer_stride", _i64), ("kv_layer_stride", _i64), ("o_layer_stride", _i64),
                 ("softmax_scale", _f32), ("chunk_len", _i32), ("lse", _P), ("status", _P),
-                ("workspace", _P), ("workspace_bytes", _sz)]
+                ("workspace", _P), ("workspace_bytes", _sz), ("role", _P), ("nexus_mass", _P)]
 
 
 # Exported C symbols, with their ctypes signatures.
@@ -179,8 +179,9 @@ def sonic_attn_prefill(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, seg_id
                        role: torch.Tensor, O: torch.Tensor, *, k_start, k_len, q_start, q_len,
                        max_q_len: int, max_k_len: int, softmax_scale: float = 0.0,
                        nexus_vis: int = NEXUS_FULL, lse=None, status=None, workspace=None,
-                       key_order: int = KEYS_AS_GIVEN, stream=None):
-    """Masked prefill.  Q, O: [n_layers, Tq, Hq, D] bf16; K, V: [n_layers, Tk, Hkv, D] bf16."""
+                       key_order: int = KEYS_AS_GIVEN, nexus_mass=None, stream=None):
+    """Masked prefill.  Q, O: [n_layers, Tq, Hq, D] bf16; K, V: [n_layers, Tk, Hkv, D] bf16;
+    lse, nexus_mass: [n_layers, Tq, Hq] float32 or None."""
     lib = load()
     nl, tq, hq, d = Q.shape
     _, tk, hkv, _ = K.shape
@@ -194,6 +195,7 @@ def sonic_attn_prefill(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, seg_id
     a.softmax_scale, a.nexus_vis = softmax_scale, nexus_vis
     a.lse, a.status = _ptr(lse), _ptr(status)
     a.key_order = key_order
+    a.nexus_mass = _ptr(nexus_mass)
     need = lib.sonic_prefill_workspace_size(ctypes.byref(a))
     ws = _workspace(need, Q.device, workspace)
     a.workspace, a.workspace_bytes = _ptr(ws), need
@@ -205,8 +207,9 @@ def sonic_attn_prefill(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, seg_id
 def sonic_attn_decode(q: torch.Tensor, K_ret: torch.Tensor, V_ret: torch.Tensor,
                       lens: torch.Tensor, O: torch.Tensor, *, kv_start, max_len: int,
                       softmax_scale: float = 0.0, chunk_len: int = 0, lse=None, status=None,
-                      workspace=None, stream=None):
-    """One decode step.  q, O: [n_layers, B, Hq, D]; K_ret, V_ret: [n_layers, T, Hkv, D]."""
+                      workspace=None, role=None, nexus_mass=None, stream=None):
+    """One decode step.  q, O: [n_layers, B, Hq, D]; K_ret, V_ret: [n_layers, T, Hkv, D];
+    lse, nexus_mass: [n_layers, B, Hq] float32 or None; role: [T] uint8 (with nexus_mass)."""
     lib = load()
     nl, B, hq, d = q.shape
     _, T, hkv, _ = K_ret.shape
@@ -216,6 +219,7 @@ def sonic_attn_decode(q: torch.Tensor, K_ret: torch.Tensor, V_ret: torch.Tensor,
     a.q_layer_stride, a.kv_layer_stride, a.o_layer_stride = q.stride(0), K_ret.stride(0), O.stride(0)
     a.softmax_scale, a.chunk_len = softmax_scale, chunk_len
     a.lse, a.status = _ptr(lse), _ptr(status)
+    a.role, a.nexus_mass = _ptr(role), _ptr(nexus_mass)
     need = lib.sonic_decode_workspace_size(ctypes.byref(a))
     ws = _workspace(need, q.device, workspace)
     a.workspace, a.workspace_bytes = _ptr(ws), need
@@ -228,7 +232,7 @@ def sonic_attn_prefill_static(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor,
                               seg_id: torch.Tensor, role: torch.Tensor, O: torch.Tensor, *,
                               k_start, k_len, q_start, q_len, max_q_len: int, max_k_len: int,
                               softmax_scale: float = 0.0, nexus_vis: int = NEXUS_FULL, lse=None,
-                              status=None, stream=None):
+                              status=None, nexus_mass=None, stream=None):
     """sonic_attn_prefill for callers that cannot allocate device memory: the
     library keeps the mask-summary scratch in a fixed 1 MiB device array, so
     no workspace is passed (and this wrapper allocates nothing either).
@@ -245,6 +249,7 @@ def sonic_attn_prefill_static(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor,
     a.q_layer_stride, a.kv_layer_stride, a.o_layer_stride = Q.stride(0), K.stride(0), O.stride(0)
     a.softmax_scale, a.nexus_vis = softmax_scale, nexus_vis
     a.lse, a.status = _ptr(lse), _ptr(status)
+    a.nexus_mass = _ptr(nexus_mass)
     _check(lib.sonic_attn_prefill_static(_ptr(Q), _ptr(K), _ptr(V), _ptr(seg_id), _ptr(role),
                                          _ptr(O), ctypes.byref(a), _stream(stream)),
            "sonic_attn_prefill_static")

@@ -44,7 +44,8 @@ def check_close(got: np.ndarray, want: np.ndarray, what: str):
 def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed: int = 0,
                 nexus_vis: int = sonic.NEXUS_FULL, n_layers: int = 1, with_lse: bool = True,
                 K=None, V=None, Q=None, key_order: int = sonic.KEYS_AS_GIVEN,
-                expect_status: int = 0, k_start=None, total_k_rows=None):
+                expect_status: int = 0, k_start=None, total_k_rows=None,
+                with_mass: bool = False):
     """Prefill of the last q_len[b] rows of every sequence (all rows if None).
     Returns a dict with the device tensors and the query layout."""
     role, seg, k_start_b, k_len = meta(batch)
@@ -62,14 +63,16 @@ def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed
         Q = inputs.randn((n_layers, Tq, hq, D), seed=seed + 3, device=dev())
     O = torch.full_like(Q, float("nan"))
     lse = torch.full((n_layers, Tq, hq), float("nan"), device=dev()) if with_lse else None
+    mass = torch.full((n_layers, Tq, hq), float("nan"), device=dev()) if with_mass else None
     status = torch.zeros(1, dtype=torch.int32, device=dev())
     sonic.sonic_attn_prefill(Q, K, V, seg, role, O, k_start=k_start, k_len=k_len,
                              q_start=i32(q_start), q_len=i32(q_len),
                              max_q_len=int(q_len.max()), max_k_len=int(batch.k_len.max()),
-                             nexus_vis=nexus_vis, lse=lse, status=status, key_order=key_order)
+                             nexus_vis=nexus_vis, lse=lse, status=status, key_order=key_order,
+                             nexus_mass=mass)
     torch.cuda.synchronize()
     assert sonic.read_status(status) == expect_status
-    return dict(K=K, V=V, Q=Q, O=O, lse=lse, q_len=q_len, q_start=q_start)
+    return dict(K=K, V=V, Q=Q, O=O, lse=lse, mass=mass, q_len=q_len, q_start=q_start)
 
 
 def oracle_prefill_rows(batch: inputs.Batch, res: dict, b: int, rows, layer: int = 0,
@@ -87,3 +90,17 @@ def oracle_prefill_rows(batch: inputs.Batch, res: dict, b: int, rows, layer: int
                                 nexus_mode=nexus_vis)
     return O, lse, f64(res["O"][layer, qs + rows]), (
         None if res["lse"] is None else f64(res["lse"][layer, qs + rows]))
+
+
+def oracle_mass_rows(batch: inputs.Batch, res: dict, b: int, rows, layer: int = 0,
+                     nexus_vis: int = oracle.NEXUS_FULL):
+    """Oracle attention mass on Nexus keys for query rows `rows` of sequence
+    b, and the GPU's."""
+    ks, kl = int(batch.k_start[b]), int(batch.k_len[b])
+    ql, qs = int(res["q_len"][b]), int(res["q_start"][b])
+    rows = np.asarray(rows, dtype=np.int64)
+    K = f64(res["K"][layer, ks:ks + kl])
+    Q = f64(res["Q"][layer, qs + rows])
+    want = oracle.nexus_mass(Q, K, batch.role[ks:ks + kl], batch.seg[ks:ks + kl], kl - ql + rows,
+                             nexus_mode=nexus_vis)
+    return want, f64(res["mass"][layer, qs + rows])

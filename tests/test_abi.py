@@ -26,7 +26,7 @@ def test_library_exports_every_declared_symbol():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(sonic.SIGNATURES)
-    assert lib.sonic_abi_version() == 1
+    assert lib.sonic_abi_version() == 2
     assert lib.sonic_status_string(4) == b"output capacity exceeded"
 
 

@@ -77,6 +77,55 @@ def test_uniform_scores_count_visible_keys(mode, order):
         H.check_close(got, O, f"seq {b}")
 
 
+MASS_ATOL = 2e-3  # attention mass on Nexus keys: a share in [0, 1]
+
+
+@pytest.mark.parametrize("order", ORDERS)
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+@pytest.mark.parametrize("D,hq,hkv,with_lse", [(128, 4, 2, True), (64, 6, 2, False)])
+def test_nexus_mass_matches_oracle(order, mode, D, hq, hkv, with_lse):
+    """The mass output on every row: random dialogues spanning several tiles,
+    a retained cache followed by a current turn (uncut tiles that mix system,
+    Nexus and current keys), and short segments (tiles on the per-key path).
+    O and lse do not change when the mass is requested."""
+    rng = np.random.default_rng(37)
+    ds = [inputs.random_dialogue(rng, max_segments=6, max_body=150, max_nexus=40, max_sys=90,
+                                 max_curr=150) for _ in range(3)]
+    ds += [inputs.Dialogue(200, [(0, 60), (0, 90), (0, 7)], 400),
+           inputs.Dialogue(30, [(20, 5)] * 30, 100)]
+    batch = inputs.Batch(ds)
+    res = H.run_prefill(batch, hq, hkv, D, seed=41, nexus_vis=mode, key_order=order,
+                        with_lse=with_lse, with_mass=True)
+    for b in range(batch.B):
+        n = int(batch.k_len[b])
+        want, got = H.oracle_mass_rows(batch, res, b, np.arange(n), nexus_vis=mode)
+        np.testing.assert_allclose(got, want, rtol=0, atol=MASS_ATOL, err_msg=f"seq {b}")
+    plain = H.run_prefill(batch, hq, hkv, D, seed=41, nexus_vis=mode, key_order=order,
+                          with_lse=with_lse)
+    assert torch.equal(plain["O"].view(torch.int16), res["O"].view(torch.int16))
+    if with_lse:
+        assert torch.equal(plain["lse"], res["lse"])
+
+
+@pytest.mark.parametrize("order", ORDERS)
+def test_nexus_mass_of_uniform_scores_is_the_visible_nexus_share(order):
+    """Q = 0: every visible probability is exactly 1, so the mass is the count
+    of visible Nexus keys over the count of visible keys, up to one fp32
+    division: a key-exact check of the Nexus bits on every tile kind."""
+    rng = np.random.default_rng(43)
+    ds = [inputs.random_dialogue(rng, max_segments=6, max_body=150, max_nexus=40, max_sys=90,
+                                 max_curr=150) for _ in range(3)]
+    ds += [inputs.Dialogue(200, [(0, 60), (0, 90), (0, 7)], 400),
+           inputs.Dialogue(30, [(20, 5)] * 30, 100), inputs.Dialogue(9, [(300, 0)], 40)]
+    batch = inputs.Batch(ds)
+    Q = torch.zeros((1, batch.total, 4, 128), dtype=torch.bfloat16, device=H.dev())
+    res = H.run_prefill(batch, 4, 2, 128, seed=47, key_order=order, Q=Q, with_mass=True)
+    for b in range(batch.B):
+        n = int(batch.k_len[b])
+        want, got = H.oracle_mass_rows(batch, res, b, np.arange(n))
+        np.testing.assert_allclose(got, want, rtol=0, atol=1e-6, err_msg=f"seq {b}")
+
+
 def test_retained_first_sequences_sharing_key_rows():
     """Two sequences over the same key rows (a shared history, different query
     blocks): each gets its own span of the permuted copy.  The key tensor has
