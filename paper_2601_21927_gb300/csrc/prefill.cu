@@ -725,18 +725,17 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const float2 nm2 = make_float2(-mref, -mref);
             float ls[4] = {0.f, 0.f, 0.f, 0.f};
             float2 rs2x = make_float2(0.f, 0.f);
+            // the Nexus part of the row sum: all of it, none, or (some Nexus
+            // keys) the keys the tile's Nexus bits select
             float lsn[2] = {0.f, 0.f};
             uint32_t nxb[4] = {0u, 0u, 0u, 0u};
-            if (kMass) {
-                if (nexus_keys == 1) {
-                    nxb[0] = nxb[1] = nxb[2] = nxb[3] = 0xffffffffu;
-                } else if (nexus_keys == 2) {
-                    const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
-                    nxb[0] = nx.x;
-                    nxb[1] = nx.y;
-                    nxb[2] = nx.z;
-                    nxb[3] = nx.w;
-                }
+            const bool some_nexus = kMass && nexus_keys == 2;
+            if (some_nexus) {
+                const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
+                nxb[0] = nx.x;
+                nxb[1] = nx.y;
+                nxb[2] = nx.z;
+                nxb[3] = nx.w;
             }
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
@@ -755,15 +754,20 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // to one (rounding moves weight between keys, it does not
                     // scale the output)
                     add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
-                    if (kMass)
-                        add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << e),
+                }
+                if (some_nexus) {
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2)
+                        add_bf16x2_to_f32_if(lsn[0], lsn[1], pk[e >> 1], nxb[c] & (1u << e),
                                              nxb[c] & (2u << e));
                 }
                 tmem_st16(tS + c * 16, pk);
             }
-            l = l * alpha + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+            const float l_tile = (ls[0] + ls[1]) + (ls[2] + ls[3]);
+            l = l * alpha + l_tile;
             if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
-            if (kMass) ln = ln * alpha + (lsn[0] + lsn[1]);
+            if (kMass)
+                ln = ln * alpha + (nexus_keys == 1 ? l_tile : (lsn[0] + lsn[1]));
             // O rescale (PV of the previous tile is complete: S of this tile was
             // issued after it, and S is done)
             if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
