@@ -17,6 +17,7 @@ builds that file with gcc and marshals numpy arrays into it:
 * :func:`nexus_mass`    -- attention mass on Nexus keys per query row and head
                            (the quantity behind A_nexus, Sec. 4.1 Eq. 9).
 * :func:`decode_nexus_mass` -- the same for one decode step.
+* :func:`routed_linear` -- linear map with the Nexus rows' own weights (Sec. 3.1).
 """
 from __future__ import annotations
 
@@ -81,6 +82,8 @@ class Oracle:
         lib.orc_nexus_mass.restype = None
         lib.orc_decode_nexus_mass.argtypes = [i64, i32, i32, i32, P, P, P, f64, P, P]
         lib.orc_decode_nexus_mass.restype = None
+        lib.orc_routed_linear.argtypes = [i64, i32, i32, P, P, P, P, P]
+        lib.orc_routed_linear.restype = None
         self.lib = lib
         self.path = so_path
 
@@ -214,6 +217,21 @@ class Oracle:
                                        float(scale), _ptr(s_buf), _ptr(mass))
         return mass
 
+    def routed_linear(self, X, W, W_nexus, role):
+        """Y [T, d_out] = X @ W.T on rows whose role is not NEXUS, X @ W_nexus.T on
+        Nexus rows.  X: [T, d_in]; W, W_nexus: [d_out, d_in]."""
+        X = _c(X, np.float64)
+        W = _c(W, np.float64)
+        W_nexus = _c(W_nexus, np.float64)
+        role = _c(role, np.uint8)
+        T, d_in = X.shape
+        d_out = W.shape[0]
+        assert W.shape == (d_out, d_in) and W_nexus.shape == (d_out, d_in)
+        Y = np.zeros((T, d_out), np.float64)
+        self.lib.orc_routed_linear(T, d_in, d_out, _ptr(X), _ptr(W), _ptr(W_nexus), _ptr(role),
+                                   _ptr(Y))
+        return Y
+
 
 def _ptr(a):
     return None if a is None else a.ctypes.data
@@ -262,3 +280,7 @@ def nexus_mass(*a, **k):
 
 def decode_nexus_mass(*a, **k):
     return default().decode_nexus_mass(*a, **k)
+
+
+def routed_linear(*a, **k):
+    return default().routed_linear(*a, **k)

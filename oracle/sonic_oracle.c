@@ -337,3 +337,29 @@ void orc_decode_nexus_mass(int64_t n, int32_t Hq, int32_t Hkv, int32_t D,
         mass[h] = all > 0.0 ? nexus / all : 0.0;
     }
 }
+
+/*
+ * Role-routed linear map (Sec. 3.1, "Nexus Insertion and Representation":
+ * Nexus tokens get dedicated projection matrices W_Q^N, W_K^N, W_V^N, W_O^N,
+ * every other token the model's own):
+ *   Y[t][n] = sum_k X[t][k] * Wsel(t)[n][k],
+ *   Wsel(t) = W_nexus if role[t] is NEXUS, W otherwise.
+ * X is [T][d_in]; W and W_nexus are [d_out][d_in] (the out x in layout of a
+ * linear layer); Y is [T][d_out].
+ */
+void orc_routed_linear(int64_t T, int32_t d_in, int32_t d_out, const double *X,
+                       const double *W, const double *W_nexus, const uint8_t *role,
+                       double *Y)
+{
+    for (int64_t t = 0; t < T; ++t) {
+        const double *w = role[t] == ORC_NEXUS ? W_nexus : W;
+        const double *x = X + t * (int64_t)d_in;
+        for (int32_t n = 0; n < d_out; ++n) {
+            const double *wn = w + (int64_t)n * d_in;
+            double acc = 0.0;
+            for (int32_t k = 0; k < d_in; ++k)
+                acc += x[k] * wn[k];
+            Y[t * (int64_t)d_out + n] = acc;
+        }
+    }
+}

@@ -333,6 +333,41 @@ def test_decode_nexus_mass_equals_sdpa_and_current_rows_of_prefill():
     assert (ORC().decode_nexus_mass(Q[-1], K[:0], role[:0]) == 0).all()
 
 
+# ------------------------------------------- role-routed projections (Sec. 3.1)
+
+def _routed_inputs(T, d_in, d_out, seed):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((T, d_in))
+    W = rng.standard_normal((d_out, d_in))
+    Wn = rng.standard_normal((d_out, d_in))
+    role = rng.choice([inputs.ROLE_SYS, inputs.ROLE_BODY, inputs.ROLE_NEXUS, inputs.ROLE_CURR],
+                      T).astype(np.uint8)
+    return X, W, Wn, role
+
+
+def test_routed_linear_equals_matmul_per_role():
+    """Nexus rows through W_nexus, all others through W: numpy matmuls of the
+    two row subsets (d_in != d_out, so a transposed weight fails)."""
+    X, W, Wn, role = _routed_inputs(37, 24, 40, seed=1)
+    Y = ORC().routed_linear(X, W, Wn, role)
+    nex = role == inputs.ROLE_NEXUS
+    np.testing.assert_allclose(Y[nex], X[nex] @ Wn.T, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(Y[~nex], X[~nex] @ W.T, rtol=1e-12, atol=1e-12)
+    assert nex.any() and (~nex).any()
+
+
+def test_routed_linear_special_cases():
+    X, W, Wn, role = _routed_inputs(20, 16, 8, seed=2)
+    # one weight for both roles: a plain linear layer
+    np.testing.assert_allclose(ORC().routed_linear(X, W, W, role), X @ W.T, rtol=1e-12,
+                               atol=1e-12)
+    # identity weights read the inputs back (d_in = d_out)
+    I = np.eye(16)
+    np.testing.assert_array_equal(ORC().routed_linear(X, I, 2 * I, role),
+                                  np.where((role == inputs.ROLE_NEXUS)[:, None], 2 * X, X))
+    assert ORC().routed_linear(X[:0], W, Wn, role[:0]).shape == (0, 8)
+
+
 # ------------------------------------------------------------ mutants
 
 _MUTANTS = {
@@ -355,6 +390,11 @@ _MUTANTS = {
                           "if (role[q] != ORC_BODY)\n                    nexus += w;"),
     # Nexus mass of a decode step over the current-turn rows instead
     "decode_mass_curr": ("if (role[t] == ORC_NEXUS)", "if (role[t] == ORC_CURR)"),
+    # role routing keyed on body rows instead of Nexus rows
+    "route_body": ("const double *w = role[t] == ORC_NEXUS ? W_nexus : W;",
+                   "const double *w = role[t] == ORC_BODY ? W_nexus : W;"),
+    # weight read transposed
+    "route_transposed": ("acc += x[k] * wn[k];", "acc += x[k] * w[(int64_t)k * d_out + n];"),
     # Nexus mass ignores the mask (every key's weight in the denominator)
     "mass_unmasked": ("            double all = 0.0, nexus = 0.0;\n            for (int64_t q = 0; q < L; ++q) {\n                if (s_buf[q] == -INFINITY)\n                    continue;",
                       "            double all = 0.0, nexus = 0.0;\n            for (int64_t q = 0; q < L; ++q) {\n                if (s_buf[q] == -INFINITY)\n                    s_buf[q] = m;"),
@@ -396,6 +436,11 @@ def _run_pins(orc):
     if not np.allclose(orc.decode_nexus_mass(q[0], K, role),
                        _sdpa_nexus_share(q, K, role, np.zeros((1, 40)))[0], rtol=0, atol=1e-12):
         failed.append("decode nexus mass")
+    X, W, Wn, role = _routed_inputs(23, 12, 20, seed=5)
+    Y = orc.routed_linear(X, W, Wn, role)
+    nex = role == inputs.ROLE_NEXUS
+    if not (np.allclose(Y[nex], X[nex] @ Wn.T) and np.allclose(Y[~nex], X[~nex] @ W.T)):
+        failed.append("routed linear")
     return failed
 
 
