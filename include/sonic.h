@@ -317,6 +317,55 @@ SONIC_API sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K_
 SONIC_API size_t sonic_decode_workspace_size(const sonic_decode_args *args);
 
 /* ------------------------------------------------------------------------- */
+/* Role-routed projections                                                   */
+/* ------------------------------------------------------------------------- */
+
+/* One output part: a range of `cols` consecutive columns of Y (the parts
+ * take Y's columns in order), written as bf16 rows of `base`. */
+typedef struct {
+    void *base;                  /* device bf16, 16-byte aligned                         */
+    int64_t row_stride;          /* elements between rows of base; multiple of 8, >= cols */
+    int32_t cols;                /* > 0, multiple of 32                                 */
+    int32_t scatter;             /* 0: row t of Y goes to row t; 1: to row dst_row[t]   */
+} sonic_out_part;
+
+typedef struct {
+    int32_t n_rows;              /* T >= 0 rows (tokens) of X                           */
+    int32_t d_in;                /* columns of X and of W: a multiple of 64             */
+    int32_t d_out;               /* rows of W = the parts' columns together; multiple of 32 */
+    int64_t x_row_stride;        /* elements between rows of X; multiple of 8, >= d_in  */
+    const int32_t *dst_row;      /* device [T] or NULL (required if a part scatters)    */
+    int32_t n_parts;             /* 1 .. 4                                              */
+    sonic_out_part parts[4];
+    int32_t *status;             /* device int32 or NULL                                */
+    void *workspace;             /* device, sonic_routed_linear_workspace_size() bytes  */
+    size_t workspace_bytes;
+} sonic_routed_linear_args;
+
+/*
+ * Role-routed linear map (Sec. 3.1: Nexus tokens have their own projection
+ * matrices W_Q^N, W_K^N, W_V^N, W_O^N):
+ *   Y[t, n] = sum_k X[t, k] * Wsel(t)[n, k],
+ *   Wsel(t) = W_nexus if role[t] == SONIC_ROLE_NEXUS, W otherwise,
+ * X [T][x_row_stride] bf16 (the first d_in columns used), W and W_nexus
+ * [d_out][d_in] bf16 contiguous (a linear layer's out x in layout; W_nexus
+ * may equal W), fp32 accumulation, Y rounded to bf16 (nearest even) and
+ * written part by part.  For a QKV projection the parts are Q (row t of the
+ * query buffer) and K and V (row dst_row[t] of this layer's K and V caches:
+ * the rows compaction reserved), so new tokens' keys and values land in the
+ * retained cache with no further copy.  Rows are grouped by role on the GPU
+ * (a stable partition, no host round trip) and the GEMM runs on the tensor
+ * cores; the workspace holds the grouped copy of X.  T = 0 does nothing.
+ */
+SONIC_API sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t *W,
+                                             const uint16_t *W_nexus, const uint8_t *role,
+                                             const sonic_routed_linear_args *args,
+                                             sonic_stream_t stream);
+
+/* Workspace bytes for sonic_routed_linear: about T * (d_in * 2 + 4) bytes. */
+SONIC_API size_t sonic_routed_linear_workspace_size(const sonic_routed_linear_args *args);
+
+/* ------------------------------------------------------------------------- */
 /* Status                                                                    */
 /* ------------------------------------------------------------------------- */
 

@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libsonic.so")
 
-SOURCES = ["api.cu", "compact.cu", "decode.cu", "prefill.cu", "prefill_static.cu"]
+SOURCES = ["api.cu", "compact.cu", "decode.cu", "prefill.cu", "prefill_static.cu", "routed.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler",
               "-fvisibility=hidden", "--expt-relaxed-constexpr", "-I" + INCLUDE, "-I" + CSRC]

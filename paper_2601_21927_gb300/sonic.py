@@ -67,6 +67,16 @@ class sonic_decode_args(ctypes.Structure):
                 ("workspace", _P), ("workspace_bytes", _sz), ("role", _P), ("nexus_mass", _P)]
 
 
+class sonic_out_part(ctypes.Structure):
+    _fields_ = [("base", _P), ("row_stride", _i64), ("cols", _i32), ("scatter", _i32)]
+
+
+class sonic_routed_linear_args(ctypes.Structure):
+    _fields_ = [("n_rows", _i32), ("d_in", _i32), ("d_out", _i32), ("x_row_stride", _i64),
+                ("dst_row", _P), ("n_parts", _i32), ("parts", sonic_out_part * 4),
+                ("status", _P), ("workspace", _P), ("workspace_bytes", _sz)]
+
+
 # Exported C symbols, with their ctypes signatures.
 SIGNATURES = {
     "sonic_compact_kv": (_i32, [_P, _P, _P, _P, _P, _P, _P,
@@ -80,6 +90,9 @@ SIGNATURES = {
     "sonic_attn_decode": (_i32, [_P, _P, _P, _P, _P,
                                  ctypes.POINTER(sonic_decode_args), _P]),
     "sonic_decode_workspace_size": (_sz, [ctypes.POINTER(sonic_decode_args)]),
+    "sonic_routed_linear": (_i32, [_P, _P, _P, _P, ctypes.POINTER(sonic_routed_linear_args),
+                                   _P]),
+    "sonic_routed_linear_workspace_size": (_sz, [ctypes.POINTER(sonic_routed_linear_args)]),
     "sonic_read_status": (_i32, [_P, _P]),
     "sonic_status_string": (ctypes.c_char_p, [_i32]),
     "sonic_abi_version": (_i32, []),
@@ -225,6 +238,35 @@ def sonic_attn_decode(q: torch.Tensor, K_ret: torch.Tensor, V_ret: torch.Tensor,
     a.workspace, a.workspace_bytes = _ptr(ws), need
     _check(lib.sonic_attn_decode(_ptr(q), _ptr(K_ret), _ptr(V_ret), _ptr(lens), _ptr(O),
                                  ctypes.byref(a), _stream(stream)), "sonic_attn_decode")
+    return ws
+
+
+def sonic_routed_linear(X: torch.Tensor, W: torch.Tensor, W_nexus: torch.Tensor,
+                        role: torch.Tensor, parts, *, dst_row=None, status=None, workspace=None,
+                        stream=None):
+    """Role-routed linear map.  X: [T, >= d_in] bf16 (row-contiguous); W, W_nexus:
+    [d_out, d_in] bf16; role: [T] uint8.  parts: list of (out, scatter) with out a
+    2-D bf16 tensor whose columns (out.shape[1]) take the next columns of Y and
+    whose rows are indexed by t (scatter False) or dst_row[t] (scatter True)."""
+    lib = load()
+    T = X.shape[0]
+    d_out, d_in = W.shape
+    a = sonic_routed_linear_args()
+    a.n_rows, a.d_in, a.d_out = T, d_in, d_out
+    a.x_row_stride = X.stride(0) if T > 0 else d_in
+    a.dst_row = _ptr(dst_row)
+    a.n_parts = len(parts)
+    for k, (out, scatter) in enumerate(parts):
+        a.parts[k].base = _ptr(out)
+        a.parts[k].row_stride = out.stride(0)
+        a.parts[k].cols = out.shape[1]
+        a.parts[k].scatter = 1 if scatter else 0
+    a.status = _ptr(status)
+    need = lib.sonic_routed_linear_workspace_size(ctypes.byref(a))
+    ws = _workspace(need, X.device, workspace)
+    a.workspace, a.workspace_bytes = _ptr(ws), need
+    _check(lib.sonic_routed_linear(_ptr(X), _ptr(W), _ptr(W_nexus), _ptr(role), ctypes.byref(a),
+                                   _stream(stream)), "sonic_routed_linear")
     return ws
 
 

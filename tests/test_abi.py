@@ -33,7 +33,9 @@ def test_library_exports_every_declared_symbol():
 def test_struct_layout_matches_c(tmp_path):
     structs = {"sonic_compact_args": sonic.sonic_compact_args,
                "sonic_prefill_args": sonic.sonic_prefill_args,
-               "sonic_decode_args": sonic.sonic_decode_args}
+               "sonic_decode_args": sonic.sonic_decode_args,
+               "sonic_out_part": sonic.sonic_out_part,
+               "sonic_routed_linear_args": sonic.sonic_routed_linear_args}
     src = ['#include <stdio.h>', '#include <stddef.h>', '#include "sonic.h"', 'int main(void){']
     for name, cls in structs.items():
         src.append(f'printf("{name} %zu\\n", sizeof({name}));')
@@ -135,3 +137,23 @@ def test_retained_first_workspace_size():
     p.total_k_rows = p.max_k_len
     p.k_start = p.k_len = p.q_start = p.q_len = 16
     assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 2
+
+
+def test_routed_linear_validation():
+    lib = sonic.load()
+    a = sonic.sonic_routed_linear_args()
+    assert lib.sonic_routed_linear(None, None, None, None, None, None) == 1
+    a.n_rows = 0
+    assert lib.sonic_routed_linear(None, None, None, None, ctypes.byref(a), None) == 0  # empty
+    a.n_rows, a.d_in, a.d_out, a.x_row_stride, a.n_parts = 10, 96, 64, 96, 1  # d_in % 64
+    a.parts[0].base, a.parts[0].row_stride, a.parts[0].cols = 16, 64, 64
+    assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
+    a.d_in = a.x_row_stride = 128
+    a.parts[0].cols = 48                      # parts must cover d_out in 32-column steps
+    assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
+    a.parts[0].cols = 64
+    a.parts[0].scatter = 1                    # scatter without dst_row
+    assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
+    a.parts[0].scatter = 0
+    assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 3  # no workspace
+    assert lib.sonic_routed_linear_workspace_size(ctypes.byref(a)) == 256 + 256 + 256 + 2560
