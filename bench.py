@@ -764,8 +764,70 @@ def extra_nexus_mass():
                         "attention mass on Nexus keys", "results": res}
 
 
+def extra_routed():
+    """Role-routed projections (Sec. 3.1): the QKV projection of a Nexus
+    generation segment step (8 x (256 body + 32 Nexus) rows, Llama-3-8B-like
+    4096 -> 4096 + 1024 + 1024, K/V into cache rows), the QKV and O
+    projections of the serving step's 12,146 prefill rows (Qwen2.5-7B-like
+    3584 -> 3584 + 512 + 512, and 3584 -> 3584), with half of those rows
+    marked Nexus in runs of 32.  Beside each: cuBLAS (torch.matmul) on the
+    two role groups plus the row scatter, as context."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    bf = torch.bfloat16
+    res = {}
+    nexus_gen = np.tile(np.r_[np.full(256, 1), np.full(32, 2)], 8).astype(np.uint8)
+    serving = np.repeat(np.tile(np.array([3, 2], np.uint8), 12146 // 64 + 1), 32)[:12146]
+    cases = {
+        "nexus_gen_qkv_T2304_4096x6144": (nexus_gen, 4096, [4096, 1024, 1024], [0, 1, 1]),
+        "serving_qkv_T12146_3584x4608": (serving, 3584, [3584, 512, 512], [0, 1, 1]),
+        "serving_o_T12146_3584x3584": (serving, 3584, [3584], [0]),
+    }
+    for name, (role, d_in, cols, scat) in cases.items():
+        T, d_out = len(role), sum(cols)
+        X = inputs.randn((T, d_in), seed=1, device=dev)
+        W = inputs.randn((d_out, d_in), seed=2, device=dev)
+        Wn = inputs.randn((d_out, d_in), seed=3, device=dev)
+        role_t = torch.as_tensor(role).to(dev)
+        cache_rows = 2 * T
+        dst = torch.as_tensor(np.random.default_rng(0).permutation(cache_rows)[:T].astype(
+            np.int32)).to(dev)
+        outs = [torch.empty((cache_rows if s else T, c), dtype=bf, device=dev)
+                for c, s in zip(cols, scat)]
+        parts = list(zip(outs, [bool(s) for s in scat]))
+        ws = sonic.sonic_routed_linear(X, W, Wn, role_t, parts, dst_row=dst)
+        ms = _ev_time(lambda: sonic.sonic_routed_linear(X, W, Wn, role_t, parts, dst_row=dst,
+                                                        workspace=ws), reps=10, warm=3)
+        nex = torch.as_tensor(np.nonzero(role == 2)[0]).to(dev)
+        oth = torch.as_tensor(np.nonzero(role != 2)[0]).to(dev)
+        dstl = dst.long()
+
+        def cublas():
+            y = torch.empty((T, d_out), dtype=bf, device=dev)
+            y[oth] = X[oth] @ W.T
+            y[nex] = X[nex] @ Wn.T
+            c0 = 0
+            for out, s in zip(outs, scat):
+                if s:
+                    out[dstl] = y[:, c0:c0 + out.shape[1]]
+                else:
+                    out.copy_(y[:, c0:c0 + out.shape[1]])
+                c0 += out.shape[1]
+        ms_ref = _ev_time(cublas, reps=10, warm=3)
+        ms_mm = _ev_time(lambda: torch.matmul(X, W.T), reps=10, warm=3)
+        fl = 2.0 * T * d_in * d_out
+        res[name] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
+                     "cublas_grouped_scatter_ms": round(ms_ref, 4),
+                     "cublas_one_matmul_ms": round(ms_mm, 4),
+                     "cublas_one_matmul_tflops": round(fl / ms_mm / 1e9, 1)}
+        del X, W, Wn, outs, ws
+        torch.cuda.empty_cache()
+    return {"workload": "role-routed QKV / O projections (bf16, fp32 accumulate)", "results": res}
+
+
 EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
-          "nexus_mass": extra_nexus_mass,
+          "nexus_mass": extra_nexus_mass, "routed": extra_routed,
           "context": extra_context, "nexus_gen": extra_nexus_gen}
 
 

@@ -10,10 +10,10 @@
 //                 (perm[g] = source row of grouped row g) and the two group
 //                 sizes;
 //   row_gather    the rows of X in grouped order (warp per row, 16-byte loads);
-//   routed_gemm   a persistent tcgen05 GEMM over 128 x 256 output tiles of the
-//                 grouped rows.  A tile never straddles the two groups, so each
-//                 tile reads one weight matrix; the epilogue writes bf16 rows
-//                 to the parts.
+//   routed_gemm   a persistent tcgen05 GEMM on CTA pairs over 256 x 256
+//                 output tiles of the grouped rows.  A tile never straddles
+//                 the two groups, so each tile reads one weight matrix; the
+//                 epilogue writes bf16 rows to the parts.
 #include "sonic_dev.cuh"
 #include "sonic_host.h"
 
@@ -21,11 +21,13 @@ namespace sonic {
 namespace {
 
 constexpr int kChunkRows = 1024;  // rows per block of the partition kernels
-constexpr int kGBM = 128;         // output tile rows (grouped rows)
+constexpr int kGBM = 256;         // output tile rows (grouped rows) of a CTA pair
+constexpr int kHalfM = 128;       // of them in each CTA
 constexpr int kGBN = 256;         // output tile columns
+constexpr int kHalfN = 128;       // weight rows each CTA stages
 constexpr int kGBK = 64;          // reduction step (one 128-byte swizzle row)
-constexpr int kGStages = 4;
-constexpr int kGThreads = 192;    // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kGStages = 6;
+constexpr int kGThreads = 192;    // warp 0 TMA, warp 1 MMA (leader), warps 2-5 epilogue
 constexpr int kMaxParts = 4;
 
 // ------------------------------------------------------------- partition
@@ -126,6 +128,15 @@ row_gather_kernel(const uint8_t *__restrict__ X, int64_t x_row_bytes, int32_t T,
 }
 
 // ------------------------------------------------------------- GEMM
+//
+// The GEMM runs on CTA pairs (clusters of two) with the 2-SM form of the
+// tensor-core MMA: a pair computes a 256 x 256 output tile, each CTA holding
+// 128 rows of A and 128 of the tile's 256 weight rows, and the even CTA
+// issues MMAs that read both CTAs' shared memory and write 128 accumulator
+// rows into each CTA's tensor memory.  The 1-SM form with a 128 x 256 tile
+// reads 96 B/clk of operands from shared memory while the TMA writes another
+// 96 B/clk into it, more than shared memory delivers; the pair form halves
+// the B traffic per SM.
 
 struct GemmPart {
     uint16_t *base;
@@ -145,8 +156,8 @@ struct GemmParams {
 };
 
 struct GemmCfg {
-    static constexpr int kABytes = kGBM * kGBK * 2;  // 16 KB
-    static constexpr int kBBytes = kGBN * kGBK * 2;  // 32 KB
+    static constexpr int kABytes = kHalfM * kGBK * 2;  // 16 KB: this CTA's 128 rows of A
+    static constexpr int kBBytes = kHalfN * kGBK * 2;  // 16 KB: its 128 weight rows
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kOffBar = kGStages * kStageBytes;
     static constexpr int kNumBars = 2 * kGStages + 5;
@@ -155,8 +166,8 @@ struct GemmCfg {
 };
 
 // Tile i of the schedule: its grouped-row start, its valid-row end, its
-// column tile and its weight matrix.  m runs fastest, so the blocks working
-// at one time share the B (weight) tiles of one column tile.
+// column tile and its weight matrix.  m runs fastest, so the pairs working
+// at one time share the weight tiles of one column tile.
 struct GemmTile {
     int row0, row_end, n, g;
 };
@@ -177,7 +188,81 @@ __device__ __forceinline__ GemmTile gemm_tile(int i, int n0, int n1, int mt0, in
     return w;
 }
 
-__global__ void __launch_bounds__(kGThreads, 1)
+// ---- CTA-pair primitives (clusters of two CTAs; rank 0 leads)
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Address of the same shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t smem_in_rank(const void *p, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+    return a;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+                 : "memory");
+}
+
+// TMA load into this CTA's shared memory, completion counted on an mbarrier
+// of either CTA of the pair: in the pair form, bit 24 of the barrier's
+// shared-memory address selects the CTA, so the leader's barrier at the same
+// offset is the address with that bit cleared.
+__device__ __forceinline__ void tma_load_pair(void *dst, const CUtensorMap *map, uint32_t bar,
+                                              int32_t c0, int32_t c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(0), "r"(0)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(dst_smem)),
+                 "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mma_pair_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive once on the mbarrier at `bar`'s offset in every CTA of `mask` when
+// the pair MMAs this thread issued so far are complete.
+__device__ __forceinline__ void commit_pair(uint64_t *bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(smem_u32(bar)),
+        "h"(mask)
+        : "memory");
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
 routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                    const __grid_constant__ CUtensorMap tmWn, const GemmParams p) {
     using C = GemmCfg;
@@ -185,20 +270,22 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
-    uint64_t *full = bars;                    // [stages] A and B tiles landed
-    uint64_t *empty = bars + kGStages;        // [stages] their MMAs are done
-    uint64_t *acc_full = bars + 2 * kGStages; // [2] accumulator complete
-    uint64_t *acc_empty = acc_full + 2;       // [2] accumulator read out (128 threads)
+    uint64_t *full = bars;                     // [stages] both CTAs' tiles landed (leader)
+    uint64_t *empty = bars + kGStages;         // [stages] the MMAs reading them are done
+    uint64_t *acc_full = bars + 2 * kGStages;  // [2] accumulator complete
+    uint64_t *acc_empty = acc_full + 2;        // [2] read out by both CTAs (leader, 256)
     uint64_t *mma_idle = acc_empty + 2;
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    if (timed_out(p.status)) return;
+    const uint32_t rank = cluster_rank();
+    const int cid = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+    // no early return: both CTAs of the pair must reach the cluster barriers
     const int n0 = p.groups[0], n1 = p.groups[1];
     const int mt0 = (n0 + kGBM - 1) / kGBM, mt1 = (n1 + kGBM - 1) / kGBM;
     const int total_m = mt0 + mt1;
-    const int n_tiles = total_m * p.n_tiles_n;
+    const int n_tiles = timed_out(p.status) ? 0 : total_m * p.n_tiles_n;
     const int nk = p.d_in / kGBK;
 
     if (tid == 0) {
@@ -208,30 +295,33 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], 128);
+            mbar_init(&acc_empty[b], 2 * 128);
         }
         mbar_init(mma_idle, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 512);
-        tmem_relinquish();
+        tmem_alloc_pair(reinterpret_cast<uint32_t *>(&misc[0]), 512);
+        tmem_relinquish_pair();
     }
     tc_fence_before();
-    __syncthreads();
+    cluster_sync_all();  // both CTAs' barriers and tensor memory are set up
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
 
     if (warp == 0) {
-        // ------------------------------------------------------------ producer
+        // ------------------------------------------------------------ producers
+        // Each CTA loads its 128 rows of A and its 128 weight rows; both
+        // count on the leader's `full` barrier, which the leader arms with
+        // the pair's bytes.
         if (lane == 0) {
             tma_prefetch_desc(&tmA);
             tma_prefetch_desc(&tmW);
             tma_prefetch_desc(&tmWn);
             int it = 0;
             bool ok = true;
-            for (int i = blockIdx.x; ok && i < n_tiles; i += gridDim.x) {
+            for (int i = cid; ok && i < n_tiles; i += n_clusters) {
                 const GemmTile w = gemm_tile(i, n0, n1, mt0, total_m);
                 const CUtensorMap *tb = w.g ? &tmWn : &tmW;
                 for (int kb = 0; kb < nk; ++kb, ++it) {
@@ -242,25 +332,27 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                         break;
                     }
                     uint8_t *a = smem + s * C::kStageBytes;
-                    mbar_arrive_expect_tx(&full[s], C::kStageBytes);
-                    tma_load_4d(a, &tmA, &full[s], kb * kGBK, w.row0, 0, 0);
-                    tma_load_4d(a + C::kABytes, tb, &full[s], kb * kGBK, w.n * kGBN, 0, 0);
+                    if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * C::kStageBytes);
+                    const uint32_t bar = smem_u32(&full[s]) & 0xFEFFFFFFu;
+                    tma_load_pair(a, &tmA, bar, kb * kGBK, w.row0 + (int)rank * kHalfM);
+                    tma_load_pair(a + C::kABytes, tb, bar, kb * kGBK,
+                                  w.n * kGBN + (int)rank * kHalfN);
                 }
             }
-            if (*abort_flag) {
-                // let the copies already issued land before the block exits
+            if (*abort_flag && rank == 0) {
+                // let the copies already issued land before the pair exits
                 for (int u = max(0, it - kGStages); u < it; ++u)
                     mbar_wait(&full[u % kGStages], (u / kGStages) & 1, p.status, abort_flag);
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        // ------------------------------------------------------------ MMA issuer (leader)
+        if (lane == 0 && rank == 0) {
             constexpr uint32_t idesc = idesc_bf16_f32(kGBM, kGBN, 0, 0);
             const uint32_t base = smem_u32(smem);
             int it = 0, j = 0;
             bool ok = true;
-            for (int i = blockIdx.x; ok && i < n_tiles; i += gridDim.x, ++j) {
+            for (int i = cid; ok && i < n_tiles; i += n_clusters, ++j) {
                 const int b = j & 1;
                 if (j >= 2 && !mbar_wait(&acc_empty[b], ((j >> 1) - 1) & 1, p.status, abort_flag))
                     break;
@@ -277,26 +369,26 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     const uint32_t b_addr = a_addr + C::kABytes;
 #pragma unroll
                     for (int kk = 0; kk < kGBK / 16; ++kk)
-                        tc_mma_ss(acc, smem_desc_sw128(a_addr + kk * 32, 16, 1024),
-                                  smem_desc_sw128(b_addr + kk * 32, 16, 1024), idesc,
-                                  (kb > 0 || kk > 0) ? 1u : 0u);
-                    tc_commit(&empty[s]);
+                        mma_pair_ss(acc, smem_desc_sw128(a_addr + kk * 32, 16, 1024),
+                                    smem_desc_sw128(b_addr + kk * 32, 16, 1024), idesc,
+                                    (kb > 0 || kk > 0) ? 1u : 0u);
+                    commit_pair(&empty[s], 3);  // frees the stage in both CTAs
                 }
-                if (ok) tc_commit(&acc_full[b]);
+                if (ok) commit_pair(&acc_full[b], 3);
             }
-            tc_commit(mma_idle);
+            commit_pair(mma_idle, 1);
             mbar_wait(mma_idle, 0, p.status, abort_flag);
         }
     } else {
         // ------------------------------------------------------------ epilogue
         const int quarter = warp & 3;
-        const int r = quarter * 32 + lane;  // tile row = TMEM lane
+        const int r = quarter * 32 + lane;  // this CTA's tile row = TMEM lane
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
         int j = 0;
-        for (int i = blockIdx.x; i < n_tiles; i += gridDim.x, ++j) {
+        for (int i = cid; i < n_tiles; i += n_clusters, ++j) {
             const int b = j & 1;
             const GemmTile w = gemm_tile(i, n0, n1, mt0, total_m);
-            const int g = w.row0 + r;
+            const int g = w.row0 + (int)rank * kHalfM + r;
             const bool valid = g < w.row_end;
             const int t = valid ? p.perm[g] : 0;
             const int dst = (valid && p.dst_row != nullptr) ? p.dst_row[t] : t;
@@ -329,13 +421,14 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             }
             // this accumulator is read out: the MMAs of tile j + 2 may reuse it
             tc_fence_before();
-            mbar_arrive(&acc_empty[b]);
+            mbar_arrive_cluster(smem_in_rank(&acc_empty[b], 0));
         }
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync_all();  // no CTA leaves while its pair may still touch its memory
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, 512);
+    if (warp == 1) tmem_dealloc_pair(tmem, 512);
 }
 
 struct RlWorkspace {
@@ -407,11 +500,14 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     const uint64_t adims[4] = {(uint64_t)a->d_in, (uint64_t)T, 1, 1};
     const uint64_t astr[3] = {(uint64_t)a->d_in * 2, (uint64_t)a->d_in * 2 * T,
                               (uint64_t)a->d_in * 2 * T};
-    const uint32_t abox[4] = {kGBK, kGBM, 1, 1};
+    // boxes: one CTA's share of a stage (128 rows of A, 128 weight rows)
+    const uint32_t abox[4] = {kGBK, kHalfM, 1, 1};
     const uint64_t wdims[4] = {(uint64_t)a->d_in, (uint64_t)a->d_out, 1, 1};
     const uint64_t wstr[3] = {(uint64_t)a->d_in * 2, (uint64_t)a->d_in * 2 * a->d_out,
                               (uint64_t)a->d_in * 2 * a->d_out};
-    const uint32_t wbox[4] = {kGBK, kGBN, 1, 1};
+    const uint32_t wbox[4] = {kGBK, kHalfN, 1, 1};
+    static_assert(kGBK * kHalfM * 2 == GemmCfg::kABytes && kGBK * kHalfN * 2 == GemmCfg::kBBytes,
+                  "TMA boxes must fill exactly one stage slot");
     CUtensorMap tA, tW, tWn;
     if (!make_tmap_bf16_4d(&tA, Xg, adims, astr, abox) ||
         !make_tmap_bf16_4d(&tW, W, wdims, wstr, wbox) ||
@@ -437,7 +533,8 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     p.n_tiles_n = (a->d_out + kGBN - 1) / kGBN;
     p.status = a->status;
     const long long max_tiles = ((long long)(T + kGBM - 1) / kGBM + 1) * p.n_tiles_n;
-    const int blocks = (int)(max_tiles < sms ? max_tiles : sms);
+    const int pairs = (int)(max_tiles < sms / 2 ? max_tiles : sms / 2);
+    const int blocks = 2 * (pairs > 0 ? pairs : 1);
     constexpr size_t smem = GemmCfg::kSmem;
     static_assert(smem <= 232448, "routed GEMM shared memory");
     cudaError_t e = cudaFuncSetAttribute(routed_gemm_kernel,
