@@ -139,6 +139,7 @@ struct PfParams {
     const TileSum *sums;
     int max_k_tiles, max_k_len;
     int B, Hq, G;
+    int pack_log2;  // query heads per tile row group: a tile is 128 >> pack_log2 rows x (1 << pack_log2) heads
     int64_t o_ls;
     int total_q_rows;
     float scale_log2;
@@ -254,10 +255,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     //       16..27 per-warp counts
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
 
-    const int qt = blockIdx.x, h = blockIdx.y;
+    // A query tile is R query rows x P heads of one KV group (P = 1 << pack_log2,
+    // R = 128 / P): tile row r is query row r / P, head h0 + r % P.  P > 1 packs
+    // the heads of short query blocks so the tile rows are not left empty.
+    const int pl2 = p.pack_log2, R = kBM >> pl2;
+    const int qt = blockIdx.x, h0 = blockIdx.y << pl2;
     const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
     const int klen = p.k_len[b], qlen = p.q_len[b];
-    if (qt * 2 * kBM >= qlen || timed_out(p.status)) return;
+    if (qt * 2 * R >= qlen || timed_out(p.status)) return;
     // key side (kk*): the rows the tiles are cut from; k*: the S_aug sequence
     const int kklen = p.key_len[b];
     if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
@@ -266,16 +271,16 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         return;
     }
     const int kstart = p.k_start[b], kkstart = p.key_start[b];
-    const int kvh = h / p.G;
-    const int pbase = klen - qlen + qt * 2 * kBM;  // position of query row 0 of tile 0
-    const bool tile1 = qt * 2 * kBM + kBM < qlen;   // tile 1 has rows
+    const int kvh = h0 / p.G;
+    const int pbase = klen - qlen + qt * 2 * R;  // position of query row 0 of tile 0
+    const bool tile1 = qt * 2 * R + R < qlen;     // tile 1 has rows
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     // ------------------------------------------------ summaries of the query tiles
     if (tid < 10) misc[4 + tid] = (tid % 5 == 0) ? 0 : ((tid % 5) & 1 ? INT_MAX : INT_MIN);
     __syncthreads();
-    if (tid < 2 * kBM && pbase + tid <= klen - 1) {
-        int32_t *qs = misc + 4 + 5 * (tid >> 7);  // flags, seg min, seg max, nexus min, nexus max
+    if (tid < 2 * R && pbase + tid <= klen - 1) {
+        int32_t *qs = misc + 4 + 5 * (tid >= R ? 1 : 0);  // flags, seg min/max, nexus min/max
         const int ro = p.role[kstart + pbase + tid];
         const int s = p.seg[kstart + pbase + tid];
         atomicMin(&qs[1], s);
@@ -303,8 +308,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
             entry = (kn ? ((kb || ko) ? 2 : 1) : 0) << 2;
             for (int qi = 0; qi < 2; ++qi) {
-                const int p0 = pbase + qi * kBM;
-                const int p1 = min(p0 + kBM - 1, klen - 1);
+                const int p0 = pbase + qi * R;
+                const int p1 = min(p0 + R - 1, klen - 1);
                 if (p0 > p1) continue;
                 const int *qs = misc + 4 + 5 * qi;
                 const bool q_has_nexus = qs[0] & 2;
@@ -370,7 +375,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh)
                     tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full, hh * 64,
-                                h, p.q_start[b] + qt * 2 * kBM + qi * kBM, layer);
+                                h0, p.q_start[b] + qt * 2 * R + qi * R, layer);
         }
         int i = 0;
         for (; i < n_list; ++i) {
@@ -592,8 +597,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int qi = (warp - 2) >> 2;
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
-        const int pos = pbase + qi * kBM + r;
-        const bool row_ok = pos <= klen - 1 && qt * 2 * kBM + qi * kBM + r < qlen;
+        const int qr = r >> pl2, h = h0 + (r & ((1 << pl2) - 1));  // query row and head of tile row r
+        const int pos = pbase + qi * R + qr;
+        const bool row_ok = pos <= klen - 1 && qt * 2 * R + qi * R + qr < qlen;
         int rp = SONIC_ROLE_SYS, sp = 0;
         if (row_ok) {
             rp = p.role[kstart + pos];
@@ -804,7 +810,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         if (ok && n_list > 0 && mbar_wait(&o_done[qi], 0, p.status, abort_flag)) {
             tc_fence_after();
             const float inv = l > 0.f ? 1.f / l : 0.f;
-            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
+            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * R + qi * R + qr;
             uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
@@ -831,7 +837,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (kMass && row_ok)
                 p.nexus_mass[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = ln * inv;
         } else if (row_ok && n_list == 0) {
-            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * kBM + qi * kBM + r;
+            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * R + qi * R + qr;
             uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
             for (int d = 0; d < D; ++d) orow[d] = 0;
             if (kLse)
@@ -1115,7 +1121,15 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     if (a->workspace == nullptr || a->workspace_bytes < need) return SONIC_ERR_WORKSPACE;
     if (reorder && workspace_layout(a).rows > (int64_t)0x7fffffff - kBN)
         return SONIC_ERR_UNSUPPORTED;
-    const long long qtiles = (a->max_q_len + 2 * kBM - 1) / (2 * kBM);
+    // Query heads packed per tile (a power of two dividing G): short query
+    // blocks take 256 / P rows per block instead of leaving tile rows empty.
+    const int G = a->n_heads_q / a->n_heads_kv;
+    int pack_log2 = 0;
+    while ((G % (2 << pack_log2)) == 0 && pack_log2 < 3 &&
+           (long long)a->max_q_len * (2 << pack_log2) <= 2 * kBM)
+        ++pack_log2;
+    const int R = kBM >> pack_log2;
+    const long long qtiles = (a->max_q_len + 2 * R - 1) / (2 * R);
     if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_q > 65535 || qtiles > 0x7fffffff)
         return SONIC_ERR_UNSUPPORTED;
 
@@ -1138,8 +1152,9 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
                             (uint64_t)a->n_layers};
     const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, kt_layer};
     const uint32_t box[4] = {64, 1, 128, 1};
+    const uint32_t qbox[4] = {64, 1u << pack_log2, (uint32_t)R, 1};  // R rows x P heads
     CUtensorMap tq, tk, tv;
-    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, box) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
+    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, qbox) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
         !make_tmap_bf16_4d(&tv, Vt, kd, ks, box))
         return SONIC_ERR_INVALID_ARGUMENT;
 
@@ -1171,7 +1186,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.max_k_len = a->max_k_len;
     p.B = a->batch;
     p.Hq = a->n_heads_q;
-    p.G = a->n_heads_q / a->n_heads_kv;
+    p.G = G;
+    p.pack_log2 = pack_log2;
     p.o_ls = a->o_layer_stride;
     p.total_q_rows = a->total_q_rows;
     const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
@@ -1196,7 +1212,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
         p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
         static_cast<TileSum *>(a->workspace), p.max_k_tiles);
-    dim3 grid((unsigned)qtiles, a->n_heads_q, a->batch * a->n_layers);
+    dim3 grid((unsigned)qtiles, a->n_heads_q >> pack_log2, a->batch * a->n_layers);
     cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
                                : launch_prefill<64>(tq, tk, tv, p, grid, stream);
     return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;

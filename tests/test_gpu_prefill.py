@@ -77,6 +77,30 @@ def test_uniform_scores_count_visible_keys(mode, order):
         H.check_close(got, O, f"seq {b}")
 
 
+@pytest.mark.parametrize("order", ORDERS)
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+@pytest.mark.parametrize("hq,hkv,max_q", [(8, 2, 32), (8, 1, 20), (16, 2, 64), (6, 3, 100)])
+def test_short_query_blocks_pack_heads(order, mode, hq, hkv, max_q):
+    """Short query blocks (the Nexus rows of a segment, a few current-turn
+    rows): the kernel packs 2, 4 or 8 query heads of a KV group into one
+    128-row tile.  Ragged q_len from 1 to max_q over multi-tile key sequences,
+    every query row and head against the oracle, with lse and Nexus mass."""
+    rng = np.random.default_rng(hq * 100 + max_q)
+    ds = [inputs.random_dialogue(rng, max_segments=6, max_body=150, max_nexus=40, max_sys=90,
+                                 max_curr=150) for _ in range(5)]
+    batch = inputs.Batch(ds)
+    q_len = np.minimum(rng.integers(1, max_q + 1, batch.B), batch.k_len)
+    res = H.run_prefill(batch, hq, hkv, 128, q_len=q_len, seed=51, nexus_vis=mode,
+                        key_order=order, with_mass=True)
+    for b in range(batch.B):
+        rows = np.arange(q_len[b])
+        O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, rows, nexus_vis=mode)
+        H.check_close(got, O, f"seq {b}")
+        np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
+        want, gm = H.oracle_mass_rows(batch, res, b, rows, nexus_vis=mode)
+        np.testing.assert_allclose(gm, want, rtol=0, atol=2e-3)
+
+
 MASS_ATOL = 2e-3  # attention mass on Nexus keys: a share in [0, 1]
 
 
