@@ -728,6 +728,38 @@ def extra_nexus_gen():
                         "ms_per_segment": round((p_ms + c_ms) / len(segs), 3)}}
 
 
+def extra_compaction():
+    """KV compaction (Sec. 3.2 body removal) at the masked-prefill shapes
+    (batch 8 x 5632 raw rows -> 1536 retained, 32 layers, 8 KV heads, D = 128:
+    3.22 GB moved) and of the long ragged histories (64 dialogues, Nexus =
+    len/2 and len/5, 4 of the 32 layers: the per-layer work is the same)."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    res = {}
+    cases = [("masked_prefill_32_layers", inputs.masked_prefill(), 32),
+             ("long_ragged_nexus_len_div_2_4_layers", inputs.long_ragged(2), 4),
+             ("long_ragged_nexus_len_div_5_4_layers", inputs.long_ragged(5), 4)]
+    for name, (batch, hd), nl in cases:
+        K = inputs.randn((nl, batch.total, hd.hkv, hd.d), seed=5, device=dev)
+        V = inputs.randn((nl, batch.total, hd.hkv, hd.d), seed=6, device=dev)
+        ret = sum(d.recipe_retained for d in batch.dialogues)
+        oK = torch.empty((nl, ret, hd.hkv, hd.d), dtype=K.dtype, device=dev)
+        oV = torch.empty_like(oK)
+        off = torch.zeros(batch.B + 1, dtype=torch.int32, device=dev)
+        r_, s_, ks, kl = t(batch.role), t(batch.seg), t(batch.k_start), t(batch.k_len)
+        ws = sonic.sonic_compact_kv(K, V, s_, r_, oK, oV, off, k_start=ks, k_len=kl)
+        ms = _ev_time(lambda: sonic.sonic_compact_kv(K, V, s_, r_, oK, oV, off, k_start=ks,
+                                                     k_len=kl, workspace=ws), reps=10, warm=3)
+        by = 2.0 * ret * hd.hkv * hd.d * 2 * 2 * nl
+        res[name] = {"ms": round(ms, 3), "gbs": round(by / ms / 1e6, 1), "gb_moved": round(by / 1e9, 2),
+                     "raw_gb": round(2.0 * batch.total * hd.hkv * hd.d * 2 * nl / 1e9, 2)}
+        del K, V, oK, oV
+        torch.cuda.empty_cache()
+    return {"workload": "KV compaction (retained rows read + written, K and V)", "results": res}
+
+
 def extra_nexus_mass():
     """Cost of the attention-mass output (Sec. 4.1 Eq. 9's A_nexus per row and
     head) on the mixed serving step at 8 layers: its prefill and its decode
@@ -827,7 +859,7 @@ def extra_routed():
 
 
 EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
-          "nexus_mass": extra_nexus_mass, "routed": extra_routed,
+          "nexus_mass": extra_nexus_mass, "routed": extra_routed, "compaction": extra_compaction,
           "context": extra_context, "nexus_gen": extra_nexus_gen}
 
 
