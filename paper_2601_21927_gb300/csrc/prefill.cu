@@ -626,30 +626,15 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // the keys' roles/segments are read (and V rows zeroed) on cut tiles
             // only, and their Nexus bits on tiles with some Nexus keys
             const bool need_meta = cut || (kMass && nexus_keys == 2);
-            if ((need_meta && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) ||
-                !mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
+            if (need_meta && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) {
                 ok = false;
                 break;
             }
-            tc_fence_after();
-            // S row into registers: four 32-column loads, one wait
-            uint32_t sr[4][32];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
-            tmem_ld_wait();
-#pragma unroll
-            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
-            // row maximum (and the mask bits of a cut tile)
+            // The mask bits of a cut tile, worked out before S is read: the MMA
+            // producing S runs meanwhile, and the mask record and the S row are
+            // never held in registers together.
             uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (!cut) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2)
-                        mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][e]),
-                                       __uint_as_float(sr[c][e + 1]));
-            } else {
+            if (cut) {
                 // the whole mask record in independent 16-byte loads
                 const uint4 *tv = reinterpret_cast<const uint4 *>(tmasks + st);
                 const uint4 nb = tv[0], nx = tv[1], hd = tv[2], bsg = tv[3], nsg = tv[4];
@@ -709,6 +694,29 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         mbits[c] = bits;
                     }
                 }
+            }
+            if (!mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            // S row into registers: four 32-column loads, one wait
+            uint32_t sr[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+            tmem_ld_wait();
+#pragma unroll
+            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
+            // row maximum (masked keys set to -inf on a cut tile)
+            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (!cut) {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2)
+                        mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][e]),
+                                       __uint_as_float(sr[c][e + 1]));
+            } else {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
