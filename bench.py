@@ -728,6 +728,50 @@ def extra_nexus_gen():
                         "ms_per_segment": round((p_ms + c_ms) / len(segs), 3)}}
 
 
+def extra_decode_graph():
+    """Decode of the Llama-3-8B-like batch (16 x 641 retained rows, 32 layers,
+    32/8 heads): one launch over all layers, and 32 per-layer launches
+    captured once in a CUDA graph and replayed."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    b2, h2 = inputs.decode_llama8b()
+    lens = np.array([x.recipe_retained + 1 for x in b2.dialogues], np.int32)
+    starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int32)
+    T, nl = int(lens.sum()), h2.n_layers
+    K = inputs.randn((nl, T, h2.hkv, h2.d), seed=7, device=dev)
+    V = inputs.randn((nl, T, h2.hkv, h2.d), seed=8, device=dev)
+    q = inputs.randn((nl, b2.B, h2.hq, h2.d), seed=9, device=dev)
+    O = torch.empty_like(q)
+    lt = torch.as_tensor(lens).to(dev)
+    st = torch.as_tensor(starts).to(dev)
+    ml = int(lens.max())
+    ws_all = sonic.sonic_attn_decode(q, K, V, lt, O, kv_start=st, max_len=ml)
+    ms_all = _ev_time(lambda: sonic.sonic_attn_decode(q, K, V, lt, O, kv_start=st, max_len=ml,
+                                                      workspace=ws_all), reps=20, warm=3)
+    ws = [sonic.sonic_attn_decode(q[l:l + 1], K[l:l + 1], V[l:l + 1], lt, O[l:l + 1],
+                                  kv_start=st, max_len=ml) for l in range(nl)]
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for l in range(nl):
+            sonic.sonic_attn_decode(q[l:l + 1], K[l:l + 1], V[l:l + 1], lt, O[l:l + 1],
+                                    kv_start=st, max_len=ml, workspace=ws[l])
+    ms_graph = _ev_time(g.replay, reps=20, warm=3)
+    ms_eager = _ev_time(lambda: [sonic.sonic_attn_decode(
+        q[l:l + 1], K[l:l + 1], V[l:l + 1], lt, O[l:l + 1], kv_start=st, max_len=ml,
+        workspace=ws[l]) for l in range(nl)], reps=20, warm=3)
+    by = (T * h2.hkv * h2.d * 2 * 2 + 2 * b2.B * h2.hq * h2.d * 2) * nl
+    rate = lambda ms: round(by / ms / 1e6, 1)
+    return {"workload": "decode, batch 16 x 641 retained rows, 32 layers, 32/8 heads, D=128 "
+                        "(1.35 GB)",
+            "results": {"one_launch_all_layers": {"ms": round(ms_all, 4), "gbs": rate(ms_all)},
+                        "per_layer_launches_cuda_graph": {"ms": round(ms_graph, 4),
+                                                          "gbs": rate(ms_graph)},
+                        "per_layer_launches_eager": {"ms": round(ms_eager, 4),
+                                                     "gbs": rate(ms_eager)}}}
+
+
 def extra_compaction():
     """KV compaction (Sec. 3.2 body removal) at the masked-prefill shapes
     (batch 8 x 5632 raw rows -> 1536 retained, 32 layers, 8 KV heads, D = 128:
@@ -860,6 +904,7 @@ def extra_routed():
 
 EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
           "nexus_mass": extra_nexus_mass, "routed": extra_routed, "compaction": extra_compaction,
+          "decode_graph": extra_decode_graph,
           "context": extra_context, "nexus_gen": extra_nexus_gen}
 
 
