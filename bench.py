@@ -846,8 +846,9 @@ def extra_routed():
     4096 -> 4096 + 1024 + 1024, K/V into cache rows), the QKV and O
     projections of the serving step's 12,146 prefill rows (Qwen2.5-7B-like
     3584 -> 3584 + 512 + 512, and 3584 -> 3584), with half of those rows
-    marked Nexus in runs of 32.  Beside each: cuBLAS (torch.matmul) on the
-    two role groups plus the row scatter, as context."""
+    marked Nexus in runs of 32, and the QKV projection of the same rows as
+    one current turn (one role: no rows are copied).  Beside each: cuBLAS
+    (torch.matmul) on the role groups plus the row scatter, as context."""
     import torch
     from paper_2601_21927_gb300 import inputs, sonic
     dev = torch.device("cuda", 0)
@@ -859,6 +860,8 @@ def extra_routed():
         "nexus_gen_qkv_T2304_4096x6144": (nexus_gen, 4096, [4096, 1024, 1024], [0, 1, 1]),
         "serving_qkv_T12146_3584x4608": (serving, 3584, [3584, 512, 512], [0, 1, 1]),
         "serving_o_T12146_3584x3584": (serving, 3584, [3584], [0]),
+        "current_turn_qkv_T12146_3584x4608": (np.full(12146, 3, np.uint8), 3584,
+                                              [3584, 512, 512], [0, 1, 1]),
     }
     for name, (role, d_in, cols, scat) in cases.items():
         T, d_out = len(role), sum(cols)

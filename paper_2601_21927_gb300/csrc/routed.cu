@@ -9,7 +9,9 @@
 //   role_order    per chunk: the stable partition [ordinary rows | Nexus rows]
 //                 (perm[g] = source row of grouped row g) and the two group
 //                 sizes;
-//   row_gather    the rows of X in grouped order (warp per row, 16-byte loads);
+//   row_gather    the rows of X in grouped order (warp per row, 16-byte loads),
+//                 except slabs of grouped rows that are runs of X's rows, which
+//                 the GEMM loads from X directly;
 //   routed_gemm   a persistent tcgen05 GEMM on CTA pairs over 256 x 256
 //                 output tiles of the grouped rows.  A tile never straddles
 //                 the two groups, so each tile reads one weight matrix; the
@@ -101,14 +103,32 @@ role_order_kernel(const uint8_t *__restrict__ role, int32_t T, int32_t n_chunks,
     }
 }
 
-// Xg[g] = X[perm[g]]: one warp per row, 16-byte loads.
+// The GEMM stages A in slabs of 128 grouped rows, counted from the start of
+// each role group (a CTA's share of a 256-row pair tile).  Grouped rows keep
+// their order within a group, so a slab is one run of consecutive rows of X
+// exactly when its first and last source rows are as far apart as its rows;
+// the GEMM then loads the slab from X itself and it is not copied.
+__device__ __forceinline__ int slab_start(int g, int n0) {
+    return g < n0 ? (g / kHalfM) * kHalfM : n0 + ((g - n0) / kHalfM) * kHalfM;
+}
+
+__device__ __forceinline__ bool slab_is_run(const int32_t *perm, int s0, int group_end) {
+    const int e = min(s0 + kHalfM, group_end);
+    return perm[e - 1] - perm[s0] == e - 1 - s0;
+}
+
+// Xg[g] = X[perm[g]] for the rows of slabs that are not runs of X: one warp
+// per row, 16-byte loads.
 __global__ void __launch_bounds__(256)
 row_gather_kernel(const uint8_t *__restrict__ X, int64_t x_row_bytes, int32_t T,
-                  int64_t row_bytes, const int32_t *__restrict__ perm, uint8_t *__restrict__ Xg) {
+                  int64_t row_bytes, const int32_t *__restrict__ perm,
+                  const int32_t *__restrict__ groups, uint8_t *__restrict__ Xg) {
     const int lane = threadIdx.x & 31;
     const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int cpr = (int)(row_bytes >> 4);
+    const int n0 = groups[0];
     for (int64_t g = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; g < T; g += n_warps) {
+        if (slab_is_run(perm, slab_start((int)g, n0), g < n0 ? n0 : T)) continue;
         const uint8_t *src = X + (int64_t)perm[g] * x_row_bytes;
         uint8_t *dst = Xg + g * row_bytes;
         for (int c0 = lane; c0 < cpr; c0 += 128) {
@@ -263,8 +283,9 @@ __device__ __forceinline__ void commit_pair(uint64_t *bar, uint16_t mask) {
 }
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
-routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
-                   const __grid_constant__ CUtensorMap tmWn, const GemmParams p) {
+routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmX,
+                   const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmWn,
+                   const GemmParams p) {
     using C = GemmCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -317,6 +338,7 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         // the pair's bytes.
         if (lane == 0) {
             tma_prefetch_desc(&tmA);
+            tma_prefetch_desc(&tmX);
             tma_prefetch_desc(&tmW);
             tma_prefetch_desc(&tmWn);
             int it = 0;
@@ -324,6 +346,12 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             for (int i = cid; ok && i < n_tiles; i += n_clusters) {
                 const GemmTile w = gemm_tile(i, n0, n1, mt0, total_m);
                 const CUtensorMap *tb = w.g ? &tmWn : &tmW;
+                // this CTA's 128 rows of A: straight from X when they are one run
+                // of X's rows, else from the grouped copy
+                const int s0 = w.row0 + (int)rank * kHalfM;
+                const bool run = s0 < w.row_end && slab_is_run(p.perm, s0, w.row_end);
+                const CUtensorMap *ta = run ? &tmX : &tmA;
+                const int arow = run ? p.perm[s0] : s0;
                 for (int kb = 0; kb < nk; ++kb, ++it) {
                     const int s = it % kGStages;
                     if (it >= kGStages &&
@@ -334,7 +362,7 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     uint8_t *a = smem + s * C::kStageBytes;
                     if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * C::kStageBytes);
                     const uint32_t bar = smem_u32(&full[s]) & 0xFEFFFFFFu;
-                    tma_load_pair(a, &tmA, bar, kb * kGBK, w.row0 + (int)rank * kHalfM);
+                    tma_load_pair(a, ta, bar, kb * kGBK, arow);
                     tma_load_pair(a + C::kABytes, tb, bar, kb * kGBK,
                                   w.n * kGBN + (int)rank * kHalfN);
                 }
@@ -508,8 +536,13 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     const uint32_t wbox[4] = {kGBK, kHalfN, 1, 1};
     static_assert(kGBK * kHalfM * 2 == GemmCfg::kABytes && kGBK * kHalfN * 2 == GemmCfg::kBBytes,
                   "TMA boxes must fill exactly one stage slot");
-    CUtensorMap tA, tW, tWn;
+    // X itself, for slabs of grouped rows that are runs of X's rows
+    const uint64_t xdims[4] = {(uint64_t)a->d_in, (uint64_t)T, 1, 1};
+    const uint64_t xstr[3] = {(uint64_t)a->x_row_stride * 2, (uint64_t)a->x_row_stride * 2 * T,
+                              (uint64_t)a->x_row_stride * 2 * T};
+    CUtensorMap tA, tX, tW, tWn;
     if (!make_tmap_bf16_4d(&tA, Xg, adims, astr, abox) ||
+        !make_tmap_bf16_4d(&tX, X, xdims, xstr, abox) ||
         !make_tmap_bf16_4d(&tW, W, wdims, wstr, wbox) ||
         !make_tmap_bf16_4d(&tWn, W_nexus, wdims, wstr, wbox))
         return SONIC_ERR_INVALID_ARGUMENT;
@@ -521,7 +554,7 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     const int gblocks = (int)((T < gwarps ? T : gwarps) + 7) / 8;
     row_gather_kernel<<<gblocks, 256, 0, stream>>>(
         reinterpret_cast<const uint8_t *>(X), a->x_row_stride * 2, T, (int64_t)a->d_in * 2, perm,
-        reinterpret_cast<uint8_t *>(Xg));
+        groups, reinterpret_cast<uint8_t *>(Xg));
 
     p.groups = groups;
     p.perm = perm;
@@ -540,6 +573,6 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     cudaError_t e = cudaFuncSetAttribute(routed_gemm_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return SONIC_ERR_CUDA;
-    routed_gemm_kernel<<<blocks, kGThreads, smem, stream>>>(tA, tW, tWn, p);
+    routed_gemm_kernel<<<blocks, kGThreads, smem, stream>>>(tA, tX, tW, tWn, p);
     return cudaGetLastError() == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
 }

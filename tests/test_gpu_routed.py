@@ -108,10 +108,22 @@ def test_qkv_parts_into_cache_rows(T):
     _check(r)
 
 
+@pytest.mark.parametrize("x_pad", [0, 64])
 @pytest.mark.parametrize("which", ["none", "all"])
-def test_one_group_empty(which):
+def test_one_group_empty(which, x_pad):
+    """One role only: every 128-row slab is a run of X's rows, loaded from X
+    itself (rows padded or not); nothing is copied."""
     role = np.full(777, inputs.ROLE_NEXUS if which == "all" else inputs.ROLE_CURR, np.uint8)
-    _check(_run(role, 256, [256, 64], [False, True], seed=7, cache_rows=900))
+    _check(_run(role, 256, [256, 64], [False, True], seed=7, cache_rows=900, x_pad=x_pad))
+
+
+def test_runs_and_copied_slabs_mixed():
+    """Long runs of one role (slabs loaded from X) next to short alternating
+    runs (slabs copied), group boundaries off the 128-row grid."""
+    role = np.r_[np.full(300, inputs.ROLE_BODY), np.full(5, inputs.ROLE_NEXUS),
+                 np.tile(np.r_[np.full(3, inputs.ROLE_CURR), np.full(4, inputs.ROLE_NEXUS)], 40),
+                 np.full(260, inputs.ROLE_NEXUS), np.full(9, inputs.ROLE_SYS)].astype(np.uint8)
+    _check(_run(role, 128, [128, 96], [False, True], seed=13, cache_rows=2000, x_pad=32))
 
 
 def test_same_weights_is_a_plain_linear_layer_and_strided_x():
