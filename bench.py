@@ -604,9 +604,13 @@ def extra_decode():
     dev = torch.device("cuda", 0)
     t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
     res = {}
-    for name, (b2, h2) in {"llama8b_641_rows": inputs.decode_llama8b(),
-                           "long_ragged_nexus_len_div_2": inputs.long_ragged(2),
-                           "long_ragged_nexus_len_div_5": inputs.long_ragged(5)}.items():
+    lr2 = inputs.long_ragged(2)
+    cases = {"llama8b_641_rows": inputs.decode_llama8b(),
+             "long_ragged_nexus_len_div_2": lr2,
+             "long_ragged_nexus_len_div_5": inputs.long_ragged(5),
+             # head_dim 64 (CUDA-core kernel): the same dialogues, 8 layers, 32/8 heads
+             "long_ragged_nexus_len_div_2_head_dim_64": (lr2[0], inputs.Heads(8, 32, 8, 64))}
+    for name, (b2, h2) in cases.items():
         lens = np.array([x.recipe_retained + 1 for x in b2.dialogues], np.int32)
         starts = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int32)
         T = int(lens.sum())

@@ -280,7 +280,7 @@ typedef struct {
     int64_t o_layer_stride;      /* elements between layers of O                        */
     float softmax_scale;         /* 0 selects 1/sqrt(head_dim)                          */
     int32_t chunk_len;           /* keys per split (0 = automatic), rounded up to the key
-                                    tile: 128 keys at head_dim 128, 32 at head_dim 64   */
+                                    tile of 128 keys                                    */
     float *lse;                  /* device [n_layers][B][Hq] or NULL                    */
     int32_t *status;             /* device int32 or NULL                                */
     void *workspace;             /* device, sonic_decode_workspace_size() bytes         */
@@ -299,10 +299,10 @@ typedef struct {
  * The keys are split into chunks of chunk_len; each (layer, sequence, KV
  * head, chunk) unit produces a partial (max, sum, accumulator) in the
  * workspace, and a second kernel merges them by log-sum-exp (a sequence that
- * fits one chunk is written directly).  At head_dim 128 one persistent block
- * per SM claims units from a counter in the workspace (zeroed on `stream`
- * before the launch), so the workspace is never empty there and concurrent
- * calls need workspaces of their own.  lens[b] = 0 gives zeros (and
+ * fits one chunk is written directly).  One persistent block per SM claims
+ * units from a counter in the workspace (zeroed on `stream` before the
+ * launch), so the workspace is never empty and concurrent calls need
+ * workspaces of their own.  lens[b] = 0 gives zeros (and
  * lse = -inf).  bf16 in/out, fp32 arithmetic.  nexus_mass (optional, role
  * then required, else SONIC_ERR_INVALID_ARGUMENT) is the decode form of the
  * quantity behind A_nexus (Sec. 4.1, Eq. 9): the share of the new token's

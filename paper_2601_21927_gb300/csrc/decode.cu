@@ -5,46 +5,23 @@
 // kept).  Every retained row of a sequence is visible to its new token.
 //
 // Split-K, HBM-bound design:
-//   decode_split   one block per (key chunk, KV head, sequence, layer).  A
-//                  producer warp streams the chunk's K and V through a ring
-//                  of 32-key shared-memory stages with TMA (128-byte swizzle,
-//                  so both access patterns below are bank-conflict free).
-//                  Eight consumer warps take turns on the tiles; each keeps
-//                  its own online softmax for the G query heads that share
-//                  the KV head:
-//                    scores  lane = key (32-key tiles), full-D dot products
-//                            against q in shared memory (broadcast reads),
-//                            packed fp32x2 FMAs, no cross-lane reduction;
-//                    P . V   lane = 4 (D=128) or 2 (D=64) output dims, keys
-//                            walked in order, p broadcast from shared memory.
-//                  The warps are merged by log-sum-exp at the end; a
-//                  single-chunk sequence writes O directly, otherwise the
-//                  partial (max, sum, unnormalised accumulator) goes to the
-//                  workspace.
+//   decode_tc      persistent blocks (one per SM) claim units (key chunk, KV
+//                  head, sequence, layer) from a counter and stream their K/V
+//                  tiles of 128 keys through a TMA ring; both contractions run
+//                  on the tensor cores with the keys in the M dimension (see
+//                  the kernel's comment); a single-chunk sequence writes O
+//                  directly, otherwise the partial (max, sum, unnormalised
+//                  accumulator) goes to the workspace.  head_dim 64 and 128.
 //   decode_combine log-sum-exp merge of the chunks of each (layer, seq, head).
-// K and V are read exactly once from HBM; softmax runs in base 2 with the
-// scale folded into q.
+// K and V are read exactly once from HBM; softmax runs in base 2.
 #include "sonic_dev.cuh"
 #include "sonic_host.h"
 
 namespace sonic {
 namespace {
 
-constexpr int kTileKeys = 32;
-constexpr int kConsumerWarps = 8;
-constexpr int kDecThreads = (kConsumerWarps + 1) * 32;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
-
-template <int D>
-struct DecCfg {
-    static constexpr int kHalves = D / 64;               // 128-byte swizzle rows per key
-    static constexpr int kTileBytes = kTileKeys * D * 2;  // K (or V) tile
-    static constexpr int kStageBytes = 2 * kTileBytes;
-    static constexpr int kStages = (D == 128) ? 12 : 24;
-    static constexpr int kChunks = D / 8;  // 16-byte pieces of one key row
-    static constexpr int kDpl = D / 32;    // P.V output dims per lane
-};
 
 struct DecParams {
     const uint16_t *q;
@@ -66,20 +43,6 @@ struct DecParams {
     float scale_log2;
 };
 
-template <int D, int GT>
-constexpr size_t dec_smem_bytes() {
-    using C = DecCfg<D>;
-    constexpr int Gp = (GT + 3) & ~3;
-    return 1024 + (size_t)C::kStages * C::kStageBytes + (size_t)GT * D * 4 +
-           (size_t)kConsumerWarps * kTileKeys * Gp * 4 + 2 * C::kStages * 8 + 16;
-}
-
-__device__ __forceinline__ uint4 lds128(const uint8_t *p) {
-    return *reinterpret_cast<const uint4 *>(p);
-}
-
-__device__ __forceinline__ float2 w2f(uint32_t w) { return make_float2(bf16lo(w), bf16hi(w)); }
-
 // Maximum of v over the 32 lanes of the warp, in one instruction.
 __device__ __forceinline__ float warp_max(float v) {
     float r;
@@ -87,251 +50,8 @@ __device__ __forceinline__ float warp_max(float v) {
     return r;
 }
 
-template <int D, int GT>
-__global__ void __launch_bounds__(kDecThreads, 1)
-decode_split_kernel(const __grid_constant__ CUtensorMap tmK,
-                    const __grid_constant__ CUtensorMap tmV, const DecParams p) {
-    using C = DecCfg<D>;
-    constexpr int Gp = (GT + 3) & ~3;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    float *q_s = reinterpret_cast<float *>(smem + C::kStages * C::kStageBytes);
-    float *p_s = q_s + GT * D;
-    uint64_t *full = reinterpret_cast<uint64_t *>(p_s + kConsumerWarps * kTileKeys * Gp);
-    uint64_t *empty = full + C::kStages;
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + C::kStages);
-
-    // The KV head is the fastest grid index: the blocks reading the head slices
-    // of the same rows are launched together and share DRAM pages.
-    const int kvh = blockIdx.x % p.Hkv, chunk = blockIdx.x / p.Hkv;
-    const int b = blockIdx.y % p.B, layer = blockIdx.y / p.B;
-    int len = p.lens[b];
-    if (len > p.max_chunks * p.chunk_len) {
-        // longer than the host-side bound: attend to the first max_len keys only
-        if (threadIdx.x == 0 && blockIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
-        len = p.max_chunks * p.chunk_len;
-    }
-    const int key0 = chunk * p.chunk_len;
-    if (key0 >= len || timed_out(p.status)) return;
-    const int nkeys = min(p.chunk_len, len - key0);
-    const int ntiles = (nkeys + kTileKeys - 1) / kTileKeys;
-    const int G = p.G;
-    const int row0 = p.kv_start[b] + key0;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-    if (tid == 0) {
-        for (int s = 0; s < C::kStages; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
-        }
-        *abort_flag = 0;
-        fence_mbar_init();
-    }
-    // q of the G heads sharing this KV head, pre-scaled into the base-2 domain.
-    const uint16_t *qp = p.q + layer * p.q_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G) * D;
-    for (int i = tid; i < GT * D; i += blockDim.x) {
-        const int g = i / D;
-        float v = 0.f;
-        if (g < G) v = __uint_as_float((uint32_t)qp[i] << 16) * p.scale_log2;
-        q_s[i] = v;
-    }
-    __syncthreads();
-
-    if (warp == kConsumerWarps) {
-        // ------------------------------------------------------------ producer
-        if (lane == 0) {
-            tma_prefetch_desc(&tmK);
-            tma_prefetch_desc(&tmV);
-            int t = 0;
-            for (; t < ntiles; ++t) {
-                const int s = t % C::kStages;
-                if (t >= C::kStages &&
-                    !mbar_wait(&empty[s], ((t / C::kStages) - 1) & 1, p.status, abort_flag))
-                    break;
-                mbar_arrive_expect_tx(&full[s], C::kStageBytes);
-                uint8_t *kd = smem + s * C::kStageBytes;
-                uint8_t *vd = kd + C::kTileBytes;
-                const int r = row0 + t * kTileKeys;
-#pragma unroll
-                for (int h = 0; h < C::kHalves; ++h) {
-                    tma_load_4d(kd + h * kTileKeys * 128, &tmK, &full[s], h * 64, kvh, r, layer);
-                    tma_load_4d(vd + h * kTileKeys * 128, &tmV, &full[s], h * 64, kvh, r, layer);
-                }
-            }
-            if (*abort_flag) {
-                // Let the copies already issued land before the block exits.
-                for (int u = max(0, t - C::kStages); u < t; ++u)
-                    mbar_wait(&full[u % C::kStages], (u / C::kStages) & 1, p.status, abort_flag);
-            }
-        }
-    }
-
-    // ------------------------------------------------------------ consumers
-    // n: the part of l on Nexus keys (only when the mass is requested)
-    const bool want_nx = p.nexus_mass != nullptr;
-    float m[GT], l[GT], n[GT];
-    float2 acc[GT][C::kDpl / 2];
-#pragma unroll
-    for (int g = 0; g < GT; ++g) {
-        m[g] = -INFINITY;
-        l[g] = 0.f;
-        n[g] = 0.f;
-#pragma unroll
-        for (int e = 0; e < C::kDpl / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
-    }
-    if (warp < kConsumerWarps) {
-        float *pw = p_s + warp * kTileKeys * Gp;
-        const int sw = lane & 7;
-        for (int t = warp; t < ntiles; t += kConsumerWarps) {
-            const int s = t % C::kStages;
-            if (!mbar_wait(&full[s], (t / C::kStages) & 1, p.status, abort_flag)) break;
-            const uint8_t *Ks = smem + s * C::kStageBytes;
-            const uint8_t *Vs = Ks + C::kTileBytes;
-            const int valid = min(kTileKeys, nkeys - t * kTileKeys);
-            const bool isn = want_nx && lane < valid &&
-                             p.role[row0 + t * kTileKeys + lane] == SONIC_ROLE_NEXUS;
-
-            // scores: lane owns key `lane` of the tile
-            float2 dk[GT];
-#pragma unroll
-            for (int g = 0; g < GT; ++g) dk[g] = make_float2(0.f, 0.f);
-#pragma unroll 2
-            for (int c = 0; c < C::kChunks; ++c) {
-                const int half = c >> 3, jj = c & 7;
-                const uint4 kw =
-                    lds128(Ks + half * (kTileKeys * 128) + lane * 128 + ((jj ^ sw) << 4));
-                const float2 a0 = w2f(kw.x), a1 = w2f(kw.y), a2 = w2f(kw.z), a3 = w2f(kw.w);
-#pragma unroll
-                for (int g = 0; g < GT; ++g) {
-                    const float4 q0 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8);
-                    const float4 q1 = *reinterpret_cast<const float4 *>(q_s + g * D + c * 8 + 4);
-                    dk[g] = __ffma2_rn(a0, make_float2(q0.x, q0.y), dk[g]);
-                    dk[g] = __ffma2_rn(a1, make_float2(q0.z, q0.w), dk[g]);
-                    dk[g] = __ffma2_rn(a2, make_float2(q1.x, q1.y), dk[g]);
-                    dk[g] = __ffma2_rn(a3, make_float2(q1.z, q1.w), dk[g]);
-                }
-            }
-            // online softmax (base 2), per query head
-#pragma unroll
-            for (int g = 0; g < GT; ++g) {
-                const float sc = lane < valid ? dk[g].x + dk[g].y : -INFINITY;
-                const float mn = fmaxf(m[g], warp_max(sc));
-                const float alpha = ex2(m[g] - mn);
-                const float pr = ex2(sc - mn);
-                l[g] = l[g] * alpha + pr;
-                if (want_nx) n[g] = n[g] * alpha + (isn ? pr : 0.f);
-#pragma unroll
-                for (int e = 0; e < C::kDpl / 2; ++e) {
-                    acc[g][e].x *= alpha;
-                    acc[g][e].y *= alpha;
-                }
-                m[g] = mn;
-                pw[lane * Gp + g] = pr;
-            }
-            __syncwarp();
-            // P . V: lane owns output dims [lane * kDpl, lane * kDpl + kDpl)
-            {
-                const int e0 = lane * C::kDpl;
-                const int half = e0 >> 6, jj = (e0 & 63) >> 3;
-                const int sub = (e0 & 7) * 2;  // byte offset inside the 16-byte piece
-                const uint8_t *vb = Vs + half * (kTileKeys * 128) + sub;
-#pragma unroll 4
-                for (int k = 0; k < valid; ++k) {
-                    const uint8_t *vrow = vb + k * 128 + ((jj ^ (k & 7)) << 4);
-                    float2 v[C::kDpl / 2];
-                    if constexpr (C::kDpl == 4) {
-                        const uint2 w = *reinterpret_cast<const uint2 *>(vrow);
-                        v[0] = w2f(w.x);
-                        v[1] = w2f(w.y);
-                    } else {
-                        v[0] = w2f(*reinterpret_cast<const uint32_t *>(vrow));
-                    }
-                    const float *pk = pw + k * Gp;
-#pragma unroll
-                    for (int g4 = 0; g4 < Gp; g4 += 4) {
-                        const float4 pv = *reinterpret_cast<const float4 *>(pk + g4);
-                        const float pp[4] = {pv.x, pv.y, pv.z, pv.w};
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            if (g4 + u < GT) {
-                                const float2 pp2 = make_float2(pp[u], pp[u]);
-#pragma unroll
-                                for (int e = 0; e < C::kDpl / 2; ++e)
-                                    acc[g4 + u][e] = __ffma2_rn(pp2, v[e], acc[g4 + u][e]);
-                            }
-                        }
-                    }
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[s]);
-        }
-        // total of the lane partial sums
-#pragma unroll
-        for (int g = 0; g < GT; ++g)
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
-                if (want_nx) n[g] += __shfl_xor_sync(0xffffffffu, n[g], o);
-            }
-    }
-    __syncthreads();
-    if (*abort_flag) return;
-
-    // ---------------------------------------------------- merge the 4 warps
-    float *macc = reinterpret_cast<float *>(smem);  // [warps][GT][D] (stage memory is free now)
-    float *mml = macc + kConsumerWarps * GT * D;    // [warps][GT][2]
-    float *mnx = mml + kConsumerWarps * GT * 2;     // [warps][GT]
-    if (warp < kConsumerWarps) {
-#pragma unroll
-        for (int g = 0; g < GT; ++g) {
-#pragma unroll
-            for (int e = 0; e < C::kDpl / 2; ++e)
-                *reinterpret_cast<float2 *>(macc + (warp * GT + g) * D + lane * C::kDpl + 2 * e) =
-                    acc[g][e];
-            if (lane == 0) {
-                mml[(warp * GT + g) * 2 + 0] = m[g];
-                mml[(warp * GT + g) * 2 + 1] = l[g];
-                mnx[warp * GT + g] = n[g];
-            }
-        }
-    }
-    __syncthreads();
-    const int n_chunks = (len + p.chunk_len - 1) / p.chunk_len;
-    const int64_t unit0 = ((int64_t)layer * p.B + b) * p.Hq + (int64_t)kvh * G;
-    for (int i = tid; i < G * D; i += blockDim.x) {
-        const int g = i / D, d = i - g * D;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, mml[(w * GT + g) * 2]);
-        float L = 0.f, a = 0.f, N = 0.f;
-#pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
-            const float f = ex2(mml[(w * GT + g) * 2] - M);
-            L += f * mml[(w * GT + g) * 2 + 1];
-            a += f * macc[(w * GT + g) * D + d];
-            N += f * mnx[w * GT + g];
-        }
-        if (n_chunks == 1) {
-            uint16_t *op = p.O + layer * p.o_ls + ((int64_t)b * p.Hq + (int64_t)kvh * G + g) * D;
-            op[d] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
-            if (d == 0 && p.lse != nullptr) p.lse[unit0 + g] = (M + __log2f(L)) * kLn2;
-            if (d == 0 && want_nx) p.nexus_mass[unit0 + g] = N / L;
-        } else {
-            const int64_t slot = (unit0 + g) * p.max_chunks + chunk;
-            p.part_acc[slot * D + d] = a;
-            if (d == 0) {
-                p.part_ml[slot * 2 + 0] = M;
-                p.part_ml[slot * 2 + 1] = L;
-                if (want_nx) p.part_nx[slot] = N;
-            }
-        }
-    }
-}
-
 // ---------------------------------------------------------------------------
-// Tensor-core decode (head_dim 128).  Both contractions run on tcgen05 with the
+// Tensor-core decode (head_dim 64 and 128).  Both contractions run on tcgen05 with the
 // keys in the M dimension: S^T = K q^T (M = 128 keys of a tile, N = 16 query
 // heads padded, K = D) and O^T += V^T P^T (M = D, N = 16, K = 128 keys, V read
 // MN-major straight from the TMA stage).  Warp 0 streams K/V tiles through a
@@ -413,13 +133,18 @@ __device__ __forceinline__ bool tc_unit(const DecParams &p, int units_x, int u, 
     return w.nkeys > 0;
 }
 
-template <int GT>
+// D = 64 or 128.  The stage layout is the D = 128 one: at D = 64 the second
+// 64-column half of each K and V tile is never loaded and stays zero (the ring
+// is zeroed at kernel start), so O^T += V^T P^T keeps M = 128 (its rows 64-127
+// accumulate zeros) and only the S^T MMAs shrink to the first half.
+template <int D, int GT>
 __global__ void __launch_bounds__(kTcThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                  const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK16,
                  const __grid_constant__ CUtensorMap tmV16, const DecParams p, int units_x,
                  int n_units, int *unit_counter) {
-    constexpr int D = 128;
+    static_assert(D == 64 || D == 128, "head_dim 64 or 128");
+    constexpr int kHalves = D / 64;  // 64-column halves loaded per K / V row
     using C = TcCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -568,9 +293,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 const int qb = k & 1;
                 if (k >= 2 && !mbar_wait(&q_empty[qb], ((k >> 1) - 1) & 1, p.status, abort_flag))
                     break;
-                mbar_arrive_expect_tx(&q_full[qb], C::kQBytes);
+                mbar_arrive_expect_tx(&q_full[qb], kHalves * (kTcN * 128));
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh)
+                for (int hh = 0; hh < kHalves; ++hh)
                     tma_load_4d(q_s + qb * C::kQBytes + hh * (kTcN * 128), &tmQ, &q_full[qb],
                                 hh * 64, w.kvh * G, w.b, w.layer);
                 for (int t = 0; t < w.ntiles; ++t, ++T) {
@@ -585,9 +310,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                     const int r = w.row0 + t * kTcKeys;
                     const int rem = w.nkeys - t * kTcKeys;
                     if (rem >= kTcKeys) {
-                        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+                        mbar_arrive_expect_tx(&full[s], 2 * kHalves * (kTcKeys * 128));
 #pragma unroll
-                        for (int hh = 0; hh < 2; ++hh) {
+                        for (int hh = 0; hh < kHalves; ++hh) {
                             tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], hh * 64, w.kvh,
                                         r, w.layer);
                             tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], hh * 64, w.kvh,
@@ -598,10 +323,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                         // (the rows past them keep older data; the softmax masks
                         // their scores and zeroes their V rows)
                         const int nb = (rem + 15) / 16;
-                        mbar_arrive_expect_tx(&full[s], nb * 4 * (16 * 128));
+                        mbar_arrive_expect_tx(&full[s], nb * 2 * kHalves * (16 * 128));
                         for (int j = 0; j < nb; ++j)
 #pragma unroll
-                            for (int hh = 0; hh < 2; ++hh) {
+                            for (int hh = 0; hh < kHalves; ++hh) {
                                 tma_load_4d(kd + hh * (kTcKeys * 128) + j * (16 * 128), &tmK16,
                                             &full[s], hh * 64, w.kvh, r + 16 * j, w.layer);
                                 tma_load_4d(vd + hh * (kTcKeys * 128) + j * (16 * 128), &tmV16,
@@ -620,7 +345,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kTcKeys, kTcN, 0, 0);
-            constexpr uint32_t idPV = idesc_bf16_f32(D, kTcN, 0, 1);
+            constexpr uint32_t idPV = idesc_bf16_f32(128, kTcN, 0, 1);  // M = 128 at D = 64 too
             const uint32_t base = smem_u32(smem), q_base = smem_u32(q_s), p_addr = smem_u32(P_s);
             // S^T of global tile T (unit number k, its tile t) from q buffer k % 2
             auto issue_s = [&](int T, int k, int t, int nt) -> bool {
@@ -762,12 +487,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 if (n_chunks == 1) {
                     uint16_t *op =
                         p.O + w.layer * p.o_ls + ((int64_t)w.b * p.Hq + (int64_t)w.kvh * G + g) * D;
-                    op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
+                    if (r < D) op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
                     if (r == 0 && p.lse != nullptr) p.lse[unit0 + g] = (m[g] + __log2f(L)) * kLn2;
                     if (r == 0 && want_nx) p.nexus_mass[unit0 + g] = Ng[g] / L;
                 } else {
                     const int64_t slot = (unit0 + g) * p.max_chunks + w.chunk;
-                    p.part_acc[slot * D + r] = a;
+                    if (r < D) p.part_acc[slot * D + r] = a;
                     if (r == 0) {
                         p.part_ml[slot * 2 + 0] = m[g];
                         p.part_ml[slot * 2 + 1] = L;
@@ -994,7 +719,7 @@ Plan make_plan(const sonic_decode_args *a) {
     Plan pl{};
     const int max_len = a->max_len > 0 ? a->max_len : 1;
     // explicit split lengths are rounded up to the kernel's key tile
-    const int tile = a->head_dim == 128 ? kTcKeys : kTileKeys;
+    const int tile = kTcKeys;
     const long long c0 = a->chunk_len < max_len ? a->chunk_len : max_len;
     int C = (int)((c0 + tile - 1) / tile * tile);
     if (C <= 0) {
@@ -1014,21 +739,8 @@ Plan make_plan(const sonic_decode_args *a) {
         if (a->nexus_mass != nullptr)
             pl.ws_nx = round_up(units_q * pl.max_chunks * sizeof(float), 256);
     }
-    if (a->head_dim == 128) pl.ws_cnt = 256;  // the persistent kernel's unit counter
+    pl.ws_cnt = 256;  // the persistent kernel's unit counter
     return pl;
-}
-
-template <int D, int GT>
-cudaError_t launch_split(const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
-                         dim3 grid, cudaStream_t stream) {
-    constexpr size_t smem = dec_smem_bytes<D, GT>();
-    static_assert(smem <= 232448, "decode shared memory");
-    auto kern = decode_split_kernel<D, GT>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    kern<<<grid, kDecThreads, smem, stream>>>(tk, tv, p);
-    return cudaGetLastError();
 }
 
 // Persistent launch: one block per SM (the stage ring takes most of shared
@@ -1037,12 +749,12 @@ struct TcMaps {
     CUtensorMap k, v, q, k16, v16;
 };
 
-template <int GT>
+template <int D, int GT>
 cudaError_t launch_tc(const TcMaps &m, const DecParams &p, int units_x, int n_units, int *counter,
                       cudaStream_t stream) {
     constexpr size_t smem = TcCfg::kSmem;
     static_assert(smem <= 232448, "decode shared memory");
-    auto kern = decode_tc_kernel<GT>;
+    auto kern = decode_tc_kernel<D, GT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
@@ -1055,32 +767,20 @@ cudaError_t launch_tc(const TcMaps &m, const DecParams &p, int units_x, int n_un
     return cudaGetLastError();
 }
 
+template <int D>
 cudaError_t dispatch_tc(int GT, const TcMaps &m, const DecParams &p, int units_x, int n_units,
                         int *counter, cudaStream_t s) {
     switch (GT) {
-        case 1: return launch_tc<1>(m, p, units_x, n_units, counter, s);
-        case 2: return launch_tc<2>(m, p, units_x, n_units, counter, s);
-        case 4: return launch_tc<4>(m, p, units_x, n_units, counter, s);
-        case 7: return launch_tc<7>(m, p, units_x, n_units, counter, s);
-        case 8: return launch_tc<8>(m, p, units_x, n_units, counter, s);
-        case 16: return launch_tc<16>(m, p, units_x, n_units, counter, s);
+        case 1: return launch_tc<D, 1>(m, p, units_x, n_units, counter, s);
+        case 2: return launch_tc<D, 2>(m, p, units_x, n_units, counter, s);
+        case 4: return launch_tc<D, 4>(m, p, units_x, n_units, counter, s);
+        case 7: return launch_tc<D, 7>(m, p, units_x, n_units, counter, s);
+        case 8: return launch_tc<D, 8>(m, p, units_x, n_units, counter, s);
+        case 16: return launch_tc<D, 16>(m, p, units_x, n_units, counter, s);
     }
     return cudaErrorInvalidValue;
 }
 
-template <int D>
-cudaError_t dispatch_g(int GT, const CUtensorMap &tk, const CUtensorMap &tv, const DecParams &p,
-                       dim3 grid, cudaStream_t s) {
-    switch (GT) {
-        case 1: return launch_split<D, 1>(tk, tv, p, grid, s);
-        case 2: return launch_split<D, 2>(tk, tv, p, grid, s);
-        case 4: return launch_split<D, 4>(tk, tv, p, grid, s);
-        case 7: return launch_split<D, 7>(tk, tv, p, grid, s);
-        case 8: return launch_split<D, 8>(tk, tv, p, grid, s);
-        case 16: return launch_split<D, 16>(tk, tv, p, grid, s);
-    }
-    return cudaErrorInvalidValue;
-}
 
 }  // namespace
 }  // namespace sonic
@@ -1133,7 +833,7 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
     const long long units_x = (long long)pl.max_chunks * a->n_heads_kv;
-    if ((D == 64 && (long long)a->batch * a->n_layers > 65535) || units_x > 0x7fffffffLL ||
+    if (units_x > 0x7fffffffLL ||
         units_x * a->batch * a->n_layers > 0x7fffffffLL)
         return SONIC_ERR_UNSUPPORTED;
 
@@ -1143,13 +843,13 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const uint64_t dims[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_kv_rows,
                               (uint64_t)a->n_layers};
     const uint64_t strides[3] = {(uint64_t)D * 2, row_elems * 2, layer_bytes};
-    const uint32_t box[4] = {64, 1, (uint32_t)(D == 128 ? kTcKeys : kTileKeys), 1};
+    const uint32_t box[4] = {64, 1, (uint32_t)kTcKeys, 1};
     CUtensorMap tk, tv;
     TcMaps tm{};
     if (!make_tmap_bf16_4d(&tk, K_ret, dims, strides, box) ||
         !make_tmap_bf16_4d(&tv, V_ret, dims, strides, box))
         return SONIC_ERR_INVALID_ARGUMENT;
-    if (D == 128) {
+    {
         tm.k = tk;
         tm.v = tv;
         const uint32_t box16[4] = {64, 1, 16, 1};
@@ -1190,12 +890,11 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
     p.scale_log2 = scale * kLog2e;
 
-    dim3 grid((unsigned)units_x, a->batch * a->n_layers);
     int *counter = reinterpret_cast<int *>(static_cast<char *>(a->workspace) + pl.ws_acc +
                                            pl.ws_ml + pl.ws_nx);
-    cudaError_t e = (D == 128) ? dispatch_tc(GT, tm, p, (int)units_x,
-                                             (int)(units_x * a->batch * a->n_layers), counter, stream)
-                               : dispatch_g<64>(GT, tk, tv, p, grid, stream);
+    const int n_units = (int)(units_x * a->batch * a->n_layers);
+    cudaError_t e = (D == 128) ? dispatch_tc<128>(GT, tm, p, (int)units_x, n_units, counter, stream)
+                               : dispatch_tc<64>(GT, tm, p, (int)units_x, n_units, counter, stream);
     if (e != cudaSuccess) return SONIC_ERR_CUDA;
     const long long units = (long long)a->n_layers * a->batch * a->n_heads_q;
     const unsigned cblocks = (unsigned)((units * 32 + 127) / 128);
