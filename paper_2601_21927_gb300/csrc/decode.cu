@@ -133,18 +133,27 @@ __device__ __forceinline__ bool tc_unit(const DecParams &p, int units_x, int u, 
     return w.nkeys > 0;
 }
 
-// D = 64 or 128.  The stage layout is the D = 128 one: at D = 64 the second
-// 64-column half of each K and V tile is never loaded and stays zero (the ring
-// is zeroed at kernel start), so O^T += V^T P^T keeps M = 128 (its rows 64-127
-// accumulate zeros) and only the S^T MMAs shrink to the first half.
-template <int D, int GT>
+// D = 64 or 128.  The stage layout is the D = 128 one.  At D = 64 either the
+// second 64-column half of each K and V tile is never loaded and stays zero
+// (the ring is zeroed at kernel start), or (kPair, when G <= 8) a unit takes
+// two KV heads: head 2i's rows fill the first half and head 2i+1's the second,
+// the 16 staged query heads hold both heads' G queries, and S^T and O^T get a
+// region per KV head (query column v belongs to head 2i for v < G, to head
+// 2i+1 after), so a 128-key tile carries as many bytes as at D = 128 for the
+// same per-tile softmax work.  O^T += V^T P^T keeps M = 128 either way (rows
+// 64-127 accumulate zeros, or the other half's data; they are never written).
+template <int D, int GT, bool kPair>
 __global__ void __launch_bounds__(kTcThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                  const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK16,
                  const __grid_constant__ CUtensorMap tmV16, const DecParams p, int units_x,
                  int n_units, int *unit_counter) {
     static_assert(D == 64 || D == 128, "head_dim 64 or 128");
-    constexpr int kHalves = D / 64;  // 64-column halves loaded per K / V row
+    static_assert(!kPair || D == 64, "KV-head pairs at head_dim 64 only");
+    constexpr int kHalves = D / 64;            // 64-column halves per K / V row
+    constexpr int kLoads = kPair ? 2 : kHalves;  // 64-column boxes per K / V tile
+    constexpr int kSStride = kPair ? 2 * kTcN : kTcN;  // TMEM columns of one S^T / O^T buffer
+    constexpr uint32_t kTmemCols = kPair ? 128 : 64;
     using C = TcCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -227,7 +236,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 64);
+        tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), kTmemCols);
         tmem_relinquish();
     }
     fence_proxy_async_smem();
@@ -235,8 +244,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
-    // TMEM: S^T [2] at columns 0 / 16, O^T [2] at 32 / 48
-    const uint32_t tS = tmem, tO = tmem + 32;
+    // TMEM: S^T [2] then O^T [2], kSStride columns each (a 16-column region
+    // per KV head of the unit)
+    const uint32_t tS = tmem, tO = tmem + 2 * kSStride;
+    const int Gv = kPair ? 2 * G : G;  // query columns of a unit
     // The k-th claimed unit (w.u = -1: none left, or a wait gave up), from
     // shared memory: the consumers never touch global memory for it.  Each
     // reader (the issuer, lane 0 of each softmax warp) frees the slot.
@@ -293,11 +304,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 const int qb = k & 1;
                 if (k >= 2 && !mbar_wait(&q_empty[qb], ((k >> 1) - 1) & 1, p.status, abort_flag))
                     break;
+                const int kvh0 = kPair ? 2 * w.kvh : w.kvh;  // first KV head of the unit
                 mbar_arrive_expect_tx(&q_full[qb], kHalves * (kTcN * 128));
 #pragma unroll
                 for (int hh = 0; hh < kHalves; ++hh)
                     tma_load_4d(q_s + qb * C::kQBytes + hh * (kTcN * 128), &tmQ, &q_full[qb],
-                                hh * 64, w.kvh * G, w.b, w.layer);
+                                hh * 64, kvh0 * G, w.b, w.layer);
                 for (int t = 0; t < w.ntiles; ++t, ++T) {
                     const int s = T % kTcStages;
                     if (T >= kTcStages &&
@@ -310,27 +322,29 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                     const int r = w.row0 + t * kTcKeys;
                     const int rem = w.nkeys - t * kTcKeys;
                     if (rem >= kTcKeys) {
-                        mbar_arrive_expect_tx(&full[s], 2 * kHalves * (kTcKeys * 128));
+                        mbar_arrive_expect_tx(&full[s], 2 * kLoads * (kTcKeys * 128));
 #pragma unroll
-                        for (int hh = 0; hh < kHalves; ++hh) {
-                            tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], hh * 64, w.kvh,
-                                        r, w.layer);
-                            tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], hh * 64, w.kvh,
-                                        r, w.layer);
+                        for (int hh = 0; hh < kLoads; ++hh) {
+                            const int dc = kPair ? 0 : hh * 64, hc = kPair ? kvh0 + hh : kvh0;
+                            tma_load_4d(kd + hh * (kTcKeys * 128), &tmK, &full[s], dc, hc, r,
+                                        w.layer);
+                            tma_load_4d(vd + hh * (kTcKeys * 128), &tmV, &full[s], dc, hc, r,
+                                        w.layer);
                         }
                     } else {
                         // a unit's last, partial tile: only its rows, in 16-row boxes
                         // (the rows past them keep older data; the softmax masks
                         // their scores and zeroes their V rows)
                         const int nb = (rem + 15) / 16;
-                        mbar_arrive_expect_tx(&full[s], nb * 2 * kHalves * (16 * 128));
+                        mbar_arrive_expect_tx(&full[s], nb * 2 * kLoads * (16 * 128));
                         for (int j = 0; j < nb; ++j)
 #pragma unroll
-                            for (int hh = 0; hh < kHalves; ++hh) {
+                            for (int hh = 0; hh < kLoads; ++hh) {
+                                const int dc = kPair ? 0 : hh * 64, hc = kPair ? kvh0 + hh : kvh0;
                                 tma_load_4d(kd + hh * (kTcKeys * 128) + j * (16 * 128), &tmK16,
-                                            &full[s], hh * 64, w.kvh, r + 16 * j, w.layer);
+                                            &full[s], dc, hc, r + 16 * j, w.layer);
                                 tma_load_4d(vd + hh * (kTcKeys * 128) + j * (16 * 128), &tmV16,
-                                            &full[s], hh * 64, w.kvh, r + 16 * j, w.layer);
+                                            &full[s], dc, hc, r + 16 * j, w.layer);
                             }
                     }
                 }
@@ -357,13 +371,27 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 tc_fence_after();
                 const uint32_t k_addr = base + (T % kTcStages) * C::kStageBytes;
                 const uint32_t q_addr = q_base + (k % C::kQBufs) * C::kQBytes;
+                const uint32_t sbuf = tS + (T & 1) * kSStride;
+                if (kPair) {
+                    // one S^T region per KV head: its K half against all staged queries
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint64_t a = smem_desc_sw128(
-                        k_addr + (kk >> 2) * (kTcKeys * 128) + (kk & 3) * 32, 16, 1024);
-                    const uint64_t bd =
-                        smem_desc_sw128(q_addr + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
-                    tc_mma_ss(tS + (T & 1) * kTcN, a, bd, idS, kk > 0 ? 1u : 0u);
+                    for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc_mma_ss(sbuf + hh * kTcN,
+                                      smem_desc_sw128(k_addr + hh * (kTcKeys * 128) + kk * 32, 16,
+                                                      1024),
+                                      smem_desc_sw128(q_addr + kk * 32, 16, 1024), idS,
+                                      kk > 0 ? 1u : 0u);
+                } else {
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        const uint64_t a = smem_desc_sw128(
+                            k_addr + (kk >> 2) * (kTcKeys * 128) + (kk & 3) * 32, 16, 1024);
+                        const uint64_t bd = smem_desc_sw128(
+                            q_addr + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
+                        tc_mma_ss(sbuf, a, bd, idS, kk > 0 ? 1u : 0u);
+                    }
                 }
                 tc_commit(&s_full[T & 1]);
                 if (t == nt - 1) tc_commit(&q_empty[k % C::kQBufs]);
@@ -417,13 +445,16 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                     const uint32_t v_addr = base + (T % kTcStages) * C::kStageBytes + C::kTileBytes;
                     const uint32_t pb = p_addr + (T & 1) * C::kPBytes;
 #pragma unroll
-                    for (int kk = 0; kk < kTcKeys / 16; ++kk) {
-                        const uint64_t a =
-                            smem_desc_sw128(v_addr + kk * (16 * 128), kTcKeys * 128, 1024);
-                        const uint64_t bd =
-                            smem_desc_sw128(pb + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
-                        tc_mma_ss(tO + (k & 1) * kTcN, a, bd, idPV, (t > 0 || kk > 0) ? 1u : 0u);
-                    }
+                    for (int hh = 0; hh < (kPair ? 2 : 1); ++hh)
+#pragma unroll
+                        for (int kk = 0; kk < kTcKeys / 16; ++kk) {
+                            const uint64_t a = smem_desc_sw128(
+                                v_addr + hh * (kTcKeys * 128) + kk * (16 * 128), kTcKeys * 128, 1024);
+                            const uint64_t bd = smem_desc_sw128(
+                                pb + (kk >> 2) * (kTcN * 128) + (kk & 3) * 32, 16, 1024);
+                            tc_mma_ss(tO + (k & 1) * kSStride + hh * kTcN, a, bd, idPV,
+                                      (t > 0 || kk > 0) ? 1u : 0u);
+                        }
                     tc_commit(o_done);
                     tc_commit(&empty[T % kTcStages]);
                     if (t == w.ntiles - 1) tc_commit(&o_last[k & 1]);
@@ -446,7 +477,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         const bool want_nx = p.nexus_mass != nullptr;
         auto epilogue = [&](const TcUnit &w, int k, const float (&m)[GT], const float (&l)[GT],
                             const float (&n)[GT]) -> bool {
-            const uint32_t tOk = tO + (k & 1) * kTcN;
+            const uint32_t tOk = tO + (k & 1) * kSStride;
             if (!mbar_wait(&o_last[k & 1], (k >> 1) & 1, p.status, abort_flag)) return false;
             tc_fence_after();
 #pragma unroll
@@ -466,6 +497,15 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             if (!mbar_wait(ep_sync, k & 1, p.status, abort_flag)) return false;
             uint32_t o[16];
             tmem_ld16(tOk + lane_base, o);
+            if (kPair) {  // query columns v >= G: the second KV head's region
+                uint32_t ob[16];
+                tmem_ld16(tOk + lane_base + kTcN, ob);
+                tmem_ld_wait();
+                reg_fence16(ob);
+#pragma unroll
+                for (int g = 0; g < 16; ++g)
+                    if (g >= G) o[g] = ob[g];
+            }
             tmem_ld_wait();
             reg_fence16(o);
             float Lg[GT], Ng[GT];
@@ -478,15 +518,16 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             tc_fence_before();
             mbar_arrive(&o_free[k & 1]);
             const int n_chunks = (w.len + p.chunk_len - 1) / p.chunk_len;
-            const int64_t unit0 = ((int64_t)w.layer * p.B + w.b) * p.Hq + (int64_t)w.kvh * G;
+            const int hb = (kPair ? 2 * w.kvh : w.kvh) * G;  // the unit's first query head
+            const int64_t unit0 = ((int64_t)w.layer * p.B + w.b) * p.Hq + hb;
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
-                if (g >= G) break;
+                if (g >= Gv) break;
                 const float L = Lg[g];
                 const float a = __uint_as_float(o[g]);
                 if (n_chunks == 1) {
                     uint16_t *op =
-                        p.O + w.layer * p.o_ls + ((int64_t)w.b * p.Hq + (int64_t)w.kvh * G + g) * D;
+                        p.O + w.layer * p.o_ls + ((int64_t)w.b * p.Hq + hb + g) * D;
                     if (r < D) op[r] = __bfloat16_as_ushort(__float2bfloat16_rn(a / L));
                     if (r == 0 && p.lse != nullptr) p.lse[unit0 + g] = (m[g] + __log2f(L)) * kLn2;
                     if (r == 0 && want_nx) p.nexus_mass[unit0 + g] = Ng[g] / L;
@@ -515,7 +556,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
             w.row0 = __shfl_sync(0xffffffffu, w.row0, 0);
             w.len = __shfl_sync(0xffffffffu, w.len, 0);
             tc_coords(p, units_x, w);
-            const uint32_t tOk = tO + (k & 1) * kTcN;
+            const uint32_t tOk = tO + (k & 1) * kSStride;
             float m[GT], l[GT], n[GT];
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
@@ -534,7 +575,16 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 }
                 tc_fence_after();
                 uint32_t sr[16];
-                tmem_ld16(tS + lane_base + (T & 1) * kTcN, sr);
+                tmem_ld16(tS + lane_base + (T & 1) * kSStride, sr);
+                if (kPair) {  // query columns v >= G: the second KV head's region
+                    uint32_t sb[16];
+                    tmem_ld16(tS + lane_base + (T & 1) * kSStride + kTcN, sb);
+                    tmem_ld_wait();
+                    reg_fence16(sb);
+#pragma unroll
+                    for (int g = 0; g < 16; ++g)
+                        if (g >= G) sr[g] = sb[g];
+                }
                 tmem_ld_wait();
                 reg_fence16(sr);
                 const bool valid = in_unit;
@@ -598,14 +648,17 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                         break;
                     }
                     tc_fence_after();
-                    uint32_t o[16];
-                    tmem_ld16(tOk + lane_base, o);
-                    tmem_ld_wait();
-                    reg_fence16(o);
 #pragma unroll
-                    for (int g = 0; g < GT; ++g)
-                        o[g] = __float_as_uint(__uint_as_float(o[g]) * alpha[g]);
-                    tmem_st16(tOk + lane_base, o);
+                    for (int hh = 0; hh < (kPair ? 2 : 1); ++hh) {
+                        uint32_t o[16];
+                        tmem_ld16(tOk + lane_base + hh * kTcN, o);
+                        tmem_ld_wait();
+                        reg_fence16(o);
+#pragma unroll
+                        for (int g = 0; g < GT; ++g)
+                            o[g] = __float_as_uint(__uint_as_float(o[g]) * alpha[g]);
+                        tmem_st16(tOk + lane_base + hh * kTcN, o);
+                    }
                     tmem_st_wait();
                 }
                 fence_proxy_async_smem();
@@ -633,7 +686,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, 64);
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
 // One warp per (layer, sequence, query head).
@@ -715,15 +768,23 @@ struct Plan {
     size_t total() const { return ws_acc + ws_ml + ws_nx + ws_cnt; }
 };
 
+// head_dim 64 with G <= 8 and an even number of KV heads: units of two KV heads.
+bool use_pairs(const sonic_decode_args *a) {
+    if (a->n_heads_kv <= 0 || a->n_heads_q % a->n_heads_kv != 0) return false;
+    const int G = a->n_heads_q / a->n_heads_kv;
+    return a->head_dim == 64 && G <= 8 && a->n_heads_kv % 2 == 0;
+}
+
 Plan make_plan(const sonic_decode_args *a) {
     Plan pl{};
+    const int kv_units = a->n_heads_kv / (use_pairs(a) ? 2 : 1);  // KV heads (or pairs) per unit row
     const int max_len = a->max_len > 0 ? a->max_len : 1;
     // explicit split lengths are rounded up to the kernel's key tile
     const int tile = kTcKeys;
     const long long c0 = a->chunk_len < max_len ? a->chunk_len : max_len;
     int C = (int)((c0 + tile - 1) / tile * tile);
     if (C <= 0) {
-        const long long units = (long long)a->batch * a->n_heads_kv * a->n_layers;
+        const long long units = (long long)a->batch * kv_units * a->n_layers;
         const long long target = 4LL * device_sm_count();
         long long splits = units >= target ? 1 : (target + units - 1) / units;
         long long c = (max_len + splits - 1) / splits;
@@ -749,12 +810,12 @@ struct TcMaps {
     CUtensorMap k, v, q, k16, v16;
 };
 
-template <int D, int GT>
+template <int D, int GT, bool kPair>
 cudaError_t launch_tc(const TcMaps &m, const DecParams &p, int units_x, int n_units, int *counter,
                       cudaStream_t stream) {
     constexpr size_t smem = TcCfg::kSmem;
     static_assert(smem <= 232448, "decode shared memory");
-    auto kern = decode_tc_kernel<D, GT>;
+    auto kern = decode_tc_kernel<D, GT, kPair>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
@@ -767,19 +828,20 @@ cudaError_t launch_tc(const TcMaps &m, const DecParams &p, int units_x, int n_un
     return cudaGetLastError();
 }
 
-template <int D>
+template <int D, bool kPair>
 cudaError_t dispatch_tc(int GT, const TcMaps &m, const DecParams &p, int units_x, int n_units,
                         int *counter, cudaStream_t s) {
     switch (GT) {
-        case 1: return launch_tc<D, 1>(m, p, units_x, n_units, counter, s);
-        case 2: return launch_tc<D, 2>(m, p, units_x, n_units, counter, s);
-        case 4: return launch_tc<D, 4>(m, p, units_x, n_units, counter, s);
-        case 7: return launch_tc<D, 7>(m, p, units_x, n_units, counter, s);
-        case 8: return launch_tc<D, 8>(m, p, units_x, n_units, counter, s);
-        case 16: return launch_tc<D, 16>(m, p, units_x, n_units, counter, s);
+        case 1: return launch_tc<D, 1, kPair>(m, p, units_x, n_units, counter, s);
+        case 2: return launch_tc<D, 2, kPair>(m, p, units_x, n_units, counter, s);
+        case 4: return launch_tc<D, 4, kPair>(m, p, units_x, n_units, counter, s);
+        case 7: return launch_tc<D, 7, kPair>(m, p, units_x, n_units, counter, s);
+        case 8: return launch_tc<D, 8, kPair>(m, p, units_x, n_units, counter, s);
+        case 16: return launch_tc<D, 16, kPair>(m, p, units_x, n_units, counter, s);
     }
     return cudaErrorInvalidValue;
 }
+
 
 
 }  // namespace
@@ -832,7 +894,8 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     const size_t need = pl.total();
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
-    const long long units_x = (long long)pl.max_chunks * a->n_heads_kv;
+    const bool pairs = use_pairs(a);
+    const long long units_x = (long long)pl.max_chunks * (a->n_heads_kv / (pairs ? 2 : 1));
     if (units_x > 0x7fffffffLL ||
         units_x * a->batch * a->n_layers > 0x7fffffffLL)
         return SONIC_ERR_UNSUPPORTED;
@@ -881,7 +944,7 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     p.status = a->status;
     p.B = a->batch;
     p.Hq = a->n_heads_q;
-    p.Hkv = a->n_heads_kv;
+    p.Hkv = a->n_heads_kv / (pairs ? 2 : 1);  // units per (chunk, sequence, layer)
     p.G = G;
     p.q_ls = a->q_layer_stride;
     p.o_ls = a->o_layer_stride;
@@ -893,8 +956,11 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     int *counter = reinterpret_cast<int *>(static_cast<char *>(a->workspace) + pl.ws_acc +
                                            pl.ws_ml + pl.ws_nx);
     const int n_units = (int)(units_x * a->batch * a->n_layers);
-    cudaError_t e = (D == 128) ? dispatch_tc<128>(GT, tm, p, (int)units_x, n_units, counter, stream)
-                               : dispatch_tc<64>(GT, tm, p, (int)units_x, n_units, counter, stream);
+    cudaError_t e =
+        D == 128 ? dispatch_tc<128, false>(GT, tm, p, (int)units_x, n_units, counter, stream)
+        : pairs  ? dispatch_tc<64, true>(g_template(2 * G), tm, p, (int)units_x, n_units, counter,
+                                         stream)
+                 : dispatch_tc<64, false>(GT, tm, p, (int)units_x, n_units, counter, stream);
     if (e != cudaSuccess) return SONIC_ERR_CUDA;
     const long long units = (long long)a->n_layers * a->batch * a->n_heads_q;
     const unsigned cblocks = (unsigned)((units * 32 + 127) / 128);

@@ -81,7 +81,8 @@ def test_ragged_lengths_and_splits(chunk_len):
 
 
 @pytest.mark.parametrize("hq,hkv,D", [(28, 4, 128), (2, 1, 64), (16, 16, 128), (32, 2, 64),
-                                      (12, 4, 128)])
+                                      (12, 4, 128), (16, 4, 64), (14, 2, 64), (8, 8, 64),
+                                      (12, 6, 64), (9, 3, 64)])
 def test_head_shapes(hq, hkv, D):
     lens = [300, 1777, 4096]
     r = _decode(lens, hq, hkv, D, n_layers=1, seed=hq + D)
