@@ -595,6 +595,45 @@ def extra_masked_prefill():
             "results": res}
 
 
+def extra_prefill_d64():
+    """The masked-prefill workload (batch 8 x 5632 rows, every row a query, full
+    mask, retained-first key order; and the current-turn rows alone) at
+    head_dim 64 with 32/8 heads, beside head_dim 128."""
+    import torch
+    from paper_2601_21927_gb300 import inputs, sonic
+    dev = torch.device("cuda", 0)
+    batch, _ = inputs.masked_prefill()
+    d = batch.dialogues[0]
+    role, seg = d.arrays()
+    L = d.length
+    t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
+    r_, s_, ks, kl = t(batch.role), t(batch.seg), t(batch.k_start), t(batch.k_len)
+    ql = np.full(batch.B, d.curr_len, np.int32)
+    qs = np.concatenate([[0], np.cumsum(ql)[:-1]]).astype(np.int32)
+    res = {}
+    for D in (64, 128):
+        K = inputs.randn((1, batch.total, 8, D), seed=1, device=dev)
+        V = inputs.randn((1, batch.total, 8, D), seed=2, device=dev)
+        Q = inputs.randn((1, batch.total, 32, D), seed=3, device=dev)
+        O = torch.empty_like(Q)
+        flops = 4.0 * D * 32 * _visible_pairs(role, seg, range(L), 0) * batch.B
+        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+            Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks, q_len=kl, max_q_len=L,
+            max_k_len=L, key_order=1))
+        res[f"all_rows_retained_first_d{D}"] = {"ms": round(ms, 3),
+                                                "tflops": round(flops / ms / 1e9, 1)}
+        Qc = inputs.randn((1, int(ql.sum()), 32, D), seed=4, device=dev)
+        Oc = torch.empty_like(Qc)
+        flops = 4.0 * D * 32 * _visible_pairs(role, seg, range(L - d.curr_len, L), 0) * batch.B
+        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=t(qs), q_len=t(ql),
+            max_q_len=int(ql.max()), max_k_len=L, key_order=1))
+        res[f"current_rows_retained_first_d{D}"] = {"ms": round(ms, 3),
+                                                    "tflops": round(flops / ms / 1e9, 1)}
+    return {"workload": "masked prefill, batch 8 x 5632 rows, 32/8 heads, head_dim 64 and 128",
+            "results": res}
+
+
 def extra_decode():
     """Decode over retained caches: Llama-3-8B-like (batch 16, 32 layers, 32/8
     heads, 641 retained rows) and 64 long ragged dialogues with Nexus =
@@ -911,7 +950,7 @@ def extra_routed():
 
 EXTRAS = {"masked_prefill": extra_masked_prefill, "decode": extra_decode,
           "nexus_mass": extra_nexus_mass, "routed": extra_routed, "compaction": extra_compaction,
-          "decode_graph": extra_decode_graph,
+          "decode_graph": extra_decode_graph, "prefill_d64": extra_prefill_d64,
           "context": extra_context, "nexus_gen": extra_nexus_gen}
 
 
