@@ -51,7 +51,7 @@
 extern "C" {
 #endif
 
-#define SONIC_ABI_VERSION 2
+#define SONIC_ABI_VERSION 3
 
 #if defined(__GNUC__)
 #define SONIC_API __attribute__((visibility("default")))
@@ -327,6 +327,8 @@ typedef struct {
     int64_t row_stride;          /* elements between rows of base; multiple of 8, >= cols */
     int32_t cols;                /* > 0, multiple of 32                                 */
     int32_t scatter;             /* 0: row t of Y goes to row t; 1: to row dst_row[t]   */
+    int64_t rows;                /* rows of base: a row index outside [0, rows) is not
+                                    written and sets SONIC_ERR_CAPACITY in *status      */
 } sonic_out_part;
 
 typedef struct {

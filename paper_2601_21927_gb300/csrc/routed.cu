@@ -161,6 +161,7 @@ row_gather_kernel(const uint8_t *__restrict__ X, int64_t x_row_bytes, int32_t T,
 struct GemmPart {
     uint16_t *base;
     int64_t stride;  // elements between rows
+    int64_t rows;    // rows of base
     int col0, cols;
     int scatter;
 };
@@ -438,6 +439,10 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     if (q < p.n_parts && col >= p.part[q].col0) k = q;
                 const GemmPart &pt = p.part[k];
                 const int64_t row = pt.scatter ? dst : t;
+                if (row < 0 || row >= pt.rows) {  // outside the part: not written
+                    set_status(p.status, SONIC_ERR_CAPACITY);
+                    continue;
+                }
                 uint4 *out = reinterpret_cast<uint4 *>(pt.base + row * pt.stride + (col - pt.col0));
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
@@ -504,10 +509,11 @@ extern "C" sonic_status_t sonic_routed_linear(const uint16_t *X, const uint16_t 
     for (int k = 0; k < a->n_parts; ++k) {
         const sonic_out_part &q = a->parts[k];
         if (q.base == nullptr || !aligned16(q.base) || q.cols <= 0 || q.cols % 32 != 0 ||
-            q.row_stride < q.cols || q.row_stride % 8 != 0)
+            q.row_stride < q.cols || q.row_stride % 8 != 0 || q.rows <= 0)
             return SONIC_ERR_INVALID_ARGUMENT;
         if (q.scatter && a->dst_row == nullptr) return SONIC_ERR_INVALID_ARGUMENT;
-        p.part[k] = GemmPart{static_cast<uint16_t *>(q.base), q.row_stride, col, q.cols,
+        if (!q.scatter && q.rows < a->n_rows) return SONIC_ERR_INVALID_ARGUMENT;
+        p.part[k] = GemmPart{static_cast<uint16_t *>(q.base), q.row_stride, q.rows, col, q.cols,
                              q.scatter ? 1 : 0};
         col += q.cols;
     }

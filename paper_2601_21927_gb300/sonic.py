@@ -68,7 +68,8 @@ class sonic_decode_args(ctypes.Structure):
 
 
 class sonic_out_part(ctypes.Structure):
-    _fields_ = [("base", _P), ("row_stride", _i64), ("cols", _i32), ("scatter", _i32)]
+    _fields_ = [("base", _P), ("row_stride", _i64), ("cols", _i32), ("scatter", _i32),
+                ("rows", _i64)]
 
 
 class sonic_routed_linear_args(ctypes.Structure):
@@ -261,6 +262,7 @@ def sonic_routed_linear(X: torch.Tensor, W: torch.Tensor, W_nexus: torch.Tensor,
         a.parts[k].row_stride = out.stride(0)
         a.parts[k].cols = out.shape[1]
         a.parts[k].scatter = 1 if scatter else 0
+        a.parts[k].rows = out.shape[0]
     a.status = _ptr(status)
     need = lib.sonic_routed_linear_workspace_size(ctypes.byref(a))
     ws = _workspace(need, X.device, workspace)

@@ -26,7 +26,7 @@ def test_library_exports_every_declared_symbol():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(sonic.SIGNATURES)
-    assert lib.sonic_abi_version() == 2
+    assert lib.sonic_abi_version() == 3
     assert lib.sonic_status_string(4) == b"output capacity exceeded"
 
 
@@ -146,7 +146,7 @@ def test_routed_linear_validation():
     a.n_rows = 0
     assert lib.sonic_routed_linear(None, None, None, None, ctypes.byref(a), None) == 0  # empty
     a.n_rows, a.d_in, a.d_out, a.x_row_stride, a.n_parts = 10, 96, 64, 96, 1  # d_in % 64
-    a.parts[0].base, a.parts[0].row_stride, a.parts[0].cols = 16, 64, 64
+    a.parts[0].base, a.parts[0].row_stride, a.parts[0].cols, a.parts[0].rows = 16, 64, 64, 10
     assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
     a.d_in = a.x_row_stride = 128
     a.parts[0].cols = 48                      # parts must cover d_out in 32-column steps
@@ -155,5 +155,8 @@ def test_routed_linear_validation():
     a.parts[0].scatter = 1                    # scatter without dst_row
     assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
     a.parts[0].scatter = 0
+    a.parts[0].rows = 9                       # fewer rows than X for an unscattered part
+    assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 1
+    a.parts[0].rows = 10
     assert lib.sonic_routed_linear(16, 16, 16, 16, ctypes.byref(a), None) == 3  # no workspace
     assert lib.sonic_routed_linear_workspace_size(ctypes.byref(a)) == 256 + 256 + 256 + 2560

@@ -144,3 +144,24 @@ def test_nexus_generation_projection_sampled_rows():
     r = _run(role, 4096, [4096, 1024, 1024], [False, True, True], seed=11, cache_rows=3000)
     rows = np.unique(np.r_[np.arange(256, 288), np.arange(0, 2304, 37)])
     _check(r, rows)
+
+
+def test_destination_rows_outside_a_part_are_reported():
+    """dst_row values past the cache's rows (or negative) are not written: the
+    status word says SONIC_ERR_CAPACITY and every row inside is still right."""
+    role = _roles(200, 21)
+    T, cache_rows = len(role), 300
+    X = inputs.randn((T, 128), seed=21, device=H.dev())
+    W, Wn = _weights(64, 128, 22), _weights(64, 128, 23)
+    dst = np.random.default_rng(21).permutation(cache_rows)[:T].astype(np.int32)
+    dst[[3, 77]] = [cache_rows + 5, -1]
+    out = torch.full((cache_rows, 64), float("nan"), dtype=torch.bfloat16, device=H.dev())
+    status = torch.zeros(1, dtype=torch.int32, device=H.dev())
+    sonic.sonic_routed_linear(X, W, Wn, torch.from_numpy(role).to(H.dev()), [(out, True)],
+                              dst_row=H.i32(dst), status=status)
+    torch.cuda.synchronize()
+    assert sonic.read_status(status) == 4
+    ok = np.setdiff1d(np.arange(T), [3, 77])
+    want = oracle.routed_linear(H.f64(X), H.f64(W), H.f64(Wn), role)[ok]
+    got = H.f64(out[torch.as_tensor(dst[ok]).long().to(H.dev())])
+    _close(got, want, "rows inside the part")
