@@ -209,8 +209,9 @@ typedef struct {
  * base pointer must be 16-byte aligned.  role and seg_id are indexed like the
  * key rows of one layer (shared by all layers); role 255 marks a row that is
  * no key (padding).  key_order picks the order the key tiles are cut in
- * (sonic_key_order_t).  A sequence with q_len[b] > k_len[b] or k_len[b] >
- * max_k_len is refused with SONIC_ERR_INVALID_ARGUMENT in *status.
+ * (sonic_key_order_t).  A sequence with q_len[b] > k_len[b], k_len[b] >
+ * max_k_len, or rows outside [0, total_k_rows) / [0, total_q_rows) is refused
+ * with SONIC_ERR_INVALID_ARGUMENT in *status (none of its rows is read).
  * nexus_mass (optional) is the per-row, per-head quantity behind A_nexus of
  * the Nexus attention regularisation (Sec. 4.1, Eq. 9):
  *   nexus_mass[i, h] = sum_{q in vis, role[q] = NEXUS} softmax(s)_q
@@ -302,7 +303,9 @@ typedef struct {
  * fits one chunk is written directly).  One persistent block per SM claims
  * units from a counter in the workspace (zeroed on `stream` before the
  * launch), so the workspace is never empty and concurrent calls need
- * workspaces of their own.  lens[b] = 0 gives zeros (and
+ * workspaces of their own.  A sequence whose rows fall outside [0, total_kv_rows) is
+ * refused with SONIC_ERR_INVALID_ARGUMENT in *status (its outputs are left
+ * undefined).  lens[b] = 0 gives zeros (and
  * lse = -inf).  bf16 in/out, fp32 arithmetic.  nexus_mass (optional, role
  * then required, else SONIC_ERR_INVALID_ARGUMENT) is the decode form of the
  * quantity behind A_nexus (Sec. 4.1, Eq. 9): the share of the new token's

@@ -38,6 +38,7 @@ struct DecParams {
     float *part_nx;   // [units][max_chunks]
     int32_t *status;
     int B, Hq, Hkv, G;
+    int64_t total_kv_rows;  // rows of K_ret, V_ret (and role) per layer
     int64_t q_ls, o_ls;
     int chunk_len, max_chunks;
     float scale_log2;
@@ -125,11 +126,17 @@ __device__ __forceinline__ bool tc_unit(const DecParams &p, int units_x, int u, 
     w.layer = y / p.B;
     int len = seq_len != nullptr ? seq_len[w.b] : p.lens[w.b];
     len = min(max(len, 0), p.max_chunks * p.chunk_len);
+    const int start = seq_start != nullptr ? seq_start[w.b] : p.kv_start[w.b];
+    if (start < 0 || (int64_t)start + len > p.total_kv_rows) {
+        // rows outside the cache: the sequence is refused, nothing is read
+        if (w.chunk == 0 && w.kvh == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        len = 0;
+    }
     const int key0 = w.chunk * p.chunk_len;
     w.len = len;
     w.nkeys = max(min(p.chunk_len, len - key0), 0);
     w.ntiles = (w.nkeys + kTcKeys - 1) / kTcKeys;
-    w.row0 = (seq_start != nullptr ? seq_start[w.b] : p.kv_start[w.b]) + key0;
+    w.row0 = start + key0;
     return w.nkeys > 0;
 }
 
@@ -945,6 +952,7 @@ extern "C" sonic_status_t sonic_attn_decode(const uint16_t *q, const uint16_t *K
     p.B = a->batch;
     p.Hq = a->n_heads_q;
     p.Hkv = a->n_heads_kv / (pairs ? 2 : 1);  // units per (chunk, sequence, layer)
+    p.total_kv_rows = a->total_kv_rows;
     p.G = G;
     p.q_ls = a->q_layer_stride;
     p.o_ls = a->o_layer_stride;

@@ -48,13 +48,28 @@ struct TileSum {
 
 // Key rows with role 255 are padding (no key): they count as invalid.
 // `pos` gives each key row's S_aug position (NULL: the row index itself).
+// A k_len outside [0, max_k_len] is refused: the sequence gets no keys.
+__device__ __forceinline__ int checked_len(int len, int max_len) {
+    return (len < 0 || len > max_len) ? 0 : len;
+}
+
+// Rows of sequence (start, len), or 0 when they fall outside [0, total) or
+// past max_len: such a sequence is refused, never read.
+__device__ __forceinline__ int seq_rows(int start, int len, int max_len, int64_t total) {
+    return (start < 0 || (int64_t)start + checked_len(len, max_len) > total) ? 0
+                                                                            : checked_len(len, max_len);
+}
+
 __global__ void __launch_bounds__(128)
 tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                     const int32_t *__restrict__ pos, const int32_t *__restrict__ k_start,
                     const int32_t *__restrict__ k_len, TileSum *__restrict__ out,
-                    int max_k_tiles) {
+                    int max_k_tiles, int64_t total_rows, int32_t *status) {
     const int t = blockIdx.x, b = blockIdx.y;
-    const int len = k_len[b];
+    const int len_in = k_len[b];
+    // a sequence outside the arrays (or longer than the tiles) gets empty summaries
+    const int len = seq_rows(k_start[b], len_in, max_k_tiles * kBN, total_rows);
+    if (t == 0 && threadIdx.x == 0 && len != len_in) set_status(status, SONIC_ERR_INVALID_ARGUMENT);
     if (t * kBN >= len && t > 0) return;
     const int r = t * kBN + threadIdx.x;
     int flags = 0, bmin = INT_MAX, bmax = INT_MIN, nmin = INT_MAX, nmax = INT_MIN, n = 0;
@@ -139,6 +154,7 @@ struct PfParams {
     const TileSum *sums;
     int max_k_tiles, max_k_len;
     int B, Hq, G;
+    int64_t total_k_rows;  // rows of role, seg_id (and K, V) per layer
     int pack_log2;  // query heads per tile row group: a tile is 128 >> pack_log2 rows x (1 << pack_log2) heads
     int64_t o_ls;
     int total_q_rows;
@@ -262,6 +278,12 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     const int qt = blockIdx.x, h0 = blockIdx.y << pl2;
     const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
     const int klen = p.k_len[b], qlen = p.q_len[b];
+    if (p.k_start[b] < 0 || (int64_t)p.k_start[b] + klen > p.total_k_rows || p.q_start[b] < 0 ||
+        qlen < 0 || (int64_t)p.q_start[b] + qlen > p.total_q_rows) {
+        // rows outside the arrays: the sequence is refused, nothing is read
+        if (qt == 0 && threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+        return;
+    }
     if (qt * 2 * R >= qlen || timed_out(p.status)) return;
     // key side (kk*): the rows the tiles are cut from; k*: the S_aug sequence
     const int kklen = p.key_len[b];
@@ -872,15 +894,12 @@ constexpr int kOrderThreads = 1024;
 
 __device__ __forceinline__ int span_of(int len) { return (len + kBN - 1) / kBN * kBN + kBN; }
 
-// A k_len outside [0, max_k_len] is refused: the sequence gets no keys.
-__device__ __forceinline__ int checked_len(int len, int max_len) {
-    return (len < 0 || len > max_len) ? 0 : len;
-}
 
 __global__ void __launch_bounds__(kOrderThreads)
 key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                  const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len, int B,
-                 int max_k_len, int64_t capacity, int32_t *__restrict__ key_start,
+                 int max_k_len, int64_t total_rows, int64_t capacity,
+                 int32_t *__restrict__ key_start,
                  int32_t *__restrict__ key_len, uint8_t *__restrict__ o_role,
                  int32_t *__restrict__ o_seg, int32_t *__restrict__ o_pos,
                  int32_t *__restrict__ o_src, int32_t *__restrict__ status) {
@@ -890,7 +909,8 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     __shared__ int sh_r;
     // start of this sequence's span: the spans of the sequences before it
     long long base = 0;
-    for (int i = tid; i < b; i += kOrderThreads) base += span_of(checked_len(k_len[i], max_k_len));
+    for (int i = tid; i < b; i += kOrderThreads)
+        base += span_of(seq_rows(k_start[i], k_len[i], max_k_len, total_rows));
     if (tid == 0) {
         sh_base = 0;
         sh_r = 0;
@@ -898,9 +918,9 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     __syncthreads();
     if (base) atomicAdd(reinterpret_cast<unsigned long long *>(&sh_base), (unsigned long long)base);
     const int len_in = k_len[b];
-    const int len = checked_len(len_in, max_k_len);
-    if (tid == 0 && len != len_in) set_status(status, SONIC_ERR_INVALID_ARGUMENT);
     const int ks = k_start[b];
+    const int len = seq_rows(ks, len_in, max_k_len, total_rows);
+    if (tid == 0 && len != len_in) set_status(status, SONIC_ERR_INVALID_ARGUMENT);
     int cnt = 0;
     for (int i = tid; i < len; i += kOrderThreads) cnt += role[ks + i] != SONIC_ROLE_BODY;
     cnt = __reduce_add_sync(0xffffffffu, cnt);
@@ -1195,6 +1215,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.B = a->batch;
     p.Hq = a->n_heads_q;
     p.G = G;
+    p.total_k_rows = a->total_k_rows;
     p.pack_log2 = pack_log2;
     p.o_ls = a->o_layer_stride;
     p.total_q_rows = a->total_q_rows;
@@ -1204,7 +1225,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
 
     if (reorder) {
         key_order_kernel<<<a->batch, kOrderThreads, 0, stream>>>(
-            role, seg_id, a->k_start, a->k_len, a->batch, a->max_k_len, ws.rows,
+            role, seg_id, a->k_start, a->k_len, a->batch, a->max_k_len, a->total_k_rows, ws.rows,
             reinterpret_cast<int32_t *>(wsb + ws.key_start),
             reinterpret_cast<int32_t *>(wsb + ws.key_len), wsb + ws.role,
             reinterpret_cast<int32_t *>(wsb + ws.seg), reinterpret_cast<int32_t *>(wsb + ws.pos),
@@ -1219,7 +1240,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     }
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
         p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
-        static_cast<TileSum *>(a->workspace), p.max_k_tiles);
+        static_cast<TileSum *>(a->workspace), p.max_k_tiles,
+        reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status);
     dim3 grid((unsigned)qtiles, a->n_heads_q >> pack_log2, a->batch * a->n_layers);
     cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
                                : launch_prefill<64>(tq, tk, tv, p, grid, stream);

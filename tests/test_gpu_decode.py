@@ -147,3 +147,24 @@ def test_empty_cache_outputs():
                             lse=lse, role=role, nexus_mass=mass)
     torch.cuda.synchronize()
     assert (O == 0).all() and torch.isneginf(lse).all() and (mass == 0).all()
+
+
+def test_sequence_outside_the_cache_is_refused():
+    """kv_start past the cache's rows: the sequence is refused
+    (SONIC_ERR_INVALID_ARGUMENT), the others are computed as usual."""
+    lens = np.array([300, 200, 129], np.int32)
+    starts = np.array([0, 300, 10_000], np.int32)
+    T, nl, hq, hkv, D = 500, 1, 8, 2, 128
+    K = inputs.randn((nl, T, hkv, D), seed=31, device=H.dev())
+    V = inputs.randn((nl, T, hkv, D), seed=32, device=H.dev())
+    q = inputs.randn((nl, 3, hq, D), seed=33, device=H.dev())
+    O = torch.full_like(q, float("nan"))
+    status = torch.zeros(1, dtype=torch.int32, device=H.dev())
+    sonic.sonic_attn_decode(q, K, V, H.i32(lens), O, kv_start=H.i32(starts), max_len=300,
+                            status=status)
+    torch.cuda.synchronize()
+    assert sonic.read_status(status) == 1
+    for b in (0, 1):
+        s0, n = int(starts[b]), int(lens[b])
+        Oref, _ = oracle.decode(H.f64(q[0, b]), H.f64(K[0, s0:s0 + n]), H.f64(V[0, s0:s0 + n]))
+        H.check_close(H.f64(O[0, b]), Oref, f"seq {b}")

@@ -217,3 +217,17 @@ def test_masked_prefill_workload_sampled_rows(order):
     # every output is finite and the lse rows are all written
     assert torch.isfinite(res["O"]).all()
     assert torch.isfinite(res["lse"]).all()
+
+
+@pytest.mark.parametrize("order", ORDERS)
+def test_sequence_outside_the_arrays_is_refused(order):
+    """A sequence whose k_start points past total_k_rows is refused
+    (SONIC_ERR_INVALID_ARGUMENT in the status word, none of its rows read);
+    the other sequences are computed as usual."""
+    ds = [inputs.Dialogue(20, [(60, 10)], 40), inputs.Dialogue(30, [(100, 20), (50, 5)], 70)]
+    batch = inputs.Batch(ds)
+    bad_start = [int(batch.k_start[0]), batch.total + 1000]
+    res = H.run_prefill(batch, 4, 2, 128, seed=61, key_order=order, k_start=bad_start,
+                        expect_status=1)
+    O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, 0, np.arange(int(batch.k_len[0])))
+    H.check_close(got, O, "seq 0")
