@@ -51,7 +51,7 @@
 extern "C" {
 #endif
 
-#define SONIC_ABI_VERSION 3
+#define SONIC_ABI_VERSION 4
 
 #if defined(__GNUC__)
 #define SONIC_API __attribute__((visibility("default")))
@@ -132,6 +132,8 @@ typedef struct {
     int32_t *status;             /* device int32 or NULL                                */
     void *workspace;             /* device, sonic_compact_workspace_size() bytes        */
     size_t workspace_bytes;
+    int32_t total_rows;          /* rows per layer of K, V, role, seg_id (> 0); a
+                                    sequence outside them is refused                    */
 } sonic_compact_args;
 
 /*
@@ -148,7 +150,9 @@ typedef struct {
  * violation sets SONIC_ERR_LAYOUT.  If offsets[B] > out_capacity_rows the
  * call sets SONIC_ERR_CAPACITY and copies only rows below the capacity.
  * K/V/out pointers must be 16-byte aligned.  B > 65535 or n_layers > 32767
- * returns SONIC_ERR_UNSUPPORTED.
+ * returns SONIC_ERR_UNSUPPORTED.  A sequence whose rows fall outside
+ * [0, total_rows) keeps no rows (ret_len 0) and sets
+ * SONIC_ERR_INVALID_ARGUMENT in *status; none of its rows is read.
  */
 SONIC_API sonic_status_t sonic_compact_kv(const void *K, const void *V, const int32_t *seg_id,
                                 const uint8_t *role, void *out_K, void *out_V,

@@ -27,6 +27,12 @@ namespace {
 constexpr int kScanThreads = 512;
 constexpr int kChunks = 64;  // pieces per sequence in the scans
 
+// Rows of sequence (start, len), or 0 when they fall outside [0, total): such a
+// sequence is refused, keeps nothing and is never read.
+__device__ __forceinline__ int32_t seq_rows(int32_t start, int32_t len, int32_t total) {
+    return (start < 0 || len < 0 || (int64_t)start + len > total) ? 0 : len;
+}
+
 // Rows [*lo, *hi) of piece c of a sequence of len rows (32-row aligned pieces).
 __device__ __forceinline__ void piece(int32_t len, int c, int32_t *lo, int32_t *hi) {
     const long long ch = (((long long)len + kChunks - 1) / kChunks + 31) & ~31LL;
@@ -37,11 +43,13 @@ __device__ __forceinline__ void piece(int32_t len, int c, int32_t *lo, int32_t *
 __global__ void __launch_bounds__(kScanThreads)
 keep_count_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                   const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
-                  int32_t *__restrict__ counts, int32_t *status) {
+                  int32_t total, int32_t *__restrict__ counts, int32_t *status) {
     const int c = blockIdx.x, b = blockIdx.y;
     const int32_t start = k_start[b];
+    const int32_t len = seq_rows(start, k_len[b], total);
+    if (c == 0 && threadIdx.x == 0 && len != k_len[b]) set_status(status, SONIC_ERR_INVALID_ARGUMENT);
     int32_t lo, hi;
-    piece(k_len[b], c, &lo, &hi);
+    piece(len, c, &lo, &hi);
     int n = 0;
     bool bad = false;
     for (int32_t t = lo + threadIdx.x; t < hi; t += blockDim.x) {
@@ -133,7 +141,7 @@ __global__ void __launch_bounds__(kScanThreads)
 keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                     const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
                     const int32_t *__restrict__ reserve, const int32_t *__restrict__ counts,
-                    const long long *__restrict__ seq_base, int32_t capacity,
+                    const long long *__restrict__ seq_base, int32_t capacity, int32_t total,
                     int32_t *__restrict__ src_idx, uint8_t *__restrict__ out_role,
                     int32_t *__restrict__ out_seg) {
     const int c = blockIdx.x, b = blockIdx.y;
@@ -143,7 +151,7 @@ keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
     // output base of this piece: the sequence's offset plus the earlier pieces
     long long base = seq_base[b];
     for (int i = 0; i < c; ++i) base += counts[b * kChunks + i];
-    const int32_t start = k_start[b], len = k_len[b];
+    const int32_t start = k_start[b], len = seq_rows(start, k_len[b], total);
     int32_t lo, hi;
     piece(len, c, &lo, &hi);
     long long running = base;
@@ -287,6 +295,7 @@ extern "C" sonic_status_t sonic_compact_kv(const void *K, const void *V, const i
     if (!aligned16(K) || !aligned16(V) || !aligned16(out_K) || !aligned16(out_V))
         return SONIC_ERR_INVALID_ARGUMENT;
     if (a->n_layers > 32767 || a->batch > 65535) return SONIC_ERR_UNSUPPORTED;
+    if (a->total_rows <= 0) return SONIC_ERR_INVALID_ARGUMENT;
     const size_t need = sonic_compact_workspace_size(a);
     if (need > 0 && (a->workspace == nullptr || a->workspace_bytes < need))
         return SONIC_ERR_WORKSPACE;
@@ -300,13 +309,13 @@ extern "C" sonic_status_t sonic_compact_kv(const void *K, const void *V, const i
 
     const dim3 pieces(kChunks, a->batch);
     keep_count_kernel<<<pieces, kScanThreads, 0, stream>>>(role, seg_id, a->k_start, a->k_len,
-                                                          counts, a->status);
+                                                          a->total_rows, counts, a->status);
     keep_bases_kernel<<<1, kScanThreads, 0, stream>>>(counts, a->reserve, a->batch,
                                                       a->out_capacity_rows, seq_base, offsets,
                                                       a->ret_len, a->status);
     keep_scatter_kernel<<<pieces, kScanThreads, 0, stream>>>(
         role, seg_id, a->k_start, a->k_len, a->reserve, counts, seq_base, a->out_capacity_rows,
-        src_idx, a->out_role, a->out_seg);
+        a->total_rows, src_idx, a->out_role, a->out_seg);
     const int sms = device_sm_count();
     // Enough blocks per (layer, K|V) to keep every SM busy with ~8 blocks.
     const int per_slice = (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers);

@@ -46,7 +46,7 @@ class sonic_compact_args(ctypes.Structure):
                 ("reserve", _P), ("row_bytes", _i64), ("in_layer_bytes", _i64),
                 ("out_layer_bytes", _i64), ("out_capacity_rows", _i32), ("ret_len", _P),
                 ("src_idx", _P), ("out_role", _P), ("out_seg", _P), ("status", _P),
-                ("workspace", _P), ("workspace_bytes", _sz)]
+                ("workspace", _P), ("workspace_bytes", _sz), ("total_rows", _i32)]
 
 
 class sonic_prefill_args(ctypes.Structure):
@@ -180,6 +180,7 @@ def sonic_compact_kv(K: torch.Tensor, V: torch.Tensor, seg_id: Optional[torch.Te
     a.out_capacity_rows = out_K.shape[1]
     a.ret_len, a.src_idx = _ptr(ret_len), _ptr(src_idx)
     a.out_role, a.out_seg, a.status = _ptr(out_role), _ptr(out_seg), _ptr(status)
+    a.total_rows = min([T, role.numel()] + ([seg_id.numel()] if seg_id is not None else []))
     need = lib.sonic_compact_workspace_size(ctypes.byref(a))
     ws = _workspace(need, K.device, workspace)
     a.workspace, a.workspace_bytes = _ptr(ws), need

@@ -26,7 +26,7 @@ def test_library_exports_every_declared_symbol():
     for n in names:
         assert hasattr(lib, n), n
     assert set(names) == set(sonic.SIGNATURES)
-    assert lib.sonic_abi_version() == 3
+    assert lib.sonic_abi_version() == 4
     assert lib.sonic_status_string(4) == b"output capacity exceeded"
 
 
@@ -66,6 +66,8 @@ def test_host_validation_rejects_before_launch():
     assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 1
     a.row_bytes = 32
     assert lib.sonic_compact_kv(17, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 1  # misaligned
+    assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 1  # no rows
+    a.total_rows = 10
     assert lib.sonic_compact_kv(16, 16, None, 16, 16, 16, 16, ctypes.byref(a), None) == 3  # no workspace
 
     p = sonic.sonic_prefill_args()

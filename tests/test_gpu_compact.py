@@ -136,3 +136,27 @@ def test_many_sequences_and_long_pieces():
     V = inputs.randn((1, batch.total, 1, 64), seed=7, device=H.dev())
     r = _run(batch, K, V, reserve=reserve)
     _check(batch, K, V, r, reserve=reserve)
+
+
+def test_sequence_outside_the_rows_is_refused():
+    """k_start past the input rows: the sequence keeps nothing (ret_len 0) and
+    the status word says SONIC_ERR_INVALID_ARGUMENT; the others are exact."""
+    ds = [inputs.Dialogue(10, [(40, 5)], 8), inputs.Dialogue(6, [(30, 4), (12, 3)], 9)]
+    batch = inputs.Batch(ds)
+    K = inputs.randn((2, batch.total, 1, 64), seed=9, device=H.dev())
+    role, seg, k_start, k_len = H.meta(batch)
+    k_start = H.i32([int(batch.k_start[0]), batch.total + 50])
+    cap = ds[0].recipe_retained
+    oK = torch.zeros((2, cap, 1, 64), dtype=K.dtype, device=H.dev())
+    oV = torch.zeros_like(oK)
+    offsets = torch.full((3,), -7, dtype=torch.int32, device=H.dev())
+    ret_len = torch.full((2,), -7, dtype=torch.int32, device=H.dev())
+    status = torch.zeros(1, dtype=torch.int32, device=H.dev())
+    sonic.sonic_compact_kv(K, K, seg, role, oK, oV, offsets, k_start=k_start, k_len=k_len,
+                           ret_len=ret_len, status=status)
+    torch.cuda.synchronize()
+    assert sonic.read_status(status) == 1
+    assert ret_len.tolist() == [cap, 0] and offsets.tolist() == [0, cap, cap]
+    keep = np.nonzero(batch.role[:int(batch.k_len[0])] != inputs.ROLE_BODY)[0]
+    assert torch.equal(oK.view(torch.int16), K[:, torch.as_tensor(keep).long().to(H.dev())]
+                       .view(torch.int16))
