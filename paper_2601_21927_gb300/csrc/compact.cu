@@ -197,7 +197,7 @@ keep_scatter_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
 // warp works on two rows at a time with all their loads issued before the
 // stores, so up to 8 x 16 bytes per thread are in flight.
 constexpr int kGatherThreads = 256;
-constexpr int kGatherUnroll = 4;
+
 
 __device__ __forceinline__ int4 ld_stream(const void *p) {
     int4 v;
@@ -207,6 +207,10 @@ __device__ __forceinline__ int4 ld_stream(const void *p) {
     return v;
 }
 
+// kGatherRows rows a warp moves per pass, kGatherUnroll 16-byte pieces of each
+// per lane per step: 2 x 4 for rows under 2 KB, 4 x 2 for larger rows (more
+// rows in flight helps the long rows; at 1 KB it measured slower).
+template <int kGatherRows, int kGatherUnroll>
 __global__ void __launch_bounds__(kGatherThreads)
 kv_gather_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
                  uint8_t *__restrict__ out_K, uint8_t *__restrict__ out_V,
@@ -222,33 +226,35 @@ kv_gather_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
     const int lane = threadIdx.x & 31;
     const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int cpr = (int)(row_bytes >> 4);  // 16-byte chunks per row
+    // each warp moves kGatherRows rows per pass (n_warps apart), every lane
+    // holding its 16-byte pieces of all of them in flight
     for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5); r0 < n_rows;
-         r0 += 2 * n_warps) {
-        const int64_t r1 = r0 + n_warps;
-        const int32_t s0 = src_idx[r0];
-        const int32_t s1 = r1 < n_rows ? src_idx[r1] : -1;
-        const uint8_t *p0 = src + (int64_t)s0 * row_bytes;
-        const uint8_t *p1 = src + (int64_t)s1 * row_bytes;
-        uint8_t *q0 = dst + r0 * row_bytes;
-        uint8_t *q1 = dst + r1 * row_bytes;
+         r0 += kGatherRows * n_warps) {
+        int32_t sr[kGatherRows];
+#pragma unroll
+        for (int k = 0; k < kGatherRows; ++k) {
+            const int64_t r = r0 + k * n_warps;
+            sr[k] = r < n_rows ? src_idx[r] : -1;
+        }
         for (int c0 = lane; c0 < cpr; c0 += 32 * kGatherUnroll) {
-            int4 v0[kGatherUnroll], v1[kGatherUnroll];
+            int4 v[kGatherRows][kGatherUnroll];
 #pragma unroll
-            for (int u = 0; u < kGatherUnroll; ++u) {
-                const int c = c0 + 32 * u;
-                if (c < cpr) {
-                    if (s0 >= 0) v0[u] = ld_stream(p0 + ((int64_t)c << 4));
-                    if (s1 >= 0) v1[u] = ld_stream(p1 + ((int64_t)c << 4));
-                }
-            }
+            for (int k = 0; k < kGatherRows; ++k)
 #pragma unroll
-            for (int u = 0; u < kGatherUnroll; ++u) {
-                const int c = c0 + 32 * u;
-                if (c < cpr) {
-                    if (s0 >= 0) *reinterpret_cast<int4 *>(q0 + ((int64_t)c << 4)) = v0[u];
-                    if (s1 >= 0) *reinterpret_cast<int4 *>(q1 + ((int64_t)c << 4)) = v1[u];
+                for (int u = 0; u < kGatherUnroll; ++u) {
+                    const int c = c0 + 32 * u;
+                    if (c < cpr && sr[k] >= 0)
+                        v[k][u] = ld_stream(src + (int64_t)sr[k] * row_bytes + ((int64_t)c << 4));
                 }
-            }
+#pragma unroll
+            for (int k = 0; k < kGatherRows; ++k)
+#pragma unroll
+                for (int u = 0; u < kGatherUnroll; ++u) {
+                    const int c = c0 + 32 * u;
+                    if (c < cpr && sr[k] >= 0)
+                        *reinterpret_cast<int4 *>(dst + (r0 + k * n_warps) * row_bytes +
+                                                  ((int64_t)c << 4)) = v[k][u];
+                }
         }
     }
 }
@@ -320,7 +326,8 @@ extern "C" sonic_status_t sonic_compact_kv(const void *K, const void *V, const i
     // Enough blocks per (layer, K|V) to keep every SM busy with ~8 blocks.
     const int per_slice = (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers);
     dim3 grid(per_slice < 1 ? 1 : per_slice, 2 * a->n_layers);
-    kv_gather_kernel<<<grid, kGatherThreads, 0, stream>>>(
+    auto gather = a->row_bytes >= 2048 ? kv_gather_kernel<4, 2> : kv_gather_kernel<2, 4>;
+    gather<<<grid, kGatherThreads, 0, stream>>>(
         static_cast<const uint8_t *>(K), static_cast<const uint8_t *>(V),
         static_cast<uint8_t *>(out_K), static_cast<uint8_t *>(out_V), offsets, src_idx, a->batch,
         a->out_capacity_rows, a->row_bytes, a->in_layer_bytes, a->out_layer_bytes);
