@@ -298,6 +298,29 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     const bool tile1 = qt * 2 * R + R < qlen;     // tile 1 has rows
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
+    // ------------------------------------------------ barriers, and Q on its way
+    // (its copy needs nothing from the tile list below, so it flies meanwhile)
+    if (tid == 0) {
+        mbar_init(q_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&kv_full[s], 32);
+            mbar_init(&kv_empty[s], 1);
+            mbar_init(&s_full[s], 1);
+            mbar_init(&p_full[s], kBM);
+            mbar_init(&o_done[s], 1);
+        }
+        mbar_init(mma_idle, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&tmQ);
+        mbar_arrive_expect_tx(q_full, (tile1 ? 2 : 1) * C::kQBytes);
+        for (int qi = 0; qi < (tile1 ? 2 : 1); ++qi)
+#pragma unroll
+            for (int hh = 0; hh < C::kHalves; ++hh)
+                tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full, hh * 64, h0,
+                            p.q_start[b] + qt * 2 * R + qi * R, layer);
+    }
+
     // ------------------------------------------------ summaries of the query tiles
     if (tid < 10) misc[4 + tid] = (tid % 5 == 0) ? 0 : ((tid % 5) & 1 ? INT_MAX : INT_MIN);
     __syncthreads();
@@ -364,20 +387,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         __syncthreads();
     }
 
-    // ------------------------------------------------ barriers and tensor memory
-    if (tid == 0) {
-        mbar_init(q_full, 1);
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&kv_full[s], 32);
-            mbar_init(&kv_empty[s], 1);
-            mbar_init(&s_full[s], 1);
-            mbar_init(&p_full[s], kBM);
-            mbar_init(&o_done[s], 1);
-        }
-        mbar_init(mma_idle, 1);
-        *abort_flag = 0;
-        fence_mbar_init();
-    }
+    // ------------------------------------------------ tensor memory
     if (warp == 1) {
         tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 512);
         tmem_relinquish();
@@ -389,15 +399,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
-            tma_prefetch_desc(&tmQ);
             tma_prefetch_desc(&tmK);
             tma_prefetch_desc(&tmV);
-            mbar_arrive_expect_tx(q_full, (tile1 ? 2 : 1) * C::kQBytes);
-            for (int qi = 0; qi < (tile1 ? 2 : 1); ++qi)
-#pragma unroll
-                for (int hh = 0; hh < C::kHalves; ++hh)
-                    tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full, hh * 64,
-                                h0, p.q_start[b] + qt * 2 * R + qi * R, layer);
         }
         int i = 0;
         for (; i < n_list; ++i) {
