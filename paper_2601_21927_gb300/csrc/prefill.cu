@@ -900,7 +900,8 @@ __device__ __forceinline__ int span_of(int len) { return (len + kBN - 1) / kBN *
 
 __global__ void __launch_bounds__(kOrderThreads)
 key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
-                 const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len, int B,
+                 const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
+                 const int32_t *__restrict__ q_len, int B,
                  int max_k_len, int64_t total_rows, int64_t capacity,
                  int32_t *__restrict__ key_start,
                  int32_t *__restrict__ key_len, uint8_t *__restrict__ o_role,
@@ -909,7 +910,7 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int sh[2][32];
     __shared__ long long sh_base;
-    __shared__ int sh_r;
+    __shared__ int sh_r, sh_smin, sh_first;
     // start of this sequence's span: the spans of the sequences before it
     long long base = 0;
     for (int i = tid; i < b; i += kOrderThreads)
@@ -917,6 +918,8 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     if (tid == 0) {
         sh_base = 0;
         sh_r = 0;
+        sh_smin = INT_MAX;
+        sh_first = INT_MAX;
     }
     __syncthreads();
     if (base) atomicAdd(reinterpret_cast<unsigned long long *>(&sh_base), (unsigned long long)base);
@@ -928,7 +931,15 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     for (int i = tid; i < len; i += kOrderThreads) cnt += role[ks + i] != SONIC_ROLE_BODY;
     cnt = __reduce_add_sync(0xffffffffu, cnt);
     if (lane == 0 && cnt) atomicAdd(&sh_r, cnt);
+    // the smallest segment among the query rows (the last q_len rows): a body
+    // row of an earlier segment is seen by no query row of this call
+    const int ql = min(max(q_len[b], 0), len);
+    int smin = INT_MAX;
+    for (int i = len - ql + tid; i < len; i += kOrderThreads) smin = min(smin, seg[ks + i]);
+    smin = __reduce_min_sync(0xffffffffu, smin);
+    if (lane == 0 && smin != INT_MAX) atomicMin(&sh_smin, smin);
     __syncthreads();
+    const int s_min = sh_smin;
     const long long start = sh_base;
     const int R = sh_r, span = span_of(len);
     if (b == B - 1 && tid == 0) key_start[B] = (int32_t)min(start + span, (long long)capacity);
@@ -975,10 +986,12 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
         if (valid) {
             const int dst = keep ? kept + pk + __popc(bk & below) : body0 + bodies + pb + __popc(bb & below);
             const int64_t o = start + dst;
+            const int sv = seg[ks + i];
             o_role[o] = (uint8_t)r;
-            o_seg[o] = seg[ks + i];
+            o_seg[o] = sv;
             o_pos[o] = i;
             o_src[o] = ks + i;
+            if (body && sv >= s_min) atomicMin(&sh_first, dst - body0);
         }
         kept += tk;
         bodies += tb;
@@ -994,6 +1007,14 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
             o_src[start + i] = -1;
         }
     }
+    // Whole 128-row tiles of bodies before the first body row a query row can
+    // see are never visited: their K/V rows are not copied (src -2).  A tile
+    // holding any such row is copied whole, so a masked key never carries
+    // stale data into P.V.
+    __syncthreads();
+    const int first = min(sh_first, len - R);  // body rows before it: unseen
+    for (int i = body0 + tid; i < body0 + (first / kBN) * kBN; i += kOrderThreads)
+        o_src[start + i] = -2;
     if (tid == 0) {
         key_start[b] = (int32_t)start;
         key_len[b] = lp;
@@ -1028,6 +1049,7 @@ kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
     for (int64_t r = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < n_rows;
          r += n_warps) {
         const int32_t s = src[r];
+        if (s == -2) continue;  // a body tile no query row of the call sees
         const uint8_t *pi = in + (int64_t)s * row_bytes;
         uint8_t *po = out + r * row_bytes;
         for (int c0 = lane; c0 < cpr; c0 += 32 * 4) {
@@ -1228,7 +1250,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
 
     if (reorder) {
         key_order_kernel<<<a->batch, kOrderThreads, 0, stream>>>(
-            role, seg_id, a->k_start, a->k_len, a->batch, a->max_k_len, a->total_k_rows, ws.rows,
+            role, seg_id, a->k_start, a->k_len, a->q_len, a->batch, a->max_k_len, a->total_k_rows,
+            ws.rows,
             reinterpret_cast<int32_t *>(wsb + ws.key_start),
             reinterpret_cast<int32_t *>(wsb + ws.key_len), wsb + ws.role,
             reinterpret_cast<int32_t *>(wsb + ws.seg), reinterpret_cast<int32_t *>(wsb + ws.pos),

@@ -231,3 +231,23 @@ def test_sequence_outside_the_arrays_is_refused(order):
                         expect_status=1)
     O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, 0, np.arange(int(batch.k_len[0])))
     H.check_close(got, O, "seq 0")
+
+
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+def test_retained_first_query_suffix_skips_unseen_bodies(mode):
+    """Queries are a suffix of S_aug starting inside a history segment: the
+    retained-first copy leaves out the body tiles of earlier segments (no
+    query row can see them) and every output still equals the oracle."""
+    ds = [inputs.Dialogue(64, [(300, 20)] * 6 + [(200, 40)], 90),
+          inputs.Dialogue(10, [(128, 16)] * 9, 33), inputs.Dialogue(0, [(700, 7)], 5)]
+    batch = inputs.Batch(ds)
+    # from the middle of the 5th segment's body / the 7th segment / the current turn
+    first = [64 + 4 * 320 + 150, 10 + 6 * 144 + 5, 700 + 7]
+    q_len = [int(batch.k_len[b]) - first[b] for b in range(batch.B)]
+    res = H.run_prefill(batch, 4, 2, 128, q_len=q_len, seed=71, nexus_vis=mode,
+                        key_order=sonic.KEYS_RETAINED_FIRST)
+    for b in range(batch.B):
+        O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, np.arange(q_len[b]),
+                                                     nexus_vis=mode)
+        H.check_close(got, O, f"seq {b}")
+        np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
