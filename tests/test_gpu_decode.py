@@ -168,3 +168,10 @@ def test_sequence_outside_the_cache_is_refused():
         s0, n = int(starts[b]), int(lens[b])
         Oref, _ = oracle.decode(H.f64(q[0, b]), H.f64(K[0, s0:s0 + n]), H.f64(V[0, s0:s0 + n]))
         H.check_close(H.f64(O[0, b]), Oref, f"seq {b}")
+
+
+def test_very_long_cache():
+    """One decode step over 500,000 retained rows (split into many chunks and
+    merged), next to a one-row sequence."""
+    r = _decode([500_000, 1], 8, 2, 128, n_layers=1, seed=41, pad=3)
+    _check(r, [(0, 0), (0, 1)])

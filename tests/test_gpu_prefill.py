@@ -251,3 +251,21 @@ def test_retained_first_query_suffix_skips_unseen_bodies(mode):
                                                      nexus_vis=mode)
         H.check_close(got, O, f"seq {b}")
         np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
+
+
+@pytest.mark.parametrize("order,L", [(sonic.KEYS_AS_GIVEN, 262144),
+                                     (sonic.KEYS_RETAINED_FIRST, 262016)])
+def test_longest_sequence(order, L):
+    """The longest key sequence the call accepts (2047 key tiles; one fewer
+    with the retained-first order, whose copy adds a tile), history segments
+    of 4000 body + 400 Nexus rows and a 64-row current turn as the queries:
+    sampled rows against the oracle."""
+    n_seg = (L - 1000 - 64) // 4400
+    sys_len = L - 64 - n_seg * 4400
+    d = inputs.Dialogue(sys_len, [(4000, 400)] * n_seg, 64)
+    assert d.length == L
+    batch = inputs.Batch([d])
+    res = H.run_prefill(batch, 8, 2, 128, q_len=[64], seed=81, key_order=order)
+    O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, 0, np.array([0, 31, 63]))
+    H.check_close(got, O, "longest sequence")
+    np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
