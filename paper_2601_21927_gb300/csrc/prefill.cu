@@ -20,6 +20,7 @@
 // numbers occur in it) as hidden (skipped entirely), fully visible (no mask
 // work) or cut by the mask.  The two tiles' softmax and MMAs interleave.
 #include <algorithm>
+#include <type_traits>
 
 #include "sonic_dev.cuh"
 #include "sonic_host.h"
@@ -560,29 +561,37 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
+        // This thread is on the path of every key tile, so its loop is
+        // specialised on the number of query tiles and unrolled over the two
+        // K/V stages, and each descriptor is a precomputed word plus a constant:
+        // an MMA then costs about two instructions besides itself.
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, 0);
             constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, 1);
-            const uint32_t q_addr = smem_u32(Qs), k_addr = smem_u32(Ks), v_addr = smem_u32(Vs);
+            constexpr uint32_t dhi = sw128_desc_hi(1024);
+            const uint32_t q_lo = sw128_desc_lo(smem_u32(Qs), 16);
+            const uint32_t k_lo = sw128_desc_lo(smem_u32(Ks), 16);
+            const uint32_t v_lo = sw128_desc_lo(smem_u32(Vs), kBN * 128);
             const int nq = tile1 ? 2 : 1;
+            // S_qi = Q_qi K^T from K stage st
             auto issue_s = [&](int qi, int st) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
-                    const uint64_t a = smem_desc_sw128(q_addr + qi * C::kQBytes + off, 16, 1024);
-                    const uint64_t bd = smem_desc_sw128(k_addr + st * C::kKVBytes + off, 16, 1024);
-                    tc_mma_ss(tmem + qi * kBN, a, bd, idS, kk > 0 ? 1u : 0u);
+                    const uint32_t off = ((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4;
+                    tc_mma_ss(tmem + qi * kBN,
+                              desc_join(q_lo + ((qi * C::kQBytes) >> 4) + off, dhi),
+                              desc_join(k_lo + ((st * C::kKVBytes) >> 4) + off, dhi), idS,
+                              kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[qi]);
             };
-            auto issue_pv = [&](int qi, int st, int j) {
+            // O_qi += P_qi V from V stage st (P over the first columns of S_qi)
+            auto issue_pv = [&](int qi, int st, bool acc0) {
 #pragma unroll
-                for (int kk = 0; kk < kBN / 16; ++kk) {
-                    const uint64_t bd = smem_desc_sw128(v_addr + st * C::kKVBytes + kk * (16 * 128),
-                                                        kBN * 128, 1024);
-                    tc_mma_ts(tmem + 256 + qi * 128, tmem + qi * kBN + kk * 8, bd, idPV,
-                              (j > 0 || kk > 0) ? 1u : 0u);
-                }
+                for (int kk = 0; kk < kBN / 16; ++kk)
+                    tc_mma_ts(tmem + 256 + qi * 128, tmem + qi * kBN + kk * 8,
+                              desc_join(v_lo + ((st * C::kKVBytes + kk * (16 * 128)) >> 4), dhi),
+                              idPV, (acc0 || kk > 0) ? 1u : 0u);
             };
             bool ok = mbar_wait(q_full, 0, p.status, abort_flag) && n_list > 0 &&
                       mbar_wait(&kv_full[0], 0, p.status, abort_flag);
@@ -590,28 +599,41 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 tc_fence_after();
                 for (int qi = 0; qi < nq; ++qi) issue_s(qi, 0);
             }
-            for (int j = 0; ok && j < n_list; ++j) {
-                const int st = j & 1, nst = (j + 1) & 1;
-                const bool more = j + 1 < n_list;
-                for (int qi = 0; qi < nq; ++qi) {
-                    if (!mbar_wait(&p_full[qi], j & 1, p.status, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    issue_pv(qi, st, j);
-                    if (!more) tc_commit(&o_done[qi]);
-                    if (qi == nq - 1) tc_commit(&kv_empty[st]);
-                    if (more) {
-                        if (qi == 0 &&
-                            !mbar_wait(&kv_full[nst], ((j + 1) >> 1) & 1, p.status, abort_flag)) {
-                            ok = false;
-                            break;
-                        }
+            // Key tile j (in stage j & 1): P.V of each query tile, then its S of
+            // tile j + 1.  The tensor pipe runs in order, so the next S never
+            // overwrites a P still being read.
+            auto main_loop = [&](auto nq_tag) {
+                constexpr int NQ = decltype(nq_tag)::value;
+                auto tile = [&](int j, auto st_tag) -> bool {
+                    constexpr int ST = decltype(st_tag)::value;
+                    const bool more = j + 1 < n_list;
+#pragma unroll
+                    for (int qi = 0; qi < NQ; ++qi) {
+                        if (!mbar_wait(&p_full[qi], ST, p.status, abort_flag)) return false;
                         tc_fence_after();
-                        issue_s(qi, nst);
+                        issue_pv(qi, ST, j > 0);
+                        if (!more) tc_commit(&o_done[qi]);
+                        if (qi == NQ - 1) tc_commit(&kv_empty[ST]);
+                        if (more) {
+                            if (qi == 0 && !mbar_wait(&kv_full[1 - ST], ((j + 1) >> 1) & 1,
+                                                      p.status, abort_flag))
+                                return false;
+                            tc_fence_after();
+                            issue_s(qi, 1 - ST);
+                        }
                     }
+                    return true;
+                };
+                for (int j = 0; ok && j < n_list; j += 2) {
+                    ok = tile(j, std::integral_constant<int, 0>{});
+                    if (ok && j + 1 < n_list) ok = tile(j + 1, std::integral_constant<int, 1>{});
                 }
+            };
+            if (ok) {
+                if (nq == 2)
+                    main_loop(std::integral_constant<int, 2>{});
+                else
+                    main_loop(std::integral_constant<int, 1>{});
             }
             // every MMA issued by this thread has finished once this arrives
             tc_commit(mma_idle);

@@ -293,6 +293,20 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
     return d;
 }
 
+// The two 32-bit words of smem_desc_sw128, for an issuing loop that forms many
+// descriptors as a fixed one plus offsets: adding (offset >> 4) to the low word
+// moves the start address, whose 14-bit field never carries into the next one
+// because shared-memory addresses stay below 2^18 bytes.
+__device__ __forceinline__ uint32_t sw128_desc_lo(uint32_t saddr, uint32_t lbo_bytes) {
+    return ((saddr >> 4) & 0x3FFFu) | (((lbo_bytes >> 4) & 0x3FFFu) << 16);
+}
+__host__ __device__ constexpr uint32_t sw128_desc_hi(uint32_t sbo_bytes) {
+    return ((sbo_bytes >> 4) & 0x3FFFu) | (1u << 14) | (2u << 29);  // version 1, SWIZZLE_128B
+}
+__device__ __forceinline__ uint64_t desc_join(uint32_t lo, uint32_t hi) {
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
 // Instruction descriptor, kind::f16: bf16 A and B, fp32 D, dense.
 // b_mn_major / a_mn_major select MN-major operands (K-major otherwise).
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N,
