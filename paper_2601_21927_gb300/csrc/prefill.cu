@@ -787,43 +787,48 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             float ls[4] = {0.f, 0.f, 0.f, 0.f};
             float2 rs2x = make_float2(0.f, 0.f);
             // the Nexus part of the row sum: all of it, none, or (some Nexus
-            // keys) the keys the tile's Nexus bits select
+            // keys) the keys the tile's Nexus bits select.  The two forms of
+            // the loop are separate instances, so the common one stays one
+            // straight run of code the compiler can interleave across chunks.
             float lsn[2] = {0.f, 0.f};
-            uint32_t nxb[4] = {0u, 0u, 0u, 0u};
-            const bool some_nexus = kMass && nexus_keys == 2;
-            if (some_nexus) {
-                const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
-                nxb[0] = nx.x;
-                nxb[1] = nx.y;
-                nxb[2] = nx.z;
-                nxb[3] = nx.w;
-            }
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t pk[16];
-#pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const float2 x = __ffma2_rn(
-                        make_float2(__uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1])), sc2,
-                        nm2);
-                    const float2 eu = make_float2(ex2(x.x), ex2(x.y));
-                    if (kLse) rs2x = __fadd2_rn(rs2x, eu);
-                    const uint32_t pr = pack_bf16x2(eu.x, eu.y);
-                    pk[e >> 1] = pr;
-                    // the row sum adds the rounded probabilities P.V multiplies
-                    // by, so O is a weighted mean of V rows with weights summing
-                    // to one (rounding moves weight between keys, it does not
-                    // scale the output)
-                    add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
+            auto exps = [&](auto nx_tag) {
+                constexpr bool NX = decltype(nx_tag)::value;
+                uint32_t nxb[4] = {0u, 0u, 0u, 0u};
+                if (NX) {
+                    const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
+                    nxb[0] = nx.x;
+                    nxb[1] = nx.y;
+                    nxb[2] = nx.z;
+                    nxb[3] = nx.w;
                 }
-                if (some_nexus) {
 #pragma unroll
-                    for (int e = 0; e < 32; e += 2)
-                        add_bf16x2_to_f32_if(lsn[0], lsn[1], pk[e >> 1], nxb[c] & (1u << e),
-                                             nxb[c] & (2u << e));
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c][e]),
+                                                                __uint_as_float(sr[c][e + 1])),
+                                                    sc2, nm2);
+                        const float2 eu = make_float2(ex2(x.x), ex2(x.y));
+                        if (kLse) rs2x = __fadd2_rn(rs2x, eu);
+                        const uint32_t pr = pack_bf16x2(eu.x, eu.y);
+                        pk[e >> 1] = pr;
+                        // the row sum adds the rounded probabilities P.V
+                        // multiplies by, so O is a weighted mean of V rows with
+                        // weights summing to one (rounding moves weight between
+                        // keys, it does not scale the output)
+                        add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
+                        if (NX)
+                            add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << e),
+                                                 nxb[c] & (2u << e));
+                    }
+                    tmem_st16(tS + c * 16, pk);
                 }
-                tmem_st16(tS + c * 16, pk);
-            }
+            };
+            if (kMass && nexus_keys == 2)
+                exps(std::true_type{});
+            else
+                exps(std::false_type{});
             const float l_tile = (ls[0] + ls[1]) + (ls[2] + ls[3]);
             l = l * alpha + l_tile;
             if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
