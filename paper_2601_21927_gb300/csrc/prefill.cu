@@ -267,6 +267,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint64_t *p_full = bars + 7;    // [2] per query tile
     uint64_t *o_done = bars + 9;    // [2] per query tile
     uint64_t *mma_idle = bars + 11;
+    uint64_t *meta_full = bars + 12;  // [2] key metadata of a stage written
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
     // misc: 0 tmem base, 2 abort, 4..13 query-tile summaries (5 per tile),
     //       16..27 per-warp counts
@@ -304,7 +305,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     if (tid == 0) {
         mbar_init(q_full, 1);
         for (int s = 0; s < 2; ++s) {
-            mbar_init(&kv_full[s], 32);
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&meta_full[s], 32);
             mbar_init(&kv_empty[s], 1);
             mbar_init(&s_full[s], 1);
             mbar_init(&p_full[s], kBM);
@@ -410,8 +412,10 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 break;
             const int kt = list[i] >> 4;
             // K/V copies first; the key metadata is built while they are in flight
+            // and has a barrier of its own, so the S MMA of a cut tile waits for
+            // the copy alone, not for the metadata
             if (lane == 0) {
-                mbar_expect_tx(&kv_full[st], 2 * C::kKVBytes);
+                mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
                 const int row = kkstart + kt * kBN;
 #pragma unroll
                 for (int hh = 0; hh < C::kHalves; ++hh) {
@@ -437,7 +441,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     }
                     __syncwarp();
                 }
-                mbar_arrive(&kv_full[st]);
+                mbar_arrive(&meta_full[st]);
                 continue;
             }
             int ro[4], sg[4], ps[4];
@@ -551,7 +555,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 tm.rlen[lane] = c0 < 0 ? 0 : (c1 < 0 ? n_valid : c1) - c0;
             }
             __syncwarp();
-            mbar_arrive(&kv_full[st]);  // 32 arrivals + the copies' bytes end the phase
+            mbar_arrive(&meta_full[st]);  // 32 arrivals end the phase
         }
         if (lane == 0 && *abort_flag) {
             // let issued copies land before the block exits
@@ -673,7 +677,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // the keys' roles/segments are read (and V rows zeroed) on cut tiles
             // only, and their Nexus bits on tiles with some Nexus keys
             const bool need_meta = cut || (kMass && nexus_keys == 2);
-            if (need_meta && !mbar_wait(&kv_full[st], (j >> 1) & 1, p.status, abort_flag)) {
+            if (need_meta && !mbar_wait(&meta_full[st], (j >> 1) & 1, p.status, abort_flag)) {
                 ok = false;
                 break;
             }
