@@ -448,19 +448,22 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             uint32_t bst[4], nst[4], rst[4];
             int pro = 255, psg = 0, pps = INT_MIN, n_valid = 0;
             TileMasks &tm = tmasks[st];
+            // all twelve loads first, none waiting on another: one memory
+            // latency per tile instead of eight in a row
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const int q = kt * kBN + w * 32 + lane;
+                const bool in = q < kklen;
+                ro[w] = in ? p.key_role[kkstart + q] : 255;
+                sg[w] = in ? p.key_seg[kkstart + q] : 0;
+                ps[w] = in ? (p.key_pos != nullptr ? p.key_pos[kkstart + q] : q) : INT_MAX;
+            }
 #pragma unroll
             for (int w = 0; w < 4; ++w) {
                 const int c = w * 32 + lane;
-                const int q = kt * kBN + c;
-                ro[w] = 255;
-                sg[w] = 0;
-                ps[w] = INT_MAX;
-                if (q < kklen) {
-                    ro[w] = p.key_role[kkstart + q];
-                    if (ro[w] != 255) {
-                        sg[w] = p.key_seg[kkstart + q];
-                        ps[w] = p.key_pos != nullptr ? p.key_pos[kkstart + q] : q;
-                    }
+                if (ro[w] == 255) {  // padding: no segment, no position
+                    sg[w] = 0;
+                    ps[w] = INT_MAX;
                 }
                 meta_role[st * kBN + c] = (uint8_t)ro[w];
                 meta_seg[st * kBN + c] = sg[w];
