@@ -246,9 +246,9 @@ SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
  * callback, runtimes that plan every device byte ahead of time, or hosts that
  * only hand over fixed buffers for inputs and outputs.  This call takes the
  * same arguments as sonic_attn_prefill except that args->workspace and
- * args->workspace_bytes are ignored: the per-tile mask summaries live in a
- * fixed 1 MiB array compiled into the library (every GPU that loads the
- * library holds it until the process exits).  It allocates nothing.
+ * args->workspace_bytes are ignored: the per-tile summaries and column masks
+ * live in a fixed 9 MiB array compiled into the library (every GPU that loads
+ * the library holds it until the process exits).  It allocates nothing.
  *  - Limit: batch * ceil(max_k_len / 128) <= 32768; larger calls return
  *    SONIC_ERR_WORKSPACE before launching anything.  Only key_order AS_GIVEN
  *    is served (RETAINED_FIRST copies K and V into the workspace):

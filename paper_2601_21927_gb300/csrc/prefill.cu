@@ -20,6 +20,7 @@
 // numbers occur in it) as hidden (skipped entirely), fully visible (no mask
 // work) or cut by the mask.  The two tiles' softmax and MMAs interleave.
 #include <algorithm>
+#include <cstddef>
 #include <type_traits>
 
 #include "sonic_dev.cuh"
@@ -61,11 +62,204 @@ __device__ __forceinline__ int seq_rows(int start, int len, int max_len, int64_t
                                                                             : checked_len(len, max_len);
 }
 
+struct TileMasks;
+
+struct PfParams {
+    // query side: the sequences as given (S_aug order)
+    const int32_t *k_start, *k_len, *q_start, *q_len;
+    const uint8_t *role;
+    const int32_t *seg;
+    // key side: the same arrays, or their retained-first permutation
+    const int32_t *key_start, *key_len;
+    const uint8_t *key_role;
+    const int32_t *key_seg;
+    const int32_t *key_pos;  // S_aug position of each key row; NULL: the row index
+    uint16_t *O;
+    float *lse;
+    float *nexus_mass;
+    int32_t *status;
+    const TileSum *sums;
+    const TileMasks *masks;  // per key tile, from the summary kernel
+    int max_k_tiles, max_k_len;
+    int B, Hq, G;
+    int64_t total_k_rows;  // rows of role, seg_id (and K, V) per layer
+    int pack_log2;  // query heads per tile row group: a tile is 128 >> pack_log2 rows x (1 << pack_log2) heads
+    int64_t o_ls;
+    int total_q_rows;
+    float scale_log2;
+    int nexus_mode;
+};
+
+template <int D>
+struct PfCfg {
+    static constexpr int kHalves = D / 64;
+    static constexpr int kQBytes = kBM * D * 2;  // one 128-row Q tile
+    static constexpr int kKVBytes = kBN * D * 2;
+    static constexpr int kOffQ = 0;                           // [2] Q tiles
+    static constexpr int kOffK = kOffQ + 2 * kQBytes;         // [2] stages
+    static constexpr int kOffV = kOffK + 2 * kKVBytes;        // [2] stages
+    static constexpr int kOffMask = kOffV + 2 * kKVBytes;     // [2] TileMasks
+    static constexpr int kOffRole = kOffMask + 2 * 256;       // [2][128] uint8
+    static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
+    static constexpr int kOffPos = kOffSeg + 2 * kBN * 4;     // [2][128] int32
+    static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [kMaxKTiles] int32
+    static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
+    static constexpr int kNumBars = 16;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 32 ints
+    static constexpr int kBytes = kOffMisc + 32 * 4;
+    static constexpr size_t kSmem = 1024 + kBytes;
+};
+
+// Column masks of one 128-key tile (bit c of word w = key 32 w + c of the
+// tile): keys that are not body rows (nb), Nexus keys (nx), and the keys of
+// each distinct segment among the body keys (bm) and among the Nexus keys
+// (nm, used by the causal-segments reading); and the valid keys as runs of
+// consecutive S_aug positions (a tile's valid keys are a prefix of its rows
+// with increasing positions, so the keys at or before a position form a
+// prefix too, whose length the runs give).  With them a row's visibility
+// mask costs a few word operations.  More than four distinct segments or
+// position runs in one tile set `fallback`: the rule is then evaluated per
+// key instead.
+struct TileMasks {
+    uint32_t nb[4], nx[4];
+    int32_t nbody, nnex, fallback, nrun;
+    int32_t bseg[4], nseg[4];
+    uint32_t bm[4][4], nm[4][4];
+    // the valid keys as runs of consecutive S_aug positions, in column order
+    int32_t rpos[4], rlen[4];
+    int32_t pad[4];
+};
+static_assert(sizeof(TileMasks) == 256, "tile masks: one 256-byte record per key tile");
+static_assert(offsetof(TileMasks, fallback) == 40, "the producer reads fallback as word 10");
+
+// Column of the n-th (from 0) set bit of a 128-bit mask, or -1.
+__device__ __forceinline__ int nth_set_bit(const uint32_t m[4], int n) {
+    int col = -1;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const int c = __popc(m[w]);
+        if (col < 0 && n < c) {
+            uint32_t x = m[w];
+            for (int i = 0; i < n; ++i) x &= x - 1;
+            col = w * 32 + __ffs(x) - 1;
+        }
+        if (col < 0) n -= c;
+    }
+    return col;
+}
+
+// The column masks of one key tile, built by one warp: lane l holds key
+// 32 w + l of the tile in ro[w], sg[w], ps[w] (role 255, segment 0 and
+// position INT_MAX for padding and rows past the sequence).
+__device__ __forceinline__ void build_tile_masks(const int (&ro)[4], const int (&sg)[4],
+                                                 const int (&ps)[4], int lane, TileMasks *tm) {
+    uint32_t bst[4], nst[4], rst[4];
+    int pro = 255, psg = 0, pps = INT_MIN, n_valid = 0;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const bool valid = ro[w] != 255;
+        const bool isb = ro[w] == SONIC_ROLE_BODY, isn = ro[w] == SONIC_ROLE_NEXUS;
+        const uint32_t nbw = __ballot_sync(0xffffffffu, valid && !isb);
+        const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
+        n_valid += __popc(__ballot_sync(0xffffffffu, valid));
+        // previous key's role/segment/position (lane 0: last key of the
+        // previous word)
+        int r_up = __shfl_up_sync(0xffffffffu, ro[w], 1);
+        int s_up = __shfl_up_sync(0xffffffffu, sg[w], 1);
+        int p_up = __shfl_up_sync(0xffffffffu, ps[w], 1);
+        if (lane == 0) {
+            r_up = pro;
+            s_up = psg;
+            p_up = pps;
+        }
+        bst[w] = __ballot_sync(0xffffffffu, isb && !(r_up == SONIC_ROLE_BODY && s_up == sg[w]));
+        nst[w] = __ballot_sync(0xffffffffu, isn && !(r_up == SONIC_ROLE_NEXUS && s_up == sg[w]));
+        rst[w] = __ballot_sync(0xffffffffu, valid && p_up != ps[w] - 1);
+        pro = __shfl_sync(0xffffffffu, ro[w], 31);
+        psg = __shfl_sync(0xffffffffu, sg[w], 31);
+        pps = __shfl_sync(0xffffffffu, ps[w], 31);
+        if (lane == 0) {
+            tm->nb[w] = nbw;
+            tm->nx[w] = nxw;
+        }
+    }
+    // distinct segments of body runs and Nexus runs (in key order)
+    int nb_n = 0, nn_n = 0, fb = 0;
+    int bsv[4] = {0, 0, 0, 0}, nsv[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        uint32_t m = bst[w];
+        while (m) {
+            const int bl = __ffs(m) - 1;
+            m &= m - 1;
+            const int v = __shfl_sync(0xffffffffu, sg[w], bl);
+            bool seen = false;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) seen |= (k < nb_n && bsv[k] == v);
+            if (!seen) {
+                if (nb_n < 4) bsv[nb_n++] = v; else fb = 1;
+            }
+        }
+        m = nst[w];
+        while (m) {
+            const int bl = __ffs(m) - 1;
+            m &= m - 1;
+            const int v = __shfl_sync(0xffffffffu, sg[w], bl);
+            bool seen = false;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) seen |= (k < nn_n && nsv[k] == v);
+            if (!seen) {
+                if (nn_n < 4) nsv[nn_n++] = v; else fb = 1;
+            }
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const uint32_t bmw = __ballot_sync(
+                0xffffffffu, k < nb_n && ro[w] == SONIC_ROLE_BODY && sg[w] == bsv[k]);
+            const uint32_t nmw = __ballot_sync(
+                0xffffffffu, k < nn_n && ro[w] == SONIC_ROLE_NEXUS && sg[w] == nsv[k]);
+            if (lane == 0) {
+                tm->bm[k][w] = bmw;
+                tm->nm[k][w] = nmw;
+            }
+        }
+    const int nrun = __popc(rst[0]) + __popc(rst[1]) + __popc(rst[2]) + __popc(rst[3]);
+    if (lane == 0) {
+        tm->nbody = nb_n;
+        tm->nnex = nn_n;
+        tm->nrun = nrun;
+        tm->fallback = fb | (nrun > 4);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            tm->bseg[k] = bsv[k];
+            tm->nseg[k] = nsv[k];
+            tm->pad[k] = 0;
+        }
+    }
+    // position run k (lane k < 4): from the k-th run start to the next one
+    // (or to the last valid key); the start's position from the lane holding it
+    const int c0 = nth_set_bit(rst, lane & 3), c1 = nth_set_bit(rst, (lane & 3) + 1);
+    int start_pos = 0;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const int v = __shfl_sync(0xffffffffu, ps[w], c0 & 31);
+        if (c0 >= 0 && (c0 >> 5) == w) start_pos = v;
+    }
+    if (lane < 4) {
+        tm->rpos[lane] = c0 < 0 ? 0 : start_pos;
+        tm->rlen[lane] = c0 < 0 ? 0 : (c1 < 0 ? n_valid : c1) - c0;
+    }
+}
+
 __global__ void __launch_bounds__(128)
 tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
                     const int32_t *__restrict__ pos, const int32_t *__restrict__ k_start,
                     const int32_t *__restrict__ k_len, TileSum *__restrict__ out,
-                    int max_k_tiles, int64_t total_rows, int32_t *status) {
+                    TileMasks *__restrict__ masks_out, int max_k_tiles, int64_t total_rows,
+                    int32_t *status) {
     const int t = blockIdx.x, b = blockIdx.y;
     const int len_in = k_len[b];
     // a sequence outside the arrays (or longer than the tiles) gets empty summaries
@@ -76,9 +270,12 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
     int flags = 0, bmin = INT_MAX, bmax = INT_MIN, nmin = INT_MAX, nmax = INT_MIN, n = 0;
     int pmin = INT_MAX, pmax = INT_MIN;
     const int ro = r < len ? role[k_start[b] + r] : 255;
+    int sv = 0, pv = INT_MAX;  // padding: no segment, no position
     if (ro != 255) {
         const int s = seg[k_start[b] + r];
-        pmin = pmax = pos ? pos[k_start[b] + r] : r;
+        sv = s;
+        pv = pos ? pos[k_start[b] + r] : r;
+        pmin = pmax = pv;
         n = 1;
         if (ro == SONIC_ROLE_BODY) {
             flags = 1;
@@ -136,88 +333,25 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
         }
         out[(int64_t)b * max_k_tiles + t] = ts;
     }
-}
-
-struct PfParams {
-    // query side: the sequences as given (S_aug order)
-    const int32_t *k_start, *k_len, *q_start, *q_len;
-    const uint8_t *role;
-    const int32_t *seg;
-    // key side: the same arrays, or their retained-first permutation
-    const int32_t *key_start, *key_len;
-    const uint8_t *key_role;
-    const int32_t *key_seg;
-    const int32_t *key_pos;  // S_aug position of each key row; NULL: the row index
-    uint16_t *O;
-    float *lse;
-    float *nexus_mass;
-    int32_t *status;
-    const TileSum *sums;
-    int max_k_tiles, max_k_len;
-    int B, Hq, G;
-    int64_t total_k_rows;  // rows of role, seg_id (and K, V) per layer
-    int pack_log2;  // query heads per tile row group: a tile is 128 >> pack_log2 rows x (1 << pack_log2) heads
-    int64_t o_ls;
-    int total_q_rows;
-    float scale_log2;
-    int nexus_mode;
-};
-
-template <int D>
-struct PfCfg {
-    static constexpr int kHalves = D / 64;
-    static constexpr int kQBytes = kBM * D * 2;  // one 128-row Q tile
-    static constexpr int kKVBytes = kBN * D * 2;
-    static constexpr int kOffQ = 0;                           // [2] Q tiles
-    static constexpr int kOffK = kOffQ + 2 * kQBytes;         // [2] stages
-    static constexpr int kOffV = kOffK + 2 * kKVBytes;        // [2] stages
-    static constexpr int kOffMask = kOffV + 2 * kKVBytes;     // [2] TileMasks
-    static constexpr int kOffRole = kOffMask + 2 * 256;       // [2][128] uint8
-    static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
-    static constexpr int kOffPos = kOffSeg + 2 * kBN * 4;     // [2][128] int32
-    static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [kMaxKTiles] int32
-    static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
-    static constexpr int kNumBars = 16;
-    static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 32 ints
-    static constexpr int kBytes = kOffMisc + 32 * 4;
-    static constexpr size_t kSmem = 1024 + kBytes;
-};
-
-// Column masks of one 128-key tile (bit c of word w = key 32 w + c of the
-// tile): keys that are not body rows (nb), Nexus keys (nx), and the keys of
-// each distinct segment among the body keys (bm) and among the Nexus keys
-// (nm, used by the causal-segments reading); and the valid keys as runs of
-// consecutive S_aug positions (a tile's valid keys are a prefix of its rows
-// with increasing positions, so the keys at or before a position form a
-// prefix too, whose length the runs give).  With them a row's visibility
-// mask costs a few word operations.  More than four distinct segments or
-// position runs in one tile set `fallback`: the rule is then evaluated per
-// key instead.
-struct TileMasks {
-    uint32_t nb[4], nx[4];
-    int32_t nbody, nnex, fallback, nrun;
-    int32_t bseg[4], nseg[4];
-    uint32_t bm[4][4], nm[4][4];
-    // the valid keys as runs of consecutive S_aug positions, in column order
-    int32_t rpos[4], rlen[4];
-};
-static_assert(sizeof(TileMasks) <= 256, "tile masks");
-
-// Column of the n-th (from 0) set bit of a 128-bit mask, or -1.
-__device__ __forceinline__ int nth_set_bit(const uint32_t m[4], int n) {
-    int col = -1;
+    // The tile's column masks, built here once per key tile rather than by
+    // every block whose query tile the key tile cuts.
+    __shared__ int s_ro[kBN], s_sg[kBN], s_ps[kBN];
+    s_ro[threadIdx.x] = ro;
+    s_sg[threadIdx.x] = sv;
+    s_ps[threadIdx.x] = pv;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        int r4[4], s4[4], p4[4];
 #pragma unroll
-    for (int w = 0; w < 4; ++w) {
-        const int c = __popc(m[w]);
-        if (col < 0 && n < c) {
-            uint32_t x = m[w];
-            for (int i = 0; i < n; ++i) x &= x - 1;
-            col = w * 32 + __ffs(x) - 1;
+        for (int k = 0; k < 4; ++k) {
+            r4[k] = s_ro[k * 32 + threadIdx.x];
+            s4[k] = s_sg[k * 32 + threadIdx.x];
+            p4[k] = s_ps[k * 32 + threadIdx.x];
         }
-        if (col < 0) n -= c;
+        build_tile_masks(r4, s4, p4, threadIdx.x, masks_out + (int64_t)b * max_k_tiles + t);
     }
-    return col;
 }
+
 
 __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, int sq,
                                         int mode) {
@@ -425,139 +559,39 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                 hh * 64, kvh, row, layer);
                 }
             }
-            // Roles / segments / S_aug positions of the tile's keys (lane = key
-            // within each 32-key word; role 255 marks padding and rows past the
-            // sequence) and their masks: needed only where a query tile is cut.
-            if ((list[i] & 3) == 0) {
-                if (kMass && ((list[i] >> 2) & 3) == 2) {
-                    // an uncut tile with some Nexus keys: their bits only
+            // The tile's column masks (built once per key tile by the summary
+            // kernel; 8 bytes per lane) where a query tile is cut or the Nexus
+            // mass needs the Nexus bits; the keys' roles / segments / S_aug
+            // positions only where the masks fall back to the per-key rule.
+            const bool cut_any = (list[i] & 3) != 0;
+            if (cut_any || (kMass && ((list[i] >> 2) & 3) == 2)) {
+                const uint2 mw =
+                    reinterpret_cast<const uint2 *>(p.masks + (int64_t)b * p.max_k_tiles + kt)[lane];
+                reinterpret_cast<uint2 *>(tmasks + st)[lane] = mw;
+                // word 10 of the record (lane 5's first word): fallback
+                const int fallback = __shfl_sync(0xffffffffu, (int)mw.x, 5);
+                if (cut_any && fallback) {
+                    int ro[4], sg[4], ps[4];
+                    // all twelve loads first, none waiting on another
 #pragma unroll
                     for (int w = 0; w < 4; ++w) {
                         const int q = kt * kBN + w * 32 + lane;
-                        const bool isn =
-                            q < kklen && p.key_role[kkstart + q] == SONIC_ROLE_NEXUS;
-                        const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
-                        if (lane == 0) tmasks[st].nx[w] = nxw;
+                        const bool in = q < kklen;
+                        ro[w] = in ? p.key_role[kkstart + q] : 255;
+                        sg[w] = in ? p.key_seg[kkstart + q] : 0;
+                        ps[w] = in ? (p.key_pos != nullptr ? p.key_pos[kkstart + q] : q) : INT_MAX;
                     }
-                    __syncwarp();
-                }
-                mbar_arrive(&meta_full[st]);
-                continue;
-            }
-            int ro[4], sg[4], ps[4];
-            uint32_t bst[4], nst[4], rst[4];
-            int pro = 255, psg = 0, pps = INT_MIN, n_valid = 0;
-            TileMasks &tm = tmasks[st];
-            // all twelve loads first, none waiting on another: one memory
-            // latency per tile instead of eight in a row
 #pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                const int q = kt * kBN + w * 32 + lane;
-                const bool in = q < kklen;
-                ro[w] = in ? p.key_role[kkstart + q] : 255;
-                sg[w] = in ? p.key_seg[kkstart + q] : 0;
-                ps[w] = in ? (p.key_pos != nullptr ? p.key_pos[kkstart + q] : q) : INT_MAX;
-            }
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                const int c = w * 32 + lane;
-                if (ro[w] == 255) {  // padding: no segment, no position
-                    sg[w] = 0;
-                    ps[w] = INT_MAX;
-                }
-                meta_role[st * kBN + c] = (uint8_t)ro[w];
-                meta_seg[st * kBN + c] = sg[w];
-                meta_pos[st * kBN + c] = ps[w];
-                const bool valid = ro[w] != 255;
-                const bool isb = ro[w] == SONIC_ROLE_BODY, isn = ro[w] == SONIC_ROLE_NEXUS;
-                const uint32_t nbw = __ballot_sync(0xffffffffu, valid && !isb);
-                const uint32_t nxw = __ballot_sync(0xffffffffu, isn);
-                n_valid += __popc(__ballot_sync(0xffffffffu, valid));
-                // previous key's role/segment/position (lane 0: last key of the
-                // previous word)
-                int r_up = __shfl_up_sync(0xffffffffu, ro[w], 1);
-                int s_up = __shfl_up_sync(0xffffffffu, sg[w], 1);
-                int p_up = __shfl_up_sync(0xffffffffu, ps[w], 1);
-                if (lane == 0) {
-                    r_up = pro;
-                    s_up = psg;
-                    p_up = pps;
-                }
-                bst[w] = __ballot_sync(0xffffffffu, isb && !(r_up == SONIC_ROLE_BODY && s_up == sg[w]));
-                nst[w] = __ballot_sync(0xffffffffu, isn && !(r_up == SONIC_ROLE_NEXUS && s_up == sg[w]));
-                rst[w] = __ballot_sync(0xffffffffu, valid && p_up != ps[w] - 1);
-                pro = __shfl_sync(0xffffffffu, ro[w], 31);
-                psg = __shfl_sync(0xffffffffu, sg[w], 31);
-                pps = __shfl_sync(0xffffffffu, ps[w], 31);
-                if (lane == 0) {
-                    tm.nb[w] = nbw;
-                    tm.nx[w] = nxw;
-                }
-            }
-            // distinct segments of body runs and Nexus runs, and the position
-            // runs (all in key order)
-            int nb_n = 0, nn_n = 0, fb = 0;
-            int bsv[4] = {0, 0, 0, 0}, nsv[4] = {0, 0, 0, 0};
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                uint32_t m = bst[w];
-                while (m) {
-                    const int bl = __ffs(m) - 1;
-                    m &= m - 1;
-                    const int v = __shfl_sync(0xffffffffu, sg[w], bl);
-                    bool seen = false;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) seen |= (k < nb_n && bsv[k] == v);
-                    if (!seen) {
-                        if (nb_n < 4) bsv[nb_n++] = v; else fb = 1;
+                    for (int w = 0; w < 4; ++w) {
+                        const int c = w * 32 + lane;
+                        const bool pad = ro[w] == 255;  // no segment, no position
+                        meta_role[st * kBN + c] = (uint8_t)ro[w];
+                        meta_seg[st * kBN + c] = pad ? 0 : sg[w];
+                        meta_pos[st * kBN + c] = pad ? INT_MAX : ps[w];
                     }
                 }
-                m = nst[w];
-                while (m) {
-                    const int bl = __ffs(m) - 1;
-                    m &= m - 1;
-                    const int v = __shfl_sync(0xffffffffu, sg[w], bl);
-                    bool seen = false;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) seen |= (k < nn_n && nsv[k] == v);
-                    if (!seen) {
-                        if (nn_n < 4) nsv[nn_n++] = v; else fb = 1;
-                    }
-                }
+                __syncwarp();
             }
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    const uint32_t bmw = __ballot_sync(
-                        0xffffffffu, k < nb_n && ro[w] == SONIC_ROLE_BODY && sg[w] == bsv[k]);
-                    const uint32_t nmw = __ballot_sync(
-                        0xffffffffu, k < nn_n && ro[w] == SONIC_ROLE_NEXUS && sg[w] == nsv[k]);
-                    if (lane == 0) {
-                        tm.bm[k][w] = bmw;
-                        tm.nm[k][w] = nmw;
-                    }
-                }
-            if (lane == 0) {
-                tm.nbody = nb_n;
-                tm.nnex = nn_n;
-                tm.nrun = __popc(rst[0]) + __popc(rst[1]) + __popc(rst[2]) + __popc(rst[3]);
-                tm.fallback = fb | (tm.nrun > 4);
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    tm.bseg[k] = bsv[k];
-                    tm.nseg[k] = nsv[k];
-                }
-            }
-            // position run k (lane k < 4): from the k-th run start to the next
-            // one (or to the last valid key); the start's position from smem
-            __syncwarp();
-            if (lane < 4) {
-                const int c0 = nth_set_bit(rst, lane), c1 = nth_set_bit(rst, lane + 1);
-                tm.rpos[lane] = c0 < 0 ? 0 : meta_pos[st * kBN + c0];
-                tm.rlen[lane] = c0 < 0 ? 0 : (c1 < 0 ? n_valid : c1) - c0;
-            }
-            __syncwarp();
             mbar_arrive(&meta_full[st]);  // 32 arrivals end the phase
         }
         if (lane == 0 && *abort_flag) {
@@ -1125,16 +1159,18 @@ int max_k_tiles_of(const sonic_prefill_args *a) {
     return a->key_order == SONIC_KEYS_RETAINED_FIRST ? t + 1 : t;
 }
 
-// Workspace: tile summaries; with the retained-first order also the
-// permuted key metadata and the permuted K and V of every layer.
+// Workspace: tile summaries and tile column masks; with the retained-first
+// order also the permuted key metadata and the permuted K and V of every layer.
 struct PfWorkspace {
-    size_t sums, key_start, key_len, role, seg, pos, src, kp, vp, total;
+    size_t sums, masks, key_start, key_len, role, seg, pos, src, kp, vp, total;
     int64_t rows;  // rows of the permuted K/V per layer
 };
 
 PfWorkspace workspace_layout(const sonic_prefill_args *a) {
     PfWorkspace w{};
-    size_t off = round_up((size_t)a->batch * max_k_tiles_of(a) * sizeof(TileSum), 256);
+    const size_t tiles = (size_t)a->batch * max_k_tiles_of(a);
+    w.masks = round_up(tiles * sizeof(TileSum), 256);
+    size_t off = w.masks + round_up(tiles * sizeof(TileMasks), 256);
     if (a->key_order == SONIC_KEYS_RETAINED_FIRST) {
         const int64_t span = (int64_t)((a->max_k_len + kBN - 1) / kBN) * kBN + kBN;
         w.rows = std::min<int64_t>((int64_t)a->batch * span,
@@ -1269,6 +1305,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.nexus_mass = a->nexus_mass;
     p.status = a->status;
     p.sums = static_cast<const TileSum *>(a->workspace);
+    p.masks = reinterpret_cast<const TileMasks *>(wsb + ws.masks);
     p.max_k_tiles = max_k_tiles_of(a);
     p.max_k_len = a->max_k_len;
     p.B = a->batch;
@@ -1300,7 +1337,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     }
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
         p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
-        static_cast<TileSum *>(a->workspace), p.max_k_tiles,
+        static_cast<TileSum *>(a->workspace), reinterpret_cast<TileMasks *>(wsb + ws.masks),
+        p.max_k_tiles,
         reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status);
     dim3 grid((unsigned)qtiles, a->n_heads_q >> pack_log2, a->batch * a->n_layers);
     cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)

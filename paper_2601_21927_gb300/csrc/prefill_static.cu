@@ -20,10 +20,10 @@
 
 namespace {
 
-// 1 MiB: room for 32768 per-tile summaries of 32 bytes, i.e.
-// batch * ceil(max_k_len / 128) <= 32768 (for example 64 sequences of up
-// to 65536 keys).
-constexpr size_t kStaticScratchBytes = size_t(1) << 20;
+// 9 MiB: room for 32768 key tiles, each with a 32-byte summary and a
+// 256-byte column-mask record, i.e. batch * ceil(max_k_len / 128) <= 32768
+// (for example 64 sequences of up to 65536 keys).
+constexpr size_t kStaticScratchBytes = size_t(9) << 20;
 
 static __device__ __align__(256) unsigned char g_prefill_scratch[kStaticScratchBytes];
 
