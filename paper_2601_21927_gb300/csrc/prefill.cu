@@ -1328,7 +1328,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
             reinterpret_cast<int32_t *>(wsb + ws.seg), reinterpret_cast<int32_t *>(wsb + ws.pos),
             reinterpret_cast<int32_t *>(wsb + ws.src), a->status);
         const int sms = device_sm_count();
-        const int per_slice = std::max(1, (sms * 8 + 2 * a->n_layers - 1) / (2 * a->n_layers));
+        // ~32 blocks per SM in all, as in the compaction copy
+        const int per_slice = std::max(1, (sms * 32 + 2 * a->n_layers - 1) / (2 * a->n_layers));
         kv_permute_kernel<<<dim3(per_slice, 2 * a->n_layers), kPermThreads, 0, stream>>>(
             reinterpret_cast<const uint8_t *>(K), reinterpret_cast<const uint8_t *>(V),
             wsb + ws.kp, wsb + ws.vp, reinterpret_cast<const int32_t *>(wsb + ws.src),
