@@ -56,6 +56,17 @@ def test_retained_first_many_runs_per_tile(mode):
     _all_rows(inputs.Batch(ds), 4, 1, 128, mode=mode, seed=13, order=sonic.KEYS_RETAINED_FIRST)
 
 
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+def test_as_given_many_segments_per_tile(mode):
+    """Key order as given with segments of 10-20 tokens: most 128-key tiles
+    hold more than four body segments and more than four position runs of
+    Nexus keys, so their column-mask records fall back to the per-key rule and
+    the producer stages the keys' roles, segments and positions."""
+    ds = [inputs.Dialogue(3, [(9, 3), (7, 6), (11, 4)] * 12, 37),
+          inputs.Dialogue(17, [(5, 5)] * 30, 60)]
+    _all_rows(inputs.Batch(ds), 4, 2, 128, mode=mode, seed=17, order=sonic.KEYS_AS_GIVEN)
+
+
 @pytest.mark.parametrize("order", ORDERS)
 @pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
 def test_uniform_scores_count_visible_keys(mode, order):
