@@ -229,8 +229,10 @@ SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K
 
 /*
  * Workspace bytes for sonic_attn_prefill with these arguments (0 for an empty
- * batch).  AS_GIVEN: 32 bytes per 128-key tile, batch * ceil(max_k_len / 128)
- * tiles.  RETAINED_FIRST adds, for R = min(batch * (align128(max_k_len) + 128),
+ * batch).  AS_GIVEN: 32 + 256 bytes per 128-key tile (its summary and its
+ * column masks), batch * ceil(max_k_len / 128) tiles, each part rounded up to
+ * 256 bytes.  RETAINED_FIRST counts one more tile per sequence and adds, for
+ * R = min(batch * (align128(max_k_len) + 128),
  * total_k_rows + 256 * batch) rows: 13 bytes of metadata per row and a K and
  * a V copy of R rows for every layer (2 * n_layers * R * n_heads_kv *
  * head_dim * 2 bytes).  Sequence b takes align128(k_len[b]) + 128 of the R
