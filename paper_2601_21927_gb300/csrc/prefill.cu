@@ -403,7 +403,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint64_t *mma_idle = bars + 11;
     uint64_t *meta_full = bars + 12;  // [2] key metadata of a stage written
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
-    // misc: 0 tmem base, 2 abort, 4..13 query-tile summaries (5 per tile),
+    // misc: 0 tmem base, 2 abort, 3 key tile 0 copied early, 4..13 query-tile
+    //       summaries (5 per tile),
     //       16..27 per-warp counts
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
 
@@ -461,6 +462,25 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     // ------------------------------------------------ summaries of the query tiles
     if (tid < 10) misc[4 + tid] = (tid % 5 == 0) ? 0 : ((tid % 5) & 1 ? INT_MAX : INT_MIN);
     __syncthreads();
+    if (tid == kPfThreads - 32) {  // a thread the summaries below leave idle
+        // Key tile 0 comes first in the tile list whenever one of its non-body
+        // keys is at or before the last row of query tile 0 (that alone lists
+        // it): its K/V copy then starts now, ahead of the list.
+        int early = 0;
+        if (kklen > 0) {
+            const TileSum ts0 = p.sums[(int64_t)b * p.max_k_tiles];
+            early = (ts0.flags & 6) != 0 && ts0.pos_min <= min(pbase + R - 1, klen - 1);
+        }
+        if (early) {
+            mbar_arrive_expect_tx(&kv_full[0], 2 * C::kKVBytes);
+#pragma unroll
+            for (int hh = 0; hh < C::kHalves; ++hh) {
+                tma_load_4d(Ks + hh * (kBN * 128), &tmK, &kv_full[0], hh * 64, kvh, kkstart, layer);
+                tma_load_4d(Vs + hh * (kBN * 128), &tmV, &kv_full[0], hh * 64, kvh, kkstart, layer);
+            }
+        }
+        misc[3] = early;
+    }
     if (tid < 2 * R && pbase + tid <= klen - 1) {
         int32_t *qs = misc + 4 + 5 * (tid >= R ? 1 : 0);  // flags, seg min/max, nexus min/max
         const int ro = p.role[kstart + pbase + tid];
@@ -548,7 +568,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             // K/V copies first; the key metadata is built while they are in flight
             // and has a barrier of its own, so the S MMA of a cut tile waits for
             // the copy alone, not for the metadata
-            if (lane == 0) {
+            if (lane == 0 && !(i == 0 && misc[3])) {
                 mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
                 const int row = kkstart + kt * kBN;
 #pragma unroll
