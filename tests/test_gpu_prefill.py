@@ -56,6 +56,23 @@ def test_retained_first_many_runs_per_tile(mode):
     _all_rows(inputs.Batch(ds), 4, 1, 128, mode=mode, seed=13, order=sonic.KEYS_RETAINED_FIRST)
 
 
+@pytest.mark.parametrize("order", ORDERS)
+def test_first_key_tile_not_listed_first(order):
+    """No system prompt and a 300-token first body: as given, key tile 0 holds
+    body rows only, which the current turn's rows never see, so the first
+    listed tile is a later one and key tile 0's copy must not start early;
+    all rows (tile 0 then seen by its own segment's rows) and current rows only."""
+    ds = [inputs.Dialogue(0, [(300, 4), (50, 3)], 40), inputs.Dialogue(0, [(260, 0), (9, 9)], 200)]
+    batch = inputs.Batch(ds)
+    _all_rows(batch, 4, 2, 128, seed=23, order=order)
+    q_len = np.array([40, 200], dtype=np.int32)
+    res = H.run_prefill(batch, 4, 2, 128, q_len=q_len, seed=29, key_order=order)
+    for b in range(batch.B):
+        O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, np.arange(q_len[b]))
+        H.check_close(got, O, f"seq {b}")
+        np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
+
+
 @pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
 def test_as_given_many_segments_per_tile(mode):
     """Key order as given with segments of 10-20 tokens: most 128-key tiles
