@@ -256,8 +256,10 @@ SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
  *    is served (RETAINED_FIRST copies K and V into the workspace):
  *    SONIC_ERR_UNSUPPORTED otherwise.
  *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress, with that device current) and caches it; make
- *    that first call before any stream capture.
+ *    (cudaGetSymbolAddress, with that device current) and caches it with the
+ *    id of the device's current context; make that first call before any
+ *    stream capture.  After a device reset the context id differs, so the
+ *    next call looks the address up again (make it outside a capture too).
  *  - Every call on a device shares the one array and leaves its contents
  *    behind; each call rewrites every entry it reads, so nothing needs
  *    clearing, but calls that overlap on the GPU (other streams, other host

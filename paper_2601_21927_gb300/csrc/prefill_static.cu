@@ -13,7 +13,12 @@
 // library holds it until the process exits.  In host code its name is only a
 // host-side stand-in, so its device address is looked up with
 // cudaGetSymbolAddress once per device (with that device current) on the
-// first call made on that device, and cached.
+// first call made on that device, and cached together with the unique id of
+// the context it belongs to.  A device reset destroys that context and the
+// module loaded into it; the next call sees a different context id and looks
+// the address up again instead of handing the kernels a dead address.
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "sonic_host.h"
@@ -29,19 +34,51 @@ static __device__ __align__(256) unsigned char g_prefill_scratch[kStaticScratchB
 
 constexpr int kMaxDevices = 64;
 void *g_scratch_ptr[kMaxDevices] = {nullptr};
+unsigned long long g_scratch_ctx[kMaxDevices] = {0};
 std::mutex g_scratch_mu;
 
-// Device address of the scratch array on the current device (looked up once).
+// Unique id of the calling thread's current context (0 when there is none or
+// the driver cannot say).  Ids are never reused within a process.
+unsigned long long current_context_id() {
+    static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+    static PFN_cuCtxGetId_v12000 get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+    });
+    if (get_current == nullptr || get_id == nullptr) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+    if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of the scratch array on the current device: looked up once
+// per device and context, then served from the cache.
 sonic_status_t scratch_address(void **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return SONIC_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return SONIC_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (g_scratch_ptr[dev] == nullptr) {
+    const unsigned long long ctx = current_context_id();
+    if (g_scratch_ptr[dev] == nullptr || ctx == 0 || ctx != g_scratch_ctx[dev]) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_prefill_scratch) != cudaSuccess || p == nullptr)
             return SONIC_ERR_CUDA;
         g_scratch_ptr[dev] = p;
+        // the lookup made the device's primary context current if it was not
+        g_scratch_ctx[dev] = current_context_id();
     }
     *out = g_scratch_ptr[dev];
     return SONIC_OK;

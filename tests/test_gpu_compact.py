@@ -122,6 +122,29 @@ def test_masked_prefill_workload_all_layers():
             assert np.array_equal(_bytes(r[name][layer:layer + 1]), want), f"{name} layer {layer}"
 
 
+@pytest.mark.parametrize("nexus_div", [2, 5])
+def test_long_ragged_histories_two_layers(nexus_div):
+    """The 64 long ragged dialogues (turns ~U[4,32] of ~U[64,1024] tokens, 256
+    system tokens, Nexus = ceil(len/2) or ceil(len/5) per history turn, 8 KV
+    heads, D = 128): their raw S_aug rows compacted for two layers, offsets,
+    source rows and every byte of both layers checked."""
+    batch, hd = inputs.long_ragged(nexus_div)
+    shape = (2, batch.total, hd.hkv, hd.d)
+    K = inputs.randn(shape, seed=50 + nexus_div, device=H.dev())
+    V = inputs.randn(shape, seed=60 + nexus_div, device=H.dev())
+    r = _run(batch, K, V, want_meta=False)
+    assert r["status"] == 0
+    off, ret_len, src = oracle.retain(batch.k_start, batch.k_len, batch.role)
+    assert r["offsets"].cpu().numpy().tolist() == off.tolist()
+    assert ret_len.tolist() == [d.recipe_retained for d in batch.dialogues]
+    np.testing.assert_array_equal(r["src_idx"].cpu().numpy(), src)
+    for layer in (0, 1):
+        for name, raw in (("oK", K), ("oV", V)):
+            want = oracle.compact_copy(_bytes(raw[layer:layer + 1]), off, ret_len, src,
+                                       int(off[-1]))
+            assert np.array_equal(_bytes(r[name][layer:layer + 1]), want), f"{name} layer {layer}"
+
+
 def test_many_sequences_and_long_pieces():
     """1,100 sequences (the base scan runs over more than one 512-wide block
     pass) plus one sequence of about 70,000 rows (each of its 64 scan pieces

@@ -89,11 +89,14 @@ def test_head_shapes(hq, hkv, D):
     _check(r, [(0, b) for b in range(3)])
 
 
-def test_long_ragged_workload_sampled():
-    """Batch 64 ragged dialogues (Nexus = ceil(len/2)), 32 layers, 32/8 heads."""
-    batch, hd = inputs.long_ragged(2)
+@pytest.mark.parametrize("nexus_div", [2, 5])
+def test_long_ragged_workload_sampled(nexus_div):
+    """Batch 64 ragged dialogues, 32/8 heads, D = 128, both Nexus budgets:
+    ceil(len/2) (50% compression) and ceil(len/5) (80%, Sec. 6 Table 1
+    caption); sampled layers and sequences of a 4-layer launch."""
+    batch, hd = inputs.long_ragged(nexus_div)
     lens = np.array([d.recipe_retained + 1 for d in batch.dialogues])
-    r = _decode(lens, hd.hq, hd.hkv, hd.d, n_layers=4, seed=13, pad=0)
+    r = _decode(lens, hd.hq, hd.hkv, hd.d, n_layers=4, seed=13 + nexus_div, pad=0)
     _check(r, [(l, b) for l in (0, 3) for b in (0, 7, 31, 63)])
     assert torch.isfinite(r["O"]).all()
 
