@@ -229,7 +229,8 @@ SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K
 
 /*
  * Workspace bytes for sonic_attn_prefill with these arguments (0 for an empty
- * batch).  AS_GIVEN: 32 + 256 bytes per 128-key tile (its summary and its
+ * batch).  AS_GIVEN: 256 bytes for the counter the persistent blocks claim
+ * work units from, then 32 + 256 bytes per 128-key tile (its summary and its
  * column masks), batch * ceil(max_k_len / 128) tiles, each part rounded up to
  * 256 bytes.  RETAINED_FIRST counts one more tile per sequence and adds, for
  * R = min(batch * (align128(max_k_len) + 128),
@@ -249,8 +250,9 @@ SONIC_API size_t sonic_prefill_workspace_size(const sonic_prefill_args *args);
  * only hand over fixed buffers for inputs and outputs.  This call takes the
  * same arguments as sonic_attn_prefill except that args->workspace and
  * args->workspace_bytes are ignored: the per-tile summaries and column masks
- * live in a fixed 9 MiB array compiled into the library (every GPU that loads
- * the library holds it until the process exits).  It allocates nothing.
+ * live in a fixed array of 9 MiB + 256 bytes compiled into the library
+ * (every GPU that loads the library holds it until the process exits).  It
+ * allocates nothing.
  *  - Limit: batch * ceil(max_k_len / 128) <= 32768; larger calls return
  *    SONIC_ERR_WORKSPACE before launching anything.  Only key_order AS_GIVEN
  *    is served (RETAINED_FIRST copies K and V into the workspace):

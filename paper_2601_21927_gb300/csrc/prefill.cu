@@ -2,10 +2,12 @@
 // mask (Sec. 3.2: Eq. 3 causal rule, Eq. 4 historical body removal, Eq. 5
 // bidirectional Nexus visibility), on the sm_103a tensor cores.
 //
-// One block computes two 128-row query tiles of one (layer, sequence, query
-// head).  Ten warps:
-//   warp 0     TMA producer: the Q tiles once, then K and V tiles (128 keys)
-//              into a 2-stage ring, with the role/segment numbers of the keys;
+// A work unit is two 128-row query tiles of one (layer, sequence, query head
+// group).  One persistent block per SM claims units from a counter; eleven
+// warps:
+//   warp 0     TMA producer: each unit's Q tiles, then K and V tiles (128
+//              keys) into a 2-stage ring, with the column masks of the tiles
+//              the mask cuts;
 //   warp 1     tcgen05 issuer: S_t = Q_t K^T into TMEM (fp32, 128 lanes x 128
 //              columns per tile), and O_t += P_t V with P read from TMEM, one
 //              elected thread issuing every MMA;
@@ -14,11 +16,15 @@
 //              the mask per element only on tiles the mask cuts, runs the
 //              online softmax in base 2, rescales its O row in TMEM when the
 //              running maximum has risen by more than 2^8, and writes P (bf16
-//              pairs) back over its S columns.
-// Before the loop the block lists the key tiles it must visit: each tile is
-// classified from precomputed per-tile summaries (which roles and segment
-// numbers occur in it) as hidden (skipped entirely), fully visible (no mask
-// work) or cut by the mask.  The two tiles' softmax and MMAs interleave.
+//              pairs) back over its S columns;
+//   warp 10    scheduler: ahead of the others, claims the next unit and lists
+//              the key tiles each of its query tiles must visit, classified
+//              from precomputed per-tile summaries (which roles, segment
+//              numbers and positions occur in a key tile) as hidden (skipped
+//              entirely), fully visible (no mask work) or cut by the mask.
+// The two query tiles' softmax and MMAs interleave, and consecutive units of
+// a block overlap: the next unit's first S products run while the softmax
+// warps finish the previous one.
 #include <algorithm>
 #include <cstddef>
 #include <type_traits>
@@ -31,7 +37,11 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kPfThreads = 320;
+constexpr int kPfThreads = 352;
+constexpr int kSchedWarp = 10;
+// warps done with a unit slot before the scheduler refills it: the producer
+// warp, the issuing thread and the eight softmax warps
+constexpr int kUnitConsumers = 10;
 constexpr int kMaxKTiles = 2048;
 constexpr float kLn2f = 0.6931471805599453f;
 constexpr float kLog2ef = 1.4426950408889634f;
@@ -80,6 +90,8 @@ struct PfParams {
     int32_t *status;
     const TileSum *sums;
     const TileMasks *masks;  // per key tile, from the summary kernel
+    int32_t *counter;        // next work unit to claim (zeroed by the summary kernel)
+    int n_units, qtiles, HG; // units = qtiles x HG x B x n_layers; HG = Hq >> pack_log2
     int max_k_tiles, max_k_len;
     int B, Hq, G;
     int64_t total_k_rows;  // rows of role, seg_id (and K, V) per layer
@@ -89,6 +101,18 @@ struct PfParams {
     float scale_log2;
     int nexus_mode;
 };
+
+// One work unit as the scheduler publishes it.
+struct UnitInfo {
+    int32_t flags;  // bit 0: no unit is left; bit 1: every query tile visits every listed key tile
+    int32_t layer, b, h0, qt;
+    int32_t nq;      // query tiles with rows: 1 or 2
+    int32_t n_list;  // key tiles listed
+    int32_t kstart, klen, kkstart, kklen, qstart, qlen;
+    int32_t pbase;    // S_aug position of query row 0 of tile 0
+    int32_t last[2];  // list index of the last key tile each query tile visits (-1: none)
+};
+static_assert(sizeof(UnitInfo) == 64, "unit record: 64 bytes");
 
 template <int D>
 struct PfCfg {
@@ -102,11 +126,12 @@ struct PfCfg {
     static constexpr int kOffRole = kOffMask + 2 * 256;       // [2][128] uint8
     static constexpr int kOffSeg = kOffRole + 2 * kBN;        // [2][128] int32
     static constexpr int kOffPos = kOffSeg + 2 * kBN * 4;     // [2][128] int32
-    static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [kMaxKTiles] int32
-    static constexpr int kOffBar = kOffList + kMaxKTiles * 4;
-    static constexpr int kNumBars = 16;
-    static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 32 ints
-    static constexpr int kBytes = kOffMisc + 32 * 4;
+    static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [2 units][kMaxKTiles] int32
+    static constexpr int kOffUnit = kOffList + 2 * kMaxKTiles * 4;  // [2] UnitInfo
+    static constexpr int kOffBar = kOffUnit + 2 * (int)sizeof(UnitInfo);
+    static constexpr int kNumBars = 24;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 16 ints
+    static constexpr int kBytes = kOffMisc + 16 * 4;
     static constexpr size_t kSmem = 1024 + kBytes;
 };
 
@@ -259,8 +284,10 @@ tile_summary_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict_
                     const int32_t *__restrict__ pos, const int32_t *__restrict__ k_start,
                     const int32_t *__restrict__ k_len, TileSum *__restrict__ out,
                     TileMasks *__restrict__ masks_out, int max_k_tiles, int64_t total_rows,
-                    int32_t *status) {
+                    int32_t *status, int32_t *unit_counter) {
     const int t = blockIdx.x, b = blockIdx.y;
+    // the attention kernel that follows claims its work units from 0
+    if (t == 0 && b == 0 && threadIdx.x == 0) *unit_counter = 0;
     const int len_in = k_len[b];
     // a sequence outside the arrays (or longer than the tiles) gets empty summaries
     const int len = seq_rows(k_start[b], len_in, max_k_tiles * kBN, total_rows);
@@ -365,19 +392,95 @@ __device__ __forceinline__ bool visible(int p, int q, int rp, int sp, int rq, in
 // rescaling O: probabilities stay below 2^8 until the next rescale.
 constexpr float kRescaleThreshold = 8.0f;
 
-// Two 128-row query tiles (tile 0 = rows 0..127 of the block's 256, tile 1 =
-// rows 128..255) share every K/V tile.  Warp roles (320 threads, so every
-// thread can hold a full 128-column S row in registers):
-//   warp 0       TMA producer (K, V, Q) and key metadata,
-//   warp 1       tcgen05 issuer and TMEM owner,
-//   warps 2-5    softmax of tile 0, warps 6-9 softmax of tile 1 (warp w
-//                reaches TMEM lanes 32 * (w % 4) .. + 31).
+// The 128-bit visibility mask of query row `pos` (role rp, segment sp) over a
+// cut key tile: from the tile's column masks, or per key from its staged
+// roles / segments / positions where the masks fall back to the per-key rule.
+__device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8_t *mrole,
+                                               const int32_t *mseg, const int32_t *mpos, int pos,
+                                               int rp, int sp, int nexus_mode,
+                                               uint32_t (&mbits)[4]) {
+    // the whole mask record in independent 16-byte loads
+    const uint4 *tv = reinterpret_cast<const uint4 *>(tmk);
+    const uint4 nb = tv[0], nx = tv[1], hd = tv[2], bsg = tv[3], nsg = tv[4];
+    uint4 bm[4], nm[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        bm[k] = tv[5 + k];
+        nm[k] = tv[9 + k];
+    }
+    if (!hd.z) {
+        // causal prefix (keys at or before this row: a prefix of the tile's
+        // columns, counted over the position runs), body keys of this row's
+        // segment, and the Nexus keys a Nexus row sees
+        const uint4 rp4 = tv[13], rl4 = tv[14];
+        const int nvis = min(max(pos - (int)rp4.x + 1, 0), (int)rl4.x) +
+                         min(max(pos - (int)rp4.y + 1, 0), (int)rl4.y) +
+                         min(max(pos - (int)rp4.z + 1, 0), (int)rl4.z) +
+                         min(max(pos - (int)rp4.w + 1, 0), (int)rl4.w);
+        const int nbody = (int)hd.x, nnex = (int)hd.y;
+        const int bs4[4] = {(int)bsg.x, (int)bsg.y, (int)bsg.z, (int)bsg.w};
+        const int ns4[4] = {(int)nsg.x, (int)nsg.y, (int)nsg.z, (int)nsg.w};
+        uint4 bw = make_uint4(0u, 0u, 0u, 0u), xw = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (k < nbody && bs4[k] == sp) {
+                bw.x |= bm[k].x; bw.y |= bm[k].y; bw.z |= bm[k].z; bw.w |= bm[k].w;
+            }
+            if (rp == SONIC_ROLE_NEXUS && nexus_mode != SONIC_NEXUS_FULL && k < nnex &&
+                ns4[k] <= sp) {
+                xw.x |= nm[k].x; xw.y |= nm[k].y; xw.z |= nm[k].z; xw.w |= nm[k].w;
+            }
+        }
+        if (rp == SONIC_ROLE_NEXUS && nexus_mode == SONIC_NEXUS_FULL) xw = nx;
+        const uint32_t nbw[4] = {nb.x, nb.y, nb.z, nb.w};
+        const uint32_t bww[4] = {bw.x, bw.y, bw.z, bw.w};
+        const uint32_t xww[4] = {xw.x, xw.y, xw.z, xw.w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const int nw = min(max(nvis - 32 * w, 0), 32);
+            const uint32_t cw = nw >= 32 ? 0xffffffffu : ((1u << nw) - 1u);
+            mbits[w] = (cw & (nbw[w] | bww[w])) | xww[w];
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint8_t *mr = mrole + c * 32;
+            const int32_t *ms = mseg + c * 32;
+            const int32_t *mp = mpos + c * 32;
+            uint32_t bits = 0;
+#pragma unroll 4
+            for (int e = 0; e < 32; ++e) {
+                const int rq = mr[e];
+                const bool v = rq != 255 && visible(pos, mp[e], rp, sp, rq, ms[e], nexus_mode);
+                bits |= (v ? 1u : 0u) << e;
+            }
+            mbits[c] = bits;
+        }
+    }
+}
+
+// One persistent block per SM walks work units: a unit is two 128-row query
+// tiles (tile 0 = rows 0..127 of its 256, tile 1 = rows 128..255) of one
+// (layer, sequence, query-head group).  Eleven warps (352 threads):
+//   warp 0       TMA producer: the unit's Q tiles, then K, V (and the key
+//                metadata of cut tiles) into a 2-stage ring that runs on
+//                across units;
+//   warp 1       tcgen05 issuer and TMEM owner;
+//   warps 2-5    softmax of query tile 0, warps 6-9 of query tile 1 (warp w
+//                reaches TMEM lanes 32 * (w % 4) .. + 31);
+//   warp 10      scheduler: claims the next unit from a counter, summarises
+//                its query tiles and lists the key tiles each of them must
+//                visit, up to two units ahead of the others.
 // TMEM (512 columns): S/P of tile 0 at 0, of tile 1 at 128, O of tile 0 at
-// 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns
-// of its S block and feeds O += P V straight from tensor memory.
+// 256, O of tile 1 at 384.  P (bf16 pairs) overwrites the first 64 columns of
+// its S block and feeds O += P V straight from tensor memory.  While the
+// softmax warps finish one unit (normalise O, write it out), the issuer
+// already runs the next unit's first S products: O is overwritten only after
+// the epilogue has read it (o_free), S/P only after the last P.V read it (the
+// tensor pipe runs in order).
 // kOut: bit 0 writes the log-sum-exp, bit 1 the attention mass on Nexus keys.
 template <int D, int kOut>
-__global__ void __launch_bounds__(kPfThreads, 1)
+__global__ void __maxnreg__(168)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const PfParams p) {
     using C = PfCfg<D>;
@@ -392,159 +495,55 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint8_t *meta_role = smem + C::kOffRole;
     int32_t *meta_seg = reinterpret_cast<int32_t *>(smem + C::kOffSeg);
     int32_t *meta_pos = reinterpret_cast<int32_t *>(smem + C::kOffPos);
-    int32_t *list = reinterpret_cast<int32_t *>(smem + C::kOffList);
+    int32_t *lists = reinterpret_cast<int32_t *>(smem + C::kOffList);  // [2][kMaxKTiles]
+    UnitInfo *units = reinterpret_cast<UnitInfo *>(smem + C::kOffUnit);  // [2]
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::kOffBar);
     uint64_t *q_full = bars + 0;
-    uint64_t *kv_full = bars + 1;   // [2]
-    uint64_t *kv_empty = bars + 3;  // [2]
-    uint64_t *s_full = bars + 5;    // [2] per query tile
-    uint64_t *p_full = bars + 7;    // [2] per query tile
-    uint64_t *o_done = bars + 9;    // [2] per query tile
-    uint64_t *mma_idle = bars + 11;
-    uint64_t *meta_full = bars + 12;  // [2] key metadata of a stage written
+    uint64_t *q_empty = bars + 1;
+    uint64_t *kv_full = bars + 2;     // [2] per ring stage
+    uint64_t *kv_empty = bars + 4;    // [2]
+    // [stage][query tile]: key metadata of a stage written, for a query tile
+    // that reads it (the key tile cuts the query tile, or has some Nexus keys
+    // and the Nexus mass is asked for).  A phase completes only for such
+    // tiles, so each softmax warpgroup waits every phase of its own barrier
+    // in turn, whatever key tiles it skips.
+    uint64_t *meta_full = bars + 6;   // [2][2]
+    uint64_t *s_full = bars + 10;     // [2] per query tile
+    uint64_t *p_full = bars + 12;     // [2]
+    uint64_t *o_done = bars + 14;     // [2]
+    uint64_t *o_free = bars + 16;     // [2]
+    uint64_t *unit_full = bars + 18;  // [2] per unit slot
+    uint64_t *unit_empty = bars + 20; // [2]
+    uint64_t *mma_idle = bars + 22;
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
-    // misc: 0 tmem base, 2 abort, 3 key tile 0 copied early, 4..13 query-tile
-    //       summaries (5 per tile),
-    //       16..27 per-warp counts
+    // misc: 0 tmem base, 2 abort
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
 
     // A query tile is R query rows x P heads of one KV group (P = 1 << pack_log2,
     // R = 128 / P): tile row r is query row r / P, head h0 + r % P.  P > 1 packs
     // the heads of short query blocks so the tile rows are not left empty.
     const int pl2 = p.pack_log2, R = kBM >> pl2;
-    const int qt = blockIdx.x, h0 = blockIdx.y << pl2;
-    const int b = blockIdx.z % p.B, layer = blockIdx.z / p.B;
-    const int klen = p.k_len[b], qlen = p.q_len[b];
-    if (p.k_start[b] < 0 || (int64_t)p.k_start[b] + klen > p.total_k_rows || p.q_start[b] < 0 ||
-        qlen < 0 || (int64_t)p.q_start[b] + qlen > p.total_q_rows) {
-        // rows outside the arrays: the sequence is refused, nothing is read
-        if (qt == 0 && threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
-        return;
-    }
-    if (qt * 2 * R >= qlen || timed_out(p.status)) return;
-    // key side (kk*): the rows the tiles are cut from; k*: the S_aug sequence
-    const int kklen = p.key_len[b];
-    if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
-        // the host-side bounds were wrong for this sequence: refuse it
-        if (threadIdx.x == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
-        return;
-    }
-    const int kstart = p.k_start[b], kkstart = p.key_start[b];
-    const int kvh = h0 / p.G;
-    const int pbase = klen - qlen + qt * 2 * R;  // position of query row 0 of tile 0
-    const bool tile1 = qt * 2 * R + R < qlen;     // tile 1 has rows
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-    // ------------------------------------------------ barriers, and Q on its way
-    // (its copy needs nothing from the tile list below, so it flies meanwhile)
     if (tid == 0) {
         mbar_init(q_full, 1);
+        mbar_init(q_empty, 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(&kv_full[s], 1);
-            mbar_init(&meta_full[s], 32);
             mbar_init(&kv_empty[s], 1);
+            mbar_init(&meta_full[2 * s], 1);
+            mbar_init(&meta_full[2 * s + 1], 1);
             mbar_init(&s_full[s], 1);
             mbar_init(&p_full[s], kBM);
             mbar_init(&o_done[s], 1);
+            mbar_init(&o_free[s], kBM);
+            mbar_init(&unit_full[s], 1);
+            mbar_init(&unit_empty[s], kUnitConsumers);
         }
         mbar_init(mma_idle, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&tmQ);
-        mbar_arrive_expect_tx(q_full, (tile1 ? 2 : 1) * C::kQBytes);
-        for (int qi = 0; qi < (tile1 ? 2 : 1); ++qi)
-#pragma unroll
-            for (int hh = 0; hh < C::kHalves; ++hh)
-                tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full, hh * 64, h0,
-                            p.q_start[b] + qt * 2 * R + qi * R, layer);
     }
-
-    // ------------------------------------------------ summaries of the query tiles
-    if (tid < 10) misc[4 + tid] = (tid % 5 == 0) ? 0 : ((tid % 5) & 1 ? INT_MAX : INT_MIN);
-    __syncthreads();
-    if (tid == kPfThreads - 32) {  // a thread the summaries below leave idle
-        // Key tile 0 comes first in the tile list whenever one of its non-body
-        // keys is at or before the last row of query tile 0 (that alone lists
-        // it): its K/V copy then starts now, ahead of the list.
-        int early = 0;
-        if (kklen > 0) {
-            const TileSum ts0 = p.sums[(int64_t)b * p.max_k_tiles];
-            early = (ts0.flags & 6) != 0 && ts0.pos_min <= min(pbase + R - 1, klen - 1);
-        }
-        if (early) {
-            mbar_arrive_expect_tx(&kv_full[0], 2 * C::kKVBytes);
-#pragma unroll
-            for (int hh = 0; hh < C::kHalves; ++hh) {
-                tma_load_4d(Ks + hh * (kBN * 128), &tmK, &kv_full[0], hh * 64, kvh, kkstart, layer);
-                tma_load_4d(Vs + hh * (kBN * 128), &tmV, &kv_full[0], hh * 64, kvh, kkstart, layer);
-            }
-        }
-        misc[3] = early;
-    }
-    if (tid < 2 * R && pbase + tid <= klen - 1) {
-        int32_t *qs = misc + 4 + 5 * (tid >= R ? 1 : 0);  // flags, seg min/max, nexus min/max
-        const int ro = p.role[kstart + pbase + tid];
-        const int s = p.seg[kstart + pbase + tid];
-        atomicMin(&qs[1], s);
-        atomicMax(&qs[2], s);
-        if (ro == SONIC_ROLE_NEXUS) {
-            atomicOr(&qs[0], 2);
-            atomicMin(&qs[3], s);
-            atomicMax(&qs[4], s);
-        }
-    }
-    __syncthreads();
-
-    // ------------------------------------------------ key tiles to visit
-    // list entry: (tile << 4) | (Nexus keys: 0 none, 1 all, 2 some) << 2
-    //             | (tile 0 needs the mask) | (tile 1 needs it) << 1
-    const int n_kt = (kklen + kBN - 1) / kBN;
-    int n_list = 0;
-    for (int c0 = 0; c0 < n_kt; c0 += kPfThreads) {
-        const int t = c0 + tid;
-        int entry = 0;
-        bool keep = false;
-        if (t < n_kt) {
-            const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
-            const int k0 = ts.pos_min, k1 = ts.pos_max;  // S_aug positions of the keys
-            const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
-            entry = (kn ? ((kb || ko) ? 2 : 1) : 0) << 2;
-            for (int qi = 0; qi < 2; ++qi) {
-                const int p0 = pbase + qi * R;
-                const int p1 = min(p0 + R - 1, klen - 1);
-                if (p0 > p1) continue;
-                const int *qs = misc + 4 + 5 * qi;
-                const bool q_has_nexus = qs[0] & 2;
-                const bool causal_part = (k0 <= p1) && (kn || ko);
-                const bool body_part =
-                    kb && (k0 <= p1) && !(ts.bseg_max < qs[1] || ts.bseg_min > qs[2]);
-                const bool nexus_part =
-                    kn && q_has_nexus &&
-                    (p.nexus_mode == SONIC_NEXUS_FULL || ts.nseg_min <= qs[4]);
-                const bool any = causal_part || body_part || nexus_part;
-                const bool full =
-                    any && ts.n_rows == kBN && k1 <= p0 &&
-                    (!kb || (ts.bseg_min == ts.bseg_max && qs[1] == qs[2] &&
-                             ts.bseg_min == qs[1])) &&
-                    (p.nexus_mode == SONIC_NEXUS_FULL || !(kn && q_has_nexus) ||
-                     ts.nseg_max <= qs[3]);
-                keep |= any;
-                if (!full) entry |= 1 << qi;
-            }
-        }
-        const unsigned bal = __ballot_sync(0xffffffffu, keep);
-        if (lane == 0) misc[16 + warp] = __popc(bal);
-        __syncthreads();
-        int base = n_list;
-        for (int w = 0; w < warp; ++w) base += misc[16 + w];
-        int tot = 0;
-        for (int w = 0; w < kPfThreads / 32; ++w) tot += misc[16 + w];
-        if (keep) list[base + __popc(bal & ((1u << lane) - 1u))] = (t << 4) | entry;
-        n_list += tot;
-        __syncthreads();
-    }
-
-    // ------------------------------------------------ tensor memory
     if (warp == 1) {
         tmem_alloc(reinterpret_cast<uint32_t *>(&misc[0]), 512);
         tmem_relinquish();
@@ -553,79 +552,299 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
-    if (warp == 0) {
+    // what the producer issued, for the drain after an abort
+    int issued_q = 0, issued_kv = 0;
+
+    if (warp == kSchedWarp) {
+        // ------------------------------------------------------------ scheduler
+        for (int k = 0;; ++k) {
+            const int slot = k & 1;
+            int end = 0, layer = 0, b = 0, hg = 0, qt = 0;
+            int kstart = 0, klen = 0, qstart = 0, qlen = 0, kkstart = 0, kklen = 0;
+            for (;;) {
+                int u = p.n_units;
+                if (lane == 0 && !*abort_flag && !timed_out(p.status)) u = atomicAdd(p.counter, 1);
+                u = __shfl_sync(0xffffffffu, u, 0);
+                if (u >= p.n_units) {
+                    end = 1;
+                    break;
+                }
+                // units: query-head group fastest, then query block (the last
+                // first: the longest lists go first), then sequence, then layer;
+                // the blocks running together read one sequence's K/V, which
+                // stays in L2
+                hg = u % p.HG;
+                int rest = u / p.HG;
+                qt = p.qtiles - 1 - rest % p.qtiles;
+                rest /= p.qtiles;
+                b = rest % p.B;
+                layer = rest / p.B;
+                klen = p.k_len[b];
+                qlen = p.q_len[b];
+                kstart = p.k_start[b];
+                qstart = p.q_start[b];
+                if (kstart < 0 || (int64_t)kstart + klen > p.total_k_rows || qstart < 0 ||
+                    qlen < 0 || (int64_t)qstart + qlen > p.total_q_rows) {
+                    // rows outside the arrays: the sequence is refused, nothing is read
+                    if (lane == 0 && hg == 0 && qt == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+                    continue;
+                }
+                if (qt * 2 * R >= qlen) continue;  // no query rows in this block
+                kklen = p.key_len[b];
+                if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
+                    // the host-side bounds were wrong for this sequence: refuse it
+                    if (lane == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
+                    continue;
+                }
+                kkstart = p.key_start[b];
+                break;
+            }
+            // The slot is free once every consumer is done with unit k - 2.  A
+            // unit takes microseconds: poll sparingly (a sleeping warp leaves
+            // its scheduler's issue slots to the softmax warps), then wait.
+            if (k >= 2) {
+                const uint32_t par = ((k >> 1) - 1) & 1;
+                const uint64_t t0 = global_ns();
+                while (!mbar_test(&unit_empty[slot], par) && !*abort_flag &&
+                       global_ns() - t0 < SONIC_WAIT_LIMIT_NS)
+                    __nanosleep(500);
+                if (!mbar_wait(&unit_empty[slot], par, p.status, abort_flag)) break;
+            }
+            UnitInfo *ui = units + slot;
+            if (end) {
+                if (lane == 0) {
+                    ui->flags = 1;
+                    mbar_arrive(&unit_full[slot]);
+                }
+                break;
+            }
+            const int pbase = klen - qlen + qt * 2 * R;  // position of query row 0 of tile 0
+            const bool tile1 = qt * 2 * R + R < qlen;
+            // summaries of the query tiles: segment range, Nexus rows and their
+            // segment range
+            int qf[2], qs0[2], qs1[2], qn0[2], qn1[2];
+#pragma unroll
+            for (int qi = 0; qi < 2; ++qi) {
+                int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
+                for (int r = lane; r < R; r += 32) {
+                    const int pos = pbase + qi * R + r;
+                    if (pos <= klen - 1) {
+                        const int ro = p.role[kstart + pos];
+                        const int s = p.seg[kstart + pos];
+                        s0 = min(s0, s);
+                        s1 = max(s1, s);
+                        if (ro == SONIC_ROLE_NEXUS) {
+                            f = 2;
+                            n0 = min(n0, s);
+                            n1 = max(n1, s);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    f |= __shfl_xor_sync(0xffffffffu, f, o);
+                    s0 = min(s0, __shfl_xor_sync(0xffffffffu, s0, o));
+                    s1 = max(s1, __shfl_xor_sync(0xffffffffu, s1, o));
+                    n0 = min(n0, __shfl_xor_sync(0xffffffffu, n0, o));
+                    n1 = max(n1, __shfl_xor_sync(0xffffffffu, n1, o));
+                }
+                qf[qi] = f;
+                qs0[qi] = s0;
+                qs1[qi] = s1;
+                qn0[qi] = n0;
+                qn1[qi] = n1;
+            }
+            // Key tiles to visit: a key tile is listed when either query tile
+            // sees some of it.  entry: (tile << 6) | (Nexus keys: 0 none, 1 all,
+            // 2 some) << 4 | (tile 1 sees it) << 3 | (tile 0 sees it) << 2
+            // | (not all of it visible to tile 1) << 1 | (... to tile 0)
+            int32_t *lst = lists + slot * kMaxKTiles;
+            const int n_kt = (kklen + kBN - 1) / kBN;
+            int n_list = 0, last0 = -1, last1 = -1, skipped = 0;
+            for (int c0 = 0; c0 < n_kt; c0 += 32) {
+                const int t = c0 + lane;
+                int entry = 0;
+                bool need[2] = {false, false};
+                if (t < n_kt) {
+                    const TileSum ts = p.sums[(int64_t)b * p.max_k_tiles + t];
+                    const int k0 = ts.pos_min, k1 = ts.pos_max;  // S_aug positions of the keys
+                    const bool kb = ts.flags & 1, kn = ts.flags & 2, ko = ts.flags & 4;
+                    entry = (t << 6) | ((kn ? ((kb || ko) ? 2 : 1) : 0) << 4);
+#pragma unroll
+                    for (int qi = 0; qi < 2; ++qi) {
+                        const int p0 = pbase + qi * R;
+                        const int p1 = min(p0 + R - 1, klen - 1);
+                        if (p0 > p1) continue;
+                        const bool q_has_nexus = qf[qi] & 2;
+                        const bool causal_part = (k0 <= p1) && (kn || ko);
+                        const bool body_part =
+                            kb && (k0 <= p1) && !(ts.bseg_max < qs0[qi] || ts.bseg_min > qs1[qi]);
+                        const bool nexus_part =
+                            kn && q_has_nexus &&
+                            (p.nexus_mode == SONIC_NEXUS_FULL || ts.nseg_min <= qn1[qi]);
+                        const bool any = causal_part || body_part || nexus_part;
+                        const bool full =
+                            any && ts.n_rows == kBN && k1 <= p0 &&
+                            (!kb || (ts.bseg_min == ts.bseg_max && qs0[qi] == qs1[qi] &&
+                                     ts.bseg_min == qs0[qi])) &&
+                            (p.nexus_mode == SONIC_NEXUS_FULL || !(kn && q_has_nexus) ||
+                             ts.nseg_max <= qn0[qi]);
+                        need[qi] = any;
+                        if (any) entry |= 4 << qi;
+                        if (!full) entry |= 1 << qi;
+                    }
+                }
+                const bool keep = need[0] || need[1];
+                const unsigned bal = __ballot_sync(0xffffffffu, keep);
+                skipped += __popc(__ballot_sync(0xffffffffu, keep && !need[0])) +
+                           (tile1 ? __popc(__ballot_sync(0xffffffffu, keep && !need[1])) : 0);
+                const unsigned b0 = __ballot_sync(0xffffffffu, need[0]);
+                const unsigned b1 = __ballot_sync(0xffffffffu, need[1]);
+                if (keep) lst[n_list + __popc(bal & ((1u << lane) - 1u))] = entry;
+                // list index of the last entry each query tile visits
+                if (b0) last0 = n_list + __popc(bal & ((2u << (31 - __clz(b0))) - 1u)) - 1;
+                if (b1) last1 = n_list + __popc(bal & ((2u << (31 - __clz(b1))) - 1u)) - 1;
+                n_list += __popc(bal);
+            }
+            // both query tiles visit every listed key tile (masked where they see
+            // none of it) unless skipping drops more than a tenth of the products
+            const bool dense = skipped * 10 <= (tile1 ? 2 : 1) * n_list;
+            if (lane == 0) {
+                ui->flags = dense ? 2 : 0;
+                ui->layer = layer;
+                ui->b = b;
+                ui->h0 = hg << pl2;
+                ui->qt = qt;
+                ui->nq = tile1 ? 2 : 1;
+                ui->n_list = n_list;
+                ui->kstart = kstart;
+                ui->klen = klen;
+                ui->kkstart = kkstart;
+                ui->kklen = kklen;
+                ui->qstart = qstart;
+                ui->qlen = qlen;
+                ui->pbase = pbase;
+                ui->last[0] = last0;
+                ui->last[1] = last1;
+            }
+            // every lane's list entries are written before lane 0 publishes the slot
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&unit_full[slot]);
+        }
+    } else if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
+            tma_prefetch_desc(&tmQ);
             tma_prefetch_desc(&tmK);
             tma_prefetch_desc(&tmV);
         }
-        int i = 0;
-        for (; i < n_list; ++i) {
-            const int st = i & 1;
-            if (i >= 2 && !mbar_wait(&kv_empty[st], ((i >> 1) - 1) & 1, p.status, abort_flag))
-                break;
-            const int kt = list[i] >> 4;
-            // K/V copies first; the key metadata is built while they are in flight
-            // and has a barrier of its own, so the S MMA of a cut tile waits for
-            // the copy alone, not for the metadata
-            if (lane == 0 && !(i == 0 && misc[3])) {
-                mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
-                const int row = kkstart + kt * kBN;
+        int g = 0;  // K/V tiles issued over all units (ring position)
+        bool ok = true;
+        for (int k = 0; ok; ++k) {
+            const int slot = k & 1;
+            if (!mbar_wait(&unit_full[slot], (k >> 1) & 1, p.status, abort_flag)) break;
+            const UnitInfo *ui = units + slot;
+            if (ui->flags & 1) break;
+            const int n_list = ui->n_list, nq = ui->nq, layer = ui->layer, b = ui->b;
+            const int kkstart = ui->kkstart, kklen = ui->kklen;
+            const bool udense = ui->flags & 2;  // both query tiles visit every listed tile
+            const int32_t *lst = lists + slot * kMaxKTiles;
+            if (n_list > 0) {
+                // Q: its buffer is free once the previous unit's last S products are done
+                if (issued_q > 0 &&
+                    !mbar_wait(q_empty, (issued_q - 1) & 1, p.status, abort_flag))
+                    break;
+                if (lane == 0) {
+                    mbar_arrive_expect_tx(q_full, nq * C::kQBytes);
+                    for (int qi = 0; qi < nq; ++qi)
 #pragma unroll
-                for (int hh = 0; hh < C::kHalves; ++hh) {
-                    tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), &tmK, &kv_full[st],
-                                hh * 64, kvh, row, layer);
-                    tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), &tmV, &kv_full[st],
-                                hh * 64, kvh, row, layer);
+                        for (int hh = 0; hh < C::kHalves; ++hh)
+                            tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
+                                        hh * 64, ui->h0, ui->qstart + ui->qt * 2 * R + qi * R,
+                                        layer);
+                }
+                ++issued_q;
+                const int kvh = ui->h0 / p.G;
+                for (int i = 0; i < n_list; ++i, ++g) {
+                    const int st = g & 1;
+                    if (g >= 2 && !mbar_wait(&kv_empty[st], ((g >> 1) - 1) & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    const int e = lst[i];
+                    const int kt = e >> 6;
+                    // query tiles visiting the key tile that read its metadata: cut
+                    // by the mask, or (Nexus mass) some of its keys are Nexus keys
+                    const bool mass_tile = kMass && ((e >> 4) & 3) == 2;
+                    const bool need_m0 = (udense || (e & 4)) && ((e & 1) || mass_tile);
+                    const bool need_m1 = nq == 2 && (udense || (e & 8)) && ((e & 2) || mass_tile);
+                    // K/V copies first; the key metadata is built while they are in
+                    // flight and has a barrier of its own, so the S product of a cut
+                    // tile waits for the copy alone
+                    if (lane == 0) {
+                        mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
+                        const int row = kkstart + kt * kBN;
+#pragma unroll
+                        for (int hh = 0; hh < C::kHalves; ++hh) {
+                            tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), &tmK, &kv_full[st],
+                                        hh * 64, kvh, row, layer);
+                            tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), &tmV, &kv_full[st],
+                                        hh * 64, kvh, row, layer);
+                        }
+                    }
+                    issued_kv = g + 1;
+                    // The tile's column masks (built once per key tile by the summary
+                    // kernel; 8 bytes per lane) where a query tile is cut or the Nexus
+                    // mass needs the Nexus bits; the keys' roles / segments / S_aug
+                    // positions only where the masks fall back to the per-key rule.
+                    const bool cut_any = (e & 3) != 0;
+                    if (need_m0 || need_m1) {
+                        const uint2 mw = reinterpret_cast<const uint2 *>(
+                            p.masks + (int64_t)b * p.max_k_tiles + kt)[lane];
+                        reinterpret_cast<uint2 *>(tmasks + st)[lane] = mw;
+                        // word 10 of the record (lane 5's first word): fallback
+                        const int fallback = __shfl_sync(0xffffffffu, (int)mw.x, 5);
+                        if (cut_any && fallback) {
+                            int ro[4], sg[4], ps[4];
+                            // all twelve loads first, none waiting on another
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const int q = kt * kBN + w * 32 + lane;
+                                const bool in = q < kklen;
+                                ro[w] = in ? p.key_role[kkstart + q] : 255;
+                                sg[w] = in ? p.key_seg[kkstart + q] : 0;
+                                ps[w] = in ? (p.key_pos != nullptr ? p.key_pos[kkstart + q] : q)
+                                           : INT_MAX;
+                            }
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const int c = w * 32 + lane;
+                                const bool pad = ro[w] == 255;  // no segment, no position
+                                meta_role[st * kBN + c] = (uint8_t)ro[w];
+                                meta_seg[st * kBN + c] = pad ? 0 : sg[w];
+                                meta_pos[st * kBN + c] = pad ? INT_MAX : ps[w];
+                            }
+                        }
+                        // every lane's metadata is written before lane 0 releases it
+                        __syncwarp();
+                        if (lane == 0) {
+                            if (need_m0) mbar_arrive(&meta_full[2 * st]);
+                            if (need_m1) mbar_arrive(&meta_full[2 * st + 1]);
+                        }
+                    }
                 }
             }
-            // The tile's column masks (built once per key tile by the summary
-            // kernel; 8 bytes per lane) where a query tile is cut or the Nexus
-            // mass needs the Nexus bits; the keys' roles / segments / S_aug
-            // positions only where the masks fall back to the per-key rule.
-            const bool cut_any = (list[i] & 3) != 0;
-            if (cut_any || (kMass && ((list[i] >> 2) & 3) == 2)) {
-                const uint2 mw =
-                    reinterpret_cast<const uint2 *>(p.masks + (int64_t)b * p.max_k_tiles + kt)[lane];
-                reinterpret_cast<uint2 *>(tmasks + st)[lane] = mw;
-                // word 10 of the record (lane 5's first word): fallback
-                const int fallback = __shfl_sync(0xffffffffu, (int)mw.x, 5);
-                if (cut_any && fallback) {
-                    int ro[4], sg[4], ps[4];
-                    // all twelve loads first, none waiting on another
-#pragma unroll
-                    for (int w = 0; w < 4; ++w) {
-                        const int q = kt * kBN + w * 32 + lane;
-                        const bool in = q < kklen;
-                        ro[w] = in ? p.key_role[kkstart + q] : 255;
-                        sg[w] = in ? p.key_seg[kkstart + q] : 0;
-                        ps[w] = in ? (p.key_pos != nullptr ? p.key_pos[kkstart + q] : q) : INT_MAX;
-                    }
-#pragma unroll
-                    for (int w = 0; w < 4; ++w) {
-                        const int c = w * 32 + lane;
-                        const bool pad = ro[w] == 255;  // no segment, no position
-                        meta_role[st * kBN + c] = (uint8_t)ro[w];
-                        meta_seg[st * kBN + c] = pad ? 0 : sg[w];
-                        meta_pos[st * kBN + c] = pad ? INT_MAX : ps[w];
-                    }
-                }
-                __syncwarp();
-            }
-            mbar_arrive(&meta_full[st]);  // 32 arrivals end the phase
-        }
-        if (lane == 0 && *abort_flag) {
-            // let issued copies land before the block exits
-            mbar_wait(q_full, 0, p.status, abort_flag);
-            for (int u = max(0, i - 2); u < i; ++u)
-                mbar_wait(&kv_full[u & 1], (u >> 1) & 1, p.status, abort_flag);
+            if (!ok) break;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&unit_empty[slot]);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         // This thread is on the path of every key tile, so its loop is
-        // specialised on the number of query tiles and unrolled over the two
-        // K/V stages, and each descriptor is a precomputed word plus a constant:
-        // an MMA then costs about two instructions besides itself.
+        // specialised on the number of query tiles and on whether both visit
+        // every listed key tile (no per-tile checks then), and each descriptor
+        // is a per-stage word plus a constant: an MMA then costs about two
+        // instructions besides itself.
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, 0);
             constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, 1);
@@ -633,342 +852,405 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const uint32_t q_lo = sw128_desc_lo(smem_u32(Qs), 16);
             const uint32_t k_lo = sw128_desc_lo(smem_u32(Ks), 16);
             const uint32_t v_lo = sw128_desc_lo(smem_u32(Vs), kBN * 128);
-            const int nq = tile1 ? 2 : 1;
-            // S_qi = Q_qi K^T from K stage st
-            auto issue_s = [&](int qi, int st) {
+            // S_qi = Q_qi K^T from the K stage whose descriptor word is kst
+            auto issue_s = [&](int qi, uint32_t kst) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = ((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4;
                     tc_mma_ss(tmem + qi * kBN,
                               desc_join(q_lo + ((qi * C::kQBytes) >> 4) + off, dhi),
-                              desc_join(k_lo + ((st * C::kKVBytes) >> 4) + off, dhi), idS,
-                              kk > 0 ? 1u : 0u);
+                              desc_join(kst + off, dhi), idS, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[qi]);
             };
-            // O_qi += P_qi V from V stage st (P over the first columns of S_qi)
-            auto issue_pv = [&](int qi, int st, bool acc0) {
+            // O_qi (+)= P_qi V from the V stage whose descriptor word is vst (P over
+            // the first columns of S_qi)
+            auto issue_pv = [&](int qi, uint32_t vst, bool acc0) {
 #pragma unroll
                 for (int kk = 0; kk < kBN / 16; ++kk)
                     tc_mma_ts(tmem + 256 + qi * 128, tmem + qi * kBN + kk * 8,
-                              desc_join(v_lo + ((st * C::kKVBytes + kk * (16 * 128)) >> 4), dhi),
-                              idPV, (acc0 || kk > 0) ? 1u : 0u);
+                              desc_join(vst + ((kk * (16 * 128)) >> 4), dhi), idPV,
+                              (acc0 || kk > 0) ? 1u : 0u);
             };
-            bool ok = mbar_wait(q_full, 0, p.status, abort_flag) && n_list > 0 &&
-                      mbar_wait(&kv_full[0], 0, p.status, abort_flag);
-            if (ok) {
-                tc_fence_after();
-                for (int qi = 0; qi < nq; ++qi) issue_s(qi, 0);
-            }
-            // Key tile j (in stage j & 1): P.V of each query tile, then its S of
-            // tile j + 1.  The tensor pipe runs in order, so the next S never
-            // overwrites a P still being read.
-            auto main_loop = [&](auto nq_tag) {
-                constexpr int NQ = decltype(nq_tag)::value;
-                auto tile = [&](int j, auto st_tag) -> bool {
-                    constexpr int ST = decltype(st_tag)::value;
-                    const bool more = j + 1 < n_list;
-#pragma unroll
-                    for (int qi = 0; qi < NQ; ++qi) {
-                        if (!mbar_wait(&p_full[qi], ST, p.status, abort_flag)) return false;
+            // descriptor words of K and V in ring stage st
+            constexpr uint32_t kStageStep = C::kKVBytes >> 4;
+            auto k_of = [&](int st) { return k_lo + (st ? kStageStep : 0u); };
+            auto v_of = [&](int st) { return v_lo + (st ? kStageStep : 0u); };
+            int g = 0, nqu = 0;          // ring position; units with work so far
+            uint32_t pw[2] = {0u, 0u};   // P phases waited per query tile
+            int uo[2] = {0, 0};          // units whose O each query tile accumulated
+            bool ok = true;
+            for (int k = 0; ok; ++k) {
+                const int slot = k & 1;
+                if (!mbar_wait(&unit_full[slot], (k >> 1) & 1, p.status, abort_flag)) break;
+                const UnitInfo *ui = units + slot;
+                if (ui->flags & 1) break;
+                const int n_list = ui->n_list, nq = ui->nq;
+                const int last[2] = {ui->last[0], ui->last[1]};
+                const int32_t *lst = lists + slot * kMaxKTiles;
+                if (n_list > 0) {
+                    ok = mbar_wait(q_full, nqu & 1, p.status, abort_flag);
+                    ++nqu;
+                    // Key tile j (ring stage (g + j) & 1): P.V of each query tile
+                    // visiting it, then that tile's S of the next key tile it
+                    // visits.  The tensor pipe runs in order, so the next S never
+                    // overwrites a P still being read.
+                    // DENSE: every query tile visits every listed key tile (no list
+                    // reads or per-tile checks on this thread's path)
+                    auto run = [&](auto nq_tag, auto dense_tag) -> bool {
+                        constexpr int NQ = decltype(nq_tag)::value;
+                        constexpr bool DENSE = decltype(dense_tag)::value;
+                        auto visits = [&](int ent, int qi) -> bool {
+                            return DENSE || ((ent >> (2 + qi)) & 1);
+                        };
+                        bool first[2] = {true, true};
+                        int e = DENSE ? 0 : lst[0];
+                        int en = (DENSE || n_list < 2) ? 0 : lst[1];
+                        if (!mbar_wait(&kv_full[g & 1], (g >> 1) & 1, p.status, abort_flag))
+                            return false;
                         tc_fence_after();
-                        issue_pv(qi, ST, j > 0);
-                        if (!more) tc_commit(&o_done[qi]);
-                        if (qi == NQ - 1) tc_commit(&kv_empty[ST]);
-                        if (more) {
-                            if (qi == 0 && !mbar_wait(&kv_full[1 - ST], ((j + 1) >> 1) & 1,
-                                                      p.status, abort_flag))
-                                return false;
-                            tc_fence_after();
-                            issue_s(qi, 1 - ST);
+#pragma unroll
+                        for (int qi = 0; qi < NQ; ++qi)
+                            if (visits(e, qi)) issue_s(qi, k_of(g & 1));
+                        if (n_list == 1) tc_commit(q_empty);
+                        // key tile j sits in ring stage (g + j) & 1; one copy of the
+                        // body, the stage entering only through descriptor words
+                        for (int j = 0; j < n_list; ++j) {
+                            const int ST = (g + j) & 1;
+                            const uint32_t vst = v_of(ST), kst_next = k_of(ST ^ 1);
+                            const bool more = j + 1 < n_list;
+                            // the entry after next, loaded a tile ahead of its use
+                            const int enn = (DENSE || j + 2 >= n_list) ? 0 : lst[j + 2];
+                            const int lastq = DENSE ? NQ - 1 : ((NQ == 2 && ((e >> 3) & 1)) ? 1 : 0);
+                            bool kv_ready = false;
+#pragma unroll
+                            for (int qi = 0; qi < NQ; ++qi) {
+                                if (visits(e, qi)) {
+                                    if (!mbar_wait(&p_full[qi], pw[qi] & 1, p.status, abort_flag))
+                                        return false;
+                                    ++pw[qi];
+                                    tc_fence_after();
+                                    const bool fst = DENSE ? j == 0 : first[qi];
+                                    if (fst && uo[qi] > 0) {
+                                        // O still holds the previous unit until its
+                                        // epilogue has read it
+                                        if (!mbar_wait(&o_free[qi], (uo[qi] - 1) & 1, p.status,
+                                                       abort_flag))
+                                            return false;
+                                        tc_fence_after();
+                                    }
+                                    issue_pv(qi, vst, !fst);
+                                    if (!DENSE) first[qi] = false;
+                                    if (j == (DENSE ? n_list - 1 : last[qi])) tc_commit(&o_done[qi]);
+                                    if (qi == lastq) tc_commit(&kv_empty[ST]);
+                                }
+                                if (more && visits(en, qi)) {
+                                    if (!kv_ready) {
+                                        const int gn = g + j + 1;
+                                        if (!mbar_wait(&kv_full[ST ^ 1], (gn >> 1) & 1, p.status,
+                                                       abort_flag))
+                                            return false;
+                                        tc_fence_after();
+                                        kv_ready = true;
+                                    }
+                                    issue_s(qi, kst_next);
+                                }
+                            }
+                            // every S product of the unit is issued: Q may be replaced
+                            if (j + 2 == n_list) tc_commit(q_empty);
+                            if (!DENSE) {
+                                e = en;
+                                en = enn;
+                            }
                         }
+                        return true;
+                    };
+                    const bool dense = ui->flags & 2;
+                    if (ok) {
+                        if (nq == 2)
+                            ok = dense ? run(std::integral_constant<int, 2>{}, std::true_type{})
+                                       : run(std::integral_constant<int, 2>{}, std::false_type{});
+                        else
+                            ok = dense ? run(std::integral_constant<int, 1>{}, std::true_type{})
+                                       : run(std::integral_constant<int, 1>{}, std::false_type{});
                     }
-                    return true;
-                };
-                for (int j = 0; ok && j < n_list; j += 2) {
-                    ok = tile(j, std::integral_constant<int, 0>{});
-                    if (ok && j + 1 < n_list) ok = tile(j + 1, std::integral_constant<int, 1>{});
+                    for (int qi = 0; qi < 2; ++qi)
+                        if ((dense && n_list > 0) ? qi < nq : last[qi] >= 0) ++uo[qi];
+                    g += n_list;
                 }
-            };
-            if (ok) {
-                if (nq == 2)
-                    main_loop(std::integral_constant<int, 2>{});
-                else
-                    main_loop(std::integral_constant<int, 1>{});
+                if (ok) mbar_arrive(&unit_empty[slot]);
             }
             // every MMA issued by this thread has finished once this arrives
             tc_commit(mma_idle);
-            mbar_wait(mma_idle, 0, p.status, abort_flag);
+            mbar_drain(mma_idle, 0);
         }
-    } else if (warp < 6 || tile1) {
+    } else {
         // ------------------------------------------------------------ softmax
         const int qi = (warp - 2) >> 2;
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
-        const int qr = r >> pl2, h = h0 + (r & ((1 << pl2) - 1));  // query row and head of tile row r
-        const int pos = pbase + qi * R + qr;
-        const bool row_ok = pos <= klen - 1 && qt * 2 * R + qi * R + qr < qlen;
-        int rp = SONIC_ROLE_SYS, sp = 0;
-        if (row_ok) {
-            rp = p.role[kstart + pos];
-            sp = p.seg[kstart + pos];
-        }
+        const int qr = r >> pl2, hoff = r & ((1 << pl2) - 1);  // query row and head of tile row r
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
         const uint32_t tS = tmem + lane_base + qi * kBN;
         const uint32_t tO = tmem + lane_base + 256 + qi * 128;
-        // l: sum of the rounded probabilities (normalises O); l_lse: of the
-        // unrounded ones, for the log-sum-exp output (kLse: lse requested)
-        float m_used = -INFINITY, l = 0.f, l_lse = 0.f;
-        // ln: the part of l on Nexus keys (kMass)
-        float ln = 0.f;
+        // Parities of the phases this warpgroup waits next, one bit each (all it
+        // needs of its counters; one register across the key-tile loop):
+        //   bit 0 / 1  metadata barrier of ring stage 0 / 1,
+        //   bit 2      S barrier,
+        //   bit 3      O barrier (o_done),
+        //   bit 4      ring stage of the unit's first key tile.
+        uint32_t ph = 0;
         bool ok = true;
-        // the next list entry is read one tile ahead: shared memory is busy
-        // feeding the tensor cores, so a load on the critical path is slow
-        int entry = n_list > 0 ? list[0] : 0;
-        for (int j = 0; j < n_list; ++j) {
-            const int st = j & 1;
-            const int kt = entry >> 4;
-            const bool cut = (entry >> qi) & 1;
-            const int nexus_keys = (entry >> 2) & 3;
-            entry = j + 1 < n_list ? list[j + 1] : 0;
-            // the keys' roles/segments are read (and V rows zeroed) on cut tiles
-            // only, and their Nexus bits on tiles with some Nexus keys
-            const bool need_meta = cut || (kMass && nexus_keys == 2);
-            if (need_meta && !mbar_wait(&meta_full[st], (j >> 1) & 1, p.status, abort_flag)) {
-                ok = false;
-                break;
-            }
-            // The mask bits of a cut tile, worked out before S is read: the MMA
-            // producing S runs meanwhile, and the mask record and the S row are
-            // never held in registers together.
-            uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-            if (cut) {
-                // the whole mask record in independent 16-byte loads
-                const uint4 *tv = reinterpret_cast<const uint4 *>(tmasks + st);
-                const uint4 nb = tv[0], nx = tv[1], hd = tv[2], bsg = tv[3], nsg = tv[4];
-                uint4 bm[4], nm[4];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    bm[k] = tv[5 + k];
-                    nm[k] = tv[9 + k];
+        for (int k = 0; ok; ++k) {
+            const int slot = k & 1;
+            if (!mbar_wait(&unit_full[slot], (k >> 1) & 1, p.status, abort_flag)) break;
+            const UnitInfo *ui = units + slot;
+            if (ui->flags & 1) break;
+            const int n_list = ui->n_list;
+            const uint32_t st0 = (ph >> 4) & 1;  // stage of key tile 0 of this unit
+            ph ^= (uint32_t)(n_list & 1) << 4;
+            if (qi < ui->nq) {
+                // (the unit's other fields are read again from its slot for the
+                // epilogue: fewer registers live across the key-tile loop)
+                const bool udense = ui->flags & 2;
+                const int last = udense ? n_list - 1 : ui->last[qi];
+                const int kklen = ui->kklen;
+                const int pos = ui->pbase + qi * R + qr;
+                int rp = SONIC_ROLE_SYS, sp = 0;
+                if (pos <= ui->klen - 1) {
+                    rp = p.role[ui->kstart + pos];
+                    sp = p.seg[ui->kstart + pos];
                 }
-                if (!hd.z) {
-                    // causal prefix (keys at or before this row: a prefix of the
-                    // tile's columns, counted over the position runs), body keys of
-                    // this row's segment, and the Nexus keys a Nexus row sees
-                    const uint4 rp4 = tv[13], rl4 = tv[14];
-                    const int nvis = min(max(pos - (int)rp4.x + 1, 0), (int)rl4.x) +
-                                     min(max(pos - (int)rp4.y + 1, 0), (int)rl4.y) +
-                                     min(max(pos - (int)rp4.z + 1, 0), (int)rl4.z) +
-                                     min(max(pos - (int)rp4.w + 1, 0), (int)rl4.w);
-                    const int nbody = (int)hd.x, nnex = (int)hd.y;
-                    const int bs4[4] = {(int)bsg.x, (int)bsg.y, (int)bsg.z, (int)bsg.w};
-                    const int ns4[4] = {(int)nsg.x, (int)nsg.y, (int)nsg.z, (int)nsg.w};
-                    uint4 bw = make_uint4(0u, 0u, 0u, 0u), xw = make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        if (k < nbody && bs4[k] == sp) {
-                            bw.x |= bm[k].x; bw.y |= bm[k].y; bw.z |= bm[k].z; bw.w |= bm[k].w;
-                        }
-                        if (rp == SONIC_ROLE_NEXUS && p.nexus_mode != SONIC_NEXUS_FULL &&
-                            k < nnex && ns4[k] <= sp) {
-                            xw.x |= nm[k].x; xw.y |= nm[k].y; xw.z |= nm[k].z; xw.w |= nm[k].w;
+                const int32_t *lst = lists + slot * kMaxKTiles;
+                // l: sum of the rounded probabilities (normalises O); l_lse: of the
+                // unrounded ones, for the log-sum-exp output (kLse: lse requested)
+                float m_used = -INFINITY, l = 0.f, l_lse = 0.f;
+                // ln: the part of l on Nexus keys (kMass)
+                float ln = 0.f;
+                // the next list entry is read one tile ahead: shared memory is busy
+                // feeding the tensor cores, so a load on the critical path is slow
+                int entry = n_list > 0 ? lst[0] : 0;
+                for (int j = 0; j <= last; ++j) {
+                    const int e = entry;
+                    entry = j + 1 < n_list ? lst[j + 1] : 0;
+                    if (!udense && !((e >> (2 + qi)) & 1)) continue;  // a tile it does not see
+                    const int st = (st0 + j) & 1;
+                    const int kt = e >> 6;
+                    const bool cut = (e >> qi) & 1;
+                    const int nexus_keys = (e >> 4) & 3;
+                    // The keys' masks are read on cut tiles only, their Nexus bits
+                    // on tiles with some Nexus keys: one phase of this tile's
+                    // metadata barrier each.
+                    const bool need_meta = cut || (kMass && nexus_keys == 2);
+                    if (need_meta) {
+                        const uint32_t mph = (ph >> st) & 1;
+                        ph ^= 1u << st;
+                        if (!mbar_wait(&meta_full[2 * st + qi], mph, p.status, abort_flag)) {
+                            ok = false;
+                            break;
                         }
                     }
-                    if (rp == SONIC_ROLE_NEXUS && p.nexus_mode == SONIC_NEXUS_FULL) xw = nx;
-                    const uint32_t nbw[4] = {nb.x, nb.y, nb.z, nb.w};
-                    const uint32_t bww[4] = {bw.x, bw.y, bw.z, bw.w};
-                    const uint32_t xww[4] = {xw.x, xw.y, xw.z, xw.w};
-#pragma unroll
-                    for (int w = 0; w < 4; ++w) {
-                        const int nw = min(max(nvis - 32 * w, 0), 32);
-                        const uint32_t cw = nw >= 32 ? 0xffffffffu : ((1u << nw) - 1u);
-                        mbits[w] = (cw & (nbw[w] | bww[w])) | xww[w];
+                    // The mask bits of a cut tile, worked out before S is read: the MMA
+                    // producing S runs meanwhile, and the mask record and the S row are
+                    // never held in registers together.
+                    uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
+                    if (cut) tile_mask_bits(tmasks + st, meta_role + st * kBN, meta_seg + st * kBN,
+                                            meta_pos + st * kBN, pos, rp, sp, p.nexus_mode, mbits);
+                    if (!mbar_wait(&s_full[qi], (ph >> 2) & 1, p.status, abort_flag)) {
+                        ok = false;
+                        break;
                     }
-                } else {
+                    ph ^= 4u;
+                    tc_fence_after();
+                    // S row into registers: four 32-column loads, one wait
+                    uint32_t sr[4][32];
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        const uint8_t *mr = meta_role + st * kBN + c * 32;
-                        const int32_t *ms = meta_seg + st * kBN + c * 32;
-                        const int32_t *mp = meta_pos + st * kBN + c * 32;
-                        uint32_t bits = 0;
-#pragma unroll 4
-                        for (int e = 0; e < 32; ++e) {
-                            const int rq = mr[e];
-                            const bool v = rq != 255 &&
-                                           visible(pos, mp[e], rp, sp, rq, ms[e], p.nexus_mode);
-                            bits |= (v ? 1u : 0u) << e;
-                        }
-                        mbits[c] = bits;
-                    }
-                }
-            }
-            if (!mbar_wait(&s_full[qi], j & 1, p.status, abort_flag)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            // S row into registers: four 32-column loads, one wait
-            uint32_t sr[4][32];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
-            tmem_ld_wait();
-#pragma unroll
-            for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
-            // row maximum (masked keys set to -inf on a cut tile)
-            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            if (!cut) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2)
-                        mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][e]),
-                                       __uint_as_float(sr[c][e + 1]));
-            } else {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        if (!((mbits[c] >> e) & 1)) sr[c][e] = __float_as_uint(-INFINITY);
-                        mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][e]));
-                    }
-            }
-            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
-            float alpha = 1.f, m_new = m_used;
-            if (j == 0) {
-                m_new = mx;
-            } else if (mx > m_used + kRescaleThreshold) {
-                m_new = mx;
-                alpha = ex2(m_used - m_new);
-            }
-            const float mref = (m_new == -INFINITY) ? 0.f : m_new;
-            // probabilities, written as bf16 pairs over the S columns
-            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
-            const float2 nm2 = make_float2(-mref, -mref);
-            float ls[4] = {0.f, 0.f, 0.f, 0.f};
-            float2 rs2x = make_float2(0.f, 0.f);
-            // the Nexus part of the row sum: all of it, none, or (some Nexus
-            // keys) the keys the tile's Nexus bits select.  The two forms of
-            // the loop are separate instances, so the common one stays one
-            // straight run of code the compiler can interleave across chunks.
-            float lsn[2] = {0.f, 0.f};
-            auto exps = [&](auto nx_tag) {
-                constexpr bool NX = decltype(nx_tag)::value;
-                uint32_t nxb[4] = {0u, 0u, 0u, 0u};
-                if (NX) {
-                    const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
-                    nxb[0] = nx.x;
-                    nxb[1] = nx.y;
-                    nxb[2] = nx.z;
-                    nxb[3] = nx.w;
-                }
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c][e]),
-                                                                __uint_as_float(sr[c][e + 1])),
-                                                    sc2, nm2);
-                        const float2 eu = make_float2(ex2(x.x), ex2(x.y));
-                        if (kLse) rs2x = __fadd2_rn(rs2x, eu);
-                        const uint32_t pr = pack_bf16x2(eu.x, eu.y);
-                        pk[e >> 1] = pr;
-                        // the row sum adds the rounded probabilities P.V
-                        // multiplies by, so O is a weighted mean of V rows with
-                        // weights summing to one (rounding moves weight between
-                        // keys, it does not scale the output)
-                        add_bf16x2_to_f32(ls[(e >> 1) & 2], ls[((e >> 1) & 2) + 1], pr);
-                        if (NX)
-                            add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << e),
-                                                 nxb[c] & (2u << e));
-                    }
-                    tmem_st16(tS + c * 16, pk);
-                }
-            };
-            if (kMass && nexus_keys == 2)
-                exps(std::true_type{});
-            else
-                exps(std::false_type{});
-            const float l_tile = (ls[0] + ls[1]) + (ls[2] + ls[3]);
-            l = l * alpha + l_tile;
-            if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
-            if (kMass)
-                ln = ln * alpha + (nexus_keys == 1 ? l_tile : (lsn[0] + lsn[1]));
-            // O rescale (PV of the previous tile is complete: S of this tile was
-            // issued after it, and S is done)
-            if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    tmem_ld32(tO + c * 32, o);
+                    for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
                     tmem_ld_wait();
-                    reg_fence32(o);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                    tmem_st32(tO + c * 32, o);
-                }
-            }
-            tmem_st_wait();
-            // Rows of V past the sequence end: zero them so 0 * garbage cannot
-            // reach the accumulator (tile 0's warps; its PV is issued first).
-            if (qi == 0 && kt * kBN + kBN > kklen && kt * kBN + r >= kklen) {
+                    for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
+                    // row maximum (masked keys set to -inf on a cut tile)
+                    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    if (!cut) {
 #pragma unroll
-                for (int hh = 0; hh < C::kHalves; ++hh) {
-                    uint4 *vr = reinterpret_cast<uint4 *>(Vs + st * C::kKVBytes +
-                                                          hh * (kBN * 128) + r * 128);
+                        for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) vr[u] = make_uint4(0, 0, 0, 0);
-                }
-                fence_proxy_async_smem();
-            }
-            tc_fence_before();
-            mbar_arrive(&p_full[qi]);
-            m_used = m_new;
-        }
-        // ------------------------------------------------------------ epilogue
-        if (ok && n_list > 0 && mbar_wait(&o_done[qi], 0, p.status, abort_flag)) {
-            tc_fence_after();
-            const float inv = l > 0.f ? 1.f / l : 0.f;
-            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * R + qi * R + qr;
-            uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
+                            for (int x = 0; x < 32; x += 2)
+                                mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][x]),
+                                               __uint_as_float(sr[c][x + 1]));
+                    } else {
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tO + c * 32, o);
-                tmem_ld_wait();
-                reg_fence32(o);
-                if (row_ok) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+                        for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e)
-                            w[e] = pack_bf16x2(__uint_as_float(o[u * 8 + 2 * e]) * inv,
-                                               __uint_as_float(o[u * 8 + 2 * e + 1]) * inv);
-                        dst[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                            for (int x = 0; x < 32; ++x) {
+                                if (!((mbits[c] >> x) & 1)) sr[c][x] = __float_as_uint(-INFINITY);
+                                mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][x]));
+                            }
                     }
+                    const float mx =
+                        fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
+                    // (m_used = -inf: no visible key so far, so l = 0 and O = 0 --
+                    // this tile starts the row whatever came before)
+                    float alpha = 1.f, m_new = m_used;
+                    if (m_used == -INFINITY) {
+                        m_new = mx;
+                    } else if (mx > m_used + kRescaleThreshold) {
+                        m_new = mx;
+                        alpha = ex2(m_used - m_new);
+                    }
+                    const float mref = (m_new == -INFINITY) ? 0.f : m_new;
+                    // probabilities, written as bf16 pairs over the S columns
+                    const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
+                    const float2 nm2 = make_float2(-mref, -mref);
+                    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+                    float2 rs2x = make_float2(0.f, 0.f);
+                    // the Nexus part of the row sum: all of it, none, or (some Nexus
+                    // keys) the keys the tile's Nexus bits select.  The two forms of
+                    // the loop are separate instances, so the common one stays one
+                    // straight run of code the compiler can interleave across chunks.
+                    float lsn[2] = {0.f, 0.f};
+                    auto exps = [&](auto nx_tag) {
+                        constexpr bool NX = decltype(nx_tag)::value;
+                        uint32_t nxb[4] = {0u, 0u, 0u, 0u};
+                        if (NX) {
+                            const uint4 nx = reinterpret_cast<const uint4 *>(tmasks + st)[1];
+                            nxb[0] = nx.x;
+                            nxb[1] = nx.y;
+                            nxb[2] = nx.z;
+                            nxb[3] = nx.w;
+                        }
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint32_t pk[16];
+#pragma unroll
+                            for (int x = 0; x < 32; x += 2) {
+                                const float2 v = __ffma2_rn(make_float2(__uint_as_float(sr[c][x]),
+                                                                        __uint_as_float(sr[c][x + 1])),
+                                                            sc2, nm2);
+                                const float2 eu = make_float2(ex2(v.x), ex2(v.y));
+                                if (kLse) rs2x = __fadd2_rn(rs2x, eu);
+                                const uint32_t pr = pack_bf16x2(eu.x, eu.y);
+                                pk[x >> 1] = pr;
+                                // the row sum adds the rounded probabilities P.V
+                                // multiplies by, so O is a weighted mean of V rows with
+                                // weights summing to one (rounding moves weight between
+                                // keys, it does not scale the output)
+                                add_bf16x2_to_f32(ls[(x >> 1) & 2], ls[((x >> 1) & 2) + 1], pr);
+                                if (NX)
+                                    add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << x),
+                                                         nxb[c] & (2u << x));
+                            }
+                            tmem_st16(tS + c * 16, pk);
+                        }
+                    };
+                    if (kMass && nexus_keys == 2)
+                        exps(std::true_type{});
+                    else
+                        exps(std::false_type{});
+                    const float l_tile = (ls[0] + ls[1]) + (ls[2] + ls[3]);
+                    l = l * alpha + l_tile;
+                    if (kLse) l_lse = l_lse * alpha + (rs2x.x + rs2x.y);
+                    if (kMass) ln = ln * alpha + (nexus_keys == 1 ? l_tile : (lsn[0] + lsn[1]));
+                    // O rescale (the previous P.V of this tile is complete: this S
+                    // was issued after it, and S is done)
+                    if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint32_t o[32];
+                            tmem_ld32(tO + c * 32, o);
+                            tmem_ld_wait();
+                            reg_fence32(o);
+#pragma unroll
+                            for (int x = 0; x < 32; ++x)
+                                o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
+                            tmem_st32(tO + c * 32, o);
+                        }
+                    }
+                    tmem_st_wait();
+                    // Rows of V past the sequence end: zero them so 0 * garbage
+                    // cannot reach the accumulator (the warps of the first query
+                    // tile visiting the key tile; its P.V is issued first).
+                    const int first_qi = (udense || (e & 4)) ? 0 : 1;
+                    if (qi == first_qi && kt * kBN + kBN > kklen && kt * kBN + r >= kklen) {
+#pragma unroll
+                        for (int hh = 0; hh < C::kHalves; ++hh) {
+                            uint4 *vr = reinterpret_cast<uint4 *>(Vs + st * C::kKVBytes +
+                                                                  hh * (kBN * 128) + r * 128);
+#pragma unroll
+                            for (int u = 0; u < 8; ++u) vr[u] = make_uint4(0, 0, 0, 0);
+                        }
+                        fence_proxy_async_smem();
+                    }
+                    tc_fence_before();
+                    mbar_arrive(&p_full[qi]);
+                    m_used = m_new;
+                }
+                if (!ok) break;
+                const int layer = ui->layer, h = ui->h0 + hoff;
+                const int qidx = ui->qt * 2 * R + qi * R + qr;  // query row within the sequence
+                const bool row_ok = pos <= ui->klen - 1 && qidx < ui->qlen;
+                const int64_t qrow = (int64_t)ui->qstart + qidx;
+                uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
+                const int64_t sidx = ((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h;
+                if (last >= 0) {
+                    // ------------------------------------------------ epilogue
+                    if (!mbar_wait(&o_done[qi], (ph >> 3) & 1, p.status, abort_flag)) break;
+                    ph ^= 8u;
+                    tc_fence_after();
+                    const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(tO + c * 32, o);
+                        tmem_ld_wait();
+                        reg_fence32(o);
+                        if (c == D / 32 - 1) {
+                            // O is read: the next unit's first P.V may overwrite it
+                            tc_fence_before();
+                            mbar_arrive(&o_free[qi]);
+                        }
+                        if (row_ok) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                uint32_t w[4];
+#pragma unroll
+                                for (int x = 0; x < 4; ++x)
+                                    w[x] = pack_bf16x2(__uint_as_float(o[u * 8 + 2 * x]) * inv,
+                                                       __uint_as_float(o[u * 8 + 2 * x + 1]) * inv);
+                                dst[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                        }
+                    }
+                    if (row_ok) {
+                        if (kLse)
+                            p.lse[sidx] = l_lse > 0.f ? (m_used + __log2f(l_lse)) * kLn2f : -INFINITY;
+                        if (kMass) p.nexus_mass[sidx] = ln * inv;
+                    }
+                } else if (row_ok) {
+                    // no key tile to visit (never for a valid layout): zeros
+                    uint4 *dst = reinterpret_cast<uint4 *>(orow);
+#pragma unroll
+                    for (int u = 0; u < D / 8; ++u) dst[u] = make_uint4(0, 0, 0, 0);
+                    if (kLse) p.lse[sidx] = -INFINITY;
+                    if (kMass) p.nexus_mass[sidx] = 0.f;
                 }
             }
-            if (kLse && row_ok)
-                p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] =
-                    l_lse > 0.f ? (m_used + __log2f(l_lse)) * kLn2f : -INFINITY;
-            if (kMass && row_ok)
-                p.nexus_mass[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = ln * inv;
-        } else if (row_ok && n_list == 0) {
-            const int64_t qrow = (int64_t)p.q_start[b] + qt * 2 * R + qi * R + qr;
-            uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
-            for (int d = 0; d < D; ++d) orow[d] = 0;
-            if (kLse)
-                p.lse[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = -INFINITY;
-            if (kMass) p.nexus_mass[((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h] = 0.f;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&unit_empty[slot]);
         }
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // After an abort no thread waits any more; let the copies the producer
+    // issued land before the block's shared memory goes away.
+    if (*abort_flag && warp == 0 && lane == 0) {
+        if (issued_q > 0) mbar_drain(q_full, (issued_q - 1) & 1);
+        for (int u = max(0, issued_kv - 2); u < issued_kv; ++u)
+            mbar_drain(&kv_full[u & 1], (u >> 1) & 1);
+    }
+    __syncthreads();
     if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
@@ -1159,7 +1441,7 @@ kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
 
 template <int D>
 cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
-                           const PfParams &p, dim3 grid, cudaStream_t s) {
+                           const PfParams &p, int grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
     const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
@@ -1179,17 +1461,20 @@ int max_k_tiles_of(const sonic_prefill_args *a) {
     return a->key_order == SONIC_KEYS_RETAINED_FIRST ? t + 1 : t;
 }
 
-// Workspace: tile summaries and tile column masks; with the retained-first
-// order also the permuted key metadata and the permuted K and V of every layer.
+// Workspace: the work-unit counter, tile summaries and tile column masks; with
+// the retained-first order also the permuted key metadata and the permuted K
+// and V of every layer.
 struct PfWorkspace {
-    size_t sums, masks, key_start, key_len, role, seg, pos, src, kp, vp, total;
+    size_t counter, sums, masks, key_start, key_len, role, seg, pos, src, kp, vp, total;
     int64_t rows;  // rows of the permuted K/V per layer
 };
 
 PfWorkspace workspace_layout(const sonic_prefill_args *a) {
     PfWorkspace w{};
     const size_t tiles = (size_t)a->batch * max_k_tiles_of(a);
-    w.masks = round_up(tiles * sizeof(TileSum), 256);
+    w.counter = 0;
+    w.sums = 256;
+    w.masks = w.sums + round_up(tiles * sizeof(TileSum), 256);
     size_t off = w.masks + round_up(tiles * sizeof(TileMasks), 256);
     if (a->key_order == SONIC_KEYS_RETAINED_FIRST) {
         const int64_t span = (int64_t)((a->max_k_len + kBN - 1) / kBN) * kBN + kBN;
@@ -1273,8 +1558,9 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         ++pack_log2;
     const int R = kBM >> pack_log2;
     const long long qtiles = (a->max_q_len + 2 * R - 1) / (2 * R);
-    if ((long long)a->batch * a->n_layers > 65535 || a->n_heads_q > 65535 || qtiles > 0x7fffffff)
-        return SONIC_ERR_UNSUPPORTED;
+    const long long HG = a->n_heads_q >> pack_log2;
+    const long long n_units = qtiles * HG * a->batch * a->n_layers;
+    if (n_units > 0x7fffffff) return SONIC_ERR_UNSUPPORTED;
 
     const uint64_t qrow = (uint64_t)a->n_heads_q * D, krow = (uint64_t)a->n_heads_kv * D;
     const uint64_t q_layer = a->n_layers > 1 ? (uint64_t)a->q_layer_stride * 2
@@ -1324,8 +1610,12 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.lse = a->lse;
     p.nexus_mass = a->nexus_mass;
     p.status = a->status;
-    p.sums = static_cast<const TileSum *>(a->workspace);
+    p.sums = reinterpret_cast<const TileSum *>(wsb + ws.sums);
     p.masks = reinterpret_cast<const TileMasks *>(wsb + ws.masks);
+    p.counter = reinterpret_cast<int32_t *>(wsb + ws.counter);
+    p.n_units = (int)n_units;
+    p.qtiles = (int)qtiles;
+    p.HG = (int)HG;
     p.max_k_tiles = max_k_tiles_of(a);
     p.max_k_len = a->max_k_len;
     p.B = a->batch;
@@ -1358,10 +1648,11 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     }
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
         p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
-        static_cast<TileSum *>(a->workspace), reinterpret_cast<TileMasks *>(wsb + ws.masks),
+        reinterpret_cast<TileSum *>(wsb + ws.sums), reinterpret_cast<TileMasks *>(wsb + ws.masks),
         p.max_k_tiles,
-        reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status);
-    dim3 grid((unsigned)qtiles, a->n_heads_q >> pack_log2, a->batch * a->n_layers);
+        reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status, p.counter);
+    // one persistent block per SM (fewer when there are fewer units)
+    const int grid = (int)std::min<long long>(device_sm_count(), n_units);
     cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
                                : launch_prefill<64>(tq, tk, tv, p, grid, stream);
     return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;

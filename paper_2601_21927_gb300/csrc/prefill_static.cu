@@ -25,10 +25,11 @@
 
 namespace {
 
-// 9 MiB: room for 32768 key tiles, each with a 32-byte summary and a
-// 256-byte column-mask record, i.e. batch * ceil(max_k_len / 128) <= 32768
-// (for example 64 sequences of up to 65536 keys).
-constexpr size_t kStaticScratchBytes = size_t(9) << 20;
+// 9 MiB + 256 bytes: the work-unit counter and room for 32768 key tiles, each
+// with a 32-byte summary and a 256-byte column-mask record, i.e.
+// batch * ceil(max_k_len / 128) <= 32768 (for example 64 sequences of up to
+// 65536 keys).
+constexpr size_t kStaticScratchBytes = (size_t(9) << 20) + 256;
 
 static __device__ __align__(256) unsigned char g_prefill_scratch[kStaticScratchBytes];
 

@@ -101,12 +101,22 @@ __device__ __forceinline__ uint64_t global_ns() {
     return t;
 }
 
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity,
+                                                   int32_t *status, volatile int *abort);
+
 // Bounded wait for the phase with the given parity to complete.  On timeout
 // records SONIC_ERR_DEVICE_TIMEOUT, raises *abort and returns false.  A wait
 // also gives up early once another thread of the block has raised *abort.
+// The first test is inline; the polling loop is one out-of-line copy per
+// translation unit, which keeps the kernels' hot loops short.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int32_t *status,
                                           volatile int *abort) {
     if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, status, abort);
+}
+
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity,
+                                                   int32_t *status, volatile int *abort) {
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -118,6 +128,24 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int32_
     set_status(status, SONIC_ERR_DEVICE_TIMEOUT);
     *abort = 1;
     return false;
+}
+
+// Longest a drain waits for one phase (ns).  Independent of
+// SONIC_WAIT_LIMIT_NS: a drain runs after an abort, when the work it waits
+// for is already issued and ends on its own.
+#ifndef SONIC_DRAIN_LIMIT_NS
+#define SONIC_DRAIN_LIMIT_NS 1000000000ull
+#endif
+
+// Wait for the phase with the given parity whatever *abort says, bounded by
+// SONIC_DRAIN_LIMIT_NS: lets issued copies and tensor-core work finish before a
+// block frees tensor memory or exits.  Returns false if the limit ran out.
+__device__ __forceinline__ bool mbar_drain(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (global_ns() - t0 > SONIC_DRAIN_LIMIT_NS) return false;
+    return true;
 }
 
 // ---------------------------------------------------------------- TMA

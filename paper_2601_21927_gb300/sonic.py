@@ -279,7 +279,7 @@ def sonic_attn_prefill_static(Q: torch.Tensor, K: torch.Tensor, V: torch.Tensor,
                               softmax_scale: float = 0.0, nexus_vis: int = NEXUS_FULL, lse=None,
                               status=None, nexus_mass=None, stream=None):
     """sonic_attn_prefill for callers that cannot allocate device memory: the
-    library keeps the tile summaries and masks in a fixed 9 MiB device array, so
+    library keeps the tile summaries and masks in a fixed ~9 MiB device array, so
     no workspace is passed (and this wrapper allocates nothing either).
     Calls overlapping on the GPU share that array and must be serialised."""
     lib = load()

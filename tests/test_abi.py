@@ -85,9 +85,9 @@ def test_host_validation_rejects_before_launch():
     assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 1
     p.nexus_vis = 0
     assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 3  # workspace
-    # one key tile: its summary (32 B) and its column masks (256 B), each part
-    # rounded up to 256 bytes
-    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256 + 256
+    # the work-unit counter (256 B), then one key tile: its summary (32 B) and
+    # its column masks (256 B), each part rounded up to 256 bytes
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256 + 256 + 256
     p.key_order = 7
     assert lib.sonic_attn_prefill(16, 16, 16, 16, 16, 16, ctypes.byref(p), None) == 1
     # the fixed-scratch entry point serves only the as-given key order
@@ -116,22 +116,22 @@ def test_python_binding_has_no_cpu_path():
 
 
 def test_retained_first_workspace_size():
-    """Workspace of the retained-first order: tile summaries (32 B) and column
-    masks (256 B) of one extra tile per sequence, 13 bytes of metadata per
-    permuted row, and a K and a V copy of every layer; each part rounded up to
-    256 bytes."""
+    """Workspace of the retained-first order: the work-unit counter (256 B),
+    tile summaries (32 B) and column masks (256 B) of one extra tile per
+    sequence, 13 bytes of metadata per permuted row, and a K and a V copy of
+    every layer; each part rounded up to 256 bytes."""
     lib = sonic.load()
     p = sonic.sonic_prefill_args()
     p.batch, p.n_layers, p.n_heads_q, p.n_heads_kv, p.head_dim = 2, 3, 8, 4, 128
     p.max_q_len, p.max_k_len, p.total_q_rows, p.total_k_rows = 300, 300, 600, 600
-    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256 + 1536  # 2 * 3 tiles
+    assert lib.sonic_prefill_workspace_size(ctypes.byref(p)) == 256 + 256 + 1536  # 2 * 3 tiles
     p.key_order = sonic.KEYS_RETAINED_FIRST
 
     def r256(x):
         return (x + 255) // 256 * 256
 
     def expect(rows):
-        return (r256(2 * 4 * 32) + r256(2 * 4 * 256) + r256(3 * 4) + r256(2 * 4) + r256(rows)
+        return (256 + r256(2 * 4 * 32) + r256(2 * 4 * 256) + r256(3 * 4) + r256(2 * 4) + r256(rows)
                 + 3 * r256(4 * rows)
                 + 2 * r256(3 * rows * 4 * 128 * 2))
 
