@@ -45,20 +45,18 @@ def _stamp() -> str:
     return h.hexdigest()
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile libsonic.so if its sources changed; returns its path."""
-    os.makedirs(OUT_DIR, exist_ok=True)
-    stamp_path = os.path.join(OUT_DIR, "libsonic.stamp")
-    stamp = _stamp()
-    if (not force and os.path.exists(LIB) and os.path.exists(stamp_path)
-            and open(stamp_path).read() == stamp):
-        return LIB
+def compile_library(lib_path: str, sources=SOURCES, defines=(), verbose: bool = False) -> str:
+    """Compile `sources` (names under csrc/) with extra -D `defines` into the
+    shared library `lib_path` (objects beside it); returns its path."""
+    out_dir = os.path.dirname(os.path.abspath(lib_path))
+    os.makedirs(out_dir, exist_ok=True)
     nvcc = _nvcc()
-    objs = []
+    tag = os.path.splitext(os.path.basename(lib_path))[0]
 
     def compile_one(src):
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
-        cmd = [nvcc] + ARCH + NVCC_FLAGS + ["-c", os.path.join(CSRC, src), "-o", obj]
+        obj = os.path.join(out_dir, f"{tag}_{src.replace('.cu', '.o')}")
+        cmd = ([nvcc] + ARCH + NVCC_FLAGS + ["-D" + d for d in defines] +
+               ["-c", os.path.join(CSRC, src), "-o", obj])
         if verbose:
             cmd += ["-Xptxas", "-v"]
         r = subprocess.run(cmd, capture_output=True, text=True)
@@ -68,14 +66,26 @@ def build(force: bool = False, verbose: bool = False) -> str:
             print(r.stderr)
         return obj
 
-    with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB + f".tmp{os.getpid()}"
+    with ThreadPoolExecutor(max_workers=len(sources)) as ex:
+        objs = list(ex.map(compile_one, sources))
+    tmp = lib_path + f".tmp{os.getpid()}"
     cmd = [nvcc] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    os.replace(tmp, lib_path)
+    return lib_path
+
+
+def build(force: bool = False, verbose: bool = False) -> str:
+    """Compile libsonic.so if its sources changed; returns its path."""
+    os.makedirs(OUT_DIR, exist_ok=True)
+    stamp_path = os.path.join(OUT_DIR, "libsonic.stamp")
+    stamp = _stamp()
+    if (not force and os.path.exists(LIB) and os.path.exists(stamp_path)
+            and open(stamp_path).read() == stamp):
+        return LIB
+    compile_library(LIB, SOURCES, verbose=verbose)
     with open(stamp_path, "w") as f:
         f.write(stamp)
     return LIB

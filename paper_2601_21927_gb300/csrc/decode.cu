@@ -271,6 +271,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         return w.u >= 0;
     };
 
+    int issued_q = 0, issued_kv = 0;  // copies the producer issued (for the drain)
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
@@ -285,7 +286,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
         // after them.
         if (lane == 0) {
             tma_prefetch_desc(&tmQ);
-            int T = 0;
+            int T = 0;  // K/V tiles issued
             int pending = atomicAdd(unit_counter, 1);
             for (int k = 0;; ++k) {
                 const int slot = k & (kUnitSlots - 1);
@@ -317,6 +318,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 for (int hh = 0; hh < kHalves; ++hh)
                     tma_load_4d(q_s + qb * C::kQBytes + hh * (kTcN * 128), &tmQ, &q_full[qb],
                                 hh * 64, kvh0 * G, w.b, w.layer);
+                issued_q = k + 1;
                 for (int t = 0; t < w.ntiles; ++t, ++T) {
                     const int s = T % kTcStages;
                     if (T >= kTcStages &&
@@ -357,10 +359,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 }
                 if (!ok) break;
             }
-            if (*abort_flag) {
-                for (int u = max(0, T - kTcStages); u < T; ++u)
-                    mbar_wait(&full[u % kTcStages], (u / kTcStages) & 1, p.status, abort_flag);
-            }
+            issued_kv = T;
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -470,8 +469,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
                 more = has_next;
                 w = nx;
             }
+            // every MMA issued by this thread has finished once this arrives (a
+            // wait bounded by time alone: tensor memory is freed after it)
             tc_commit(mma_idle);
-            mbar_wait(mma_idle, 0, p.status, abort_flag);
+            mbar_drain(mma_idle, 0);
         }
     } else {
         // ------------------------------------------------------------ softmax
@@ -693,6 +694,16 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant_
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // After an abort no thread waits any more; let the copies the producer
+    // issued land before the block's shared memory goes away (older ones have:
+    // their buffers were waited free before being refilled).
+    if (*abort_flag && warp == 0 && lane == 0) {
+        for (int k = max(0, issued_q - C::kQBufs); k < issued_q; ++k)
+            mbar_drain(&q_full[k % C::kQBufs], (k / C::kQBufs) & 1);
+        for (int u = max(0, issued_kv - kTcStages); u < issued_kv; ++u)
+            mbar_drain(&full[u % kTcStages], (u / kTcStages) & 1);
+    }
+    __syncthreads();
     if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 

@@ -209,6 +209,10 @@ __device__ __forceinline__ GemmTile gemm_tile(int i, int n0, int n1, int mt0, in
     return w;
 }
 
+// After an abort, how long the non-leading CTA of a pair leaves its issued
+// copies to land before it may exit (ns).
+constexpr uint64_t kCopyGraceNs = 200000;
+
 // ---- CTA-pair primitives (clusters of two CTAs; rank 0 leads)
 
 __device__ __forceinline__ uint32_t cluster_rank() {
@@ -332,6 +336,7 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
 
+    int issued = 0;  // pipeline stages this CTA's producer filled (for the drain)
     if (warp == 0) {
         // ------------------------------------------------------------ producers
         // Each CTA loads its 128 rows of A and its 128 weight rows; both
@@ -366,12 +371,8 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     tma_load_pair(a, ta, bar, kb * kGBK, arow);
                     tma_load_pair(a + C::kABytes, tb, bar, kb * kGBK,
                                   w.n * kGBN + (int)rank * kHalfN);
+                    issued = it + 1;
                 }
-            }
-            if (*abort_flag && rank == 0) {
-                // let the copies already issued land before the pair exits
-                for (int u = max(0, it - kGStages); u < it; ++u)
-                    mbar_wait(&full[u % kGStages], (u / kGStages) & 1, p.status, abort_flag);
             }
         }
     } else if (warp == 1) {
@@ -405,8 +406,10 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                 }
                 if (ok) commit_pair(&acc_full[b], 3);
             }
+            // every MMA issued by this thread has finished once this arrives (a
+            // wait bounded by time alone: the pair's memory is released after it)
             commit_pair(mma_idle, 1);
-            mbar_wait(mma_idle, 0, p.status, abort_flag);
+            mbar_drain(mma_idle, 0);
         }
     } else {
         // ------------------------------------------------------------ epilogue
@@ -458,6 +461,22 @@ routed_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         }
     }
     tc_fence_before();
+    __syncthreads();
+    // After an abort no thread of this CTA waits any more; let the copies in
+    // flight land before the pair's memory goes away.  Both CTAs' copies of a
+    // stage complete on the leader's barrier, so the leader drains the stages
+    // it armed; the other CTA cannot wait on that barrier and gives its own
+    // copies a bounded grace period instead (a copy that is issued lands in
+    // microseconds).
+    if (*abort_flag && warp == 0 && lane == 0) {
+        if (rank == 0) {
+            for (int u = max(0, issued - kGStages); u < issued; ++u)
+                mbar_drain(&full[u % kGStages], (u / kGStages) & 1);
+        } else if (issued > 0) {
+            const uint64_t t0 = global_ns();
+            while (global_ns() - t0 < kCopyGraceNs) __nanosleep(1000);
+        }
+    }
     __syncthreads();
     cluster_sync_all();  // no CTA leaves while its pair may still touch its memory
     tc_fence_after();

@@ -18,6 +18,11 @@
 #ifndef SONIC_WAIT_LIMIT_NS
 #define SONIC_WAIT_LIMIT_NS 2000000000ull
 #endif
+// A waiting thread reads the clock (and the block's abort flag) once every
+// SONIC_WAIT_CHECK_MASK + 1 polls.
+#ifndef SONIC_WAIT_CHECK_MASK
+#define SONIC_WAIT_CHECK_MASK 255u
+#endif
 
 namespace sonic {
 
@@ -120,7 +125,7 @@ static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parit
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 0) {
+        if ((i & SONIC_WAIT_CHECK_MASK) == 0) {
             if (*abort) return false;
             if (global_ns() - t0 > SONIC_WAIT_LIMIT_NS) break;
         }

@@ -116,12 +116,20 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         if not build_if_missing:
             raise ImportError(f"libsonic.so not built ({path}); run __graft_entry__.build()")
         _build.build()
+    _lib = open_library(path)
+    return _lib
+
+
+def open_library(path: str) -> ctypes.CDLL:
+    """A libsonic build at `path` with the C signatures applied (entry points
+    the build lacks are skipped)."""
     lib = ctypes.CDLL(path)
     for name, (res, args) in SIGNATURES.items():
+        if not hasattr(lib, name):
+            continue
         fn = getattr(lib, name)
         fn.restype = res
         fn.argtypes = args
-    _lib = lib
     return lib
 
 
