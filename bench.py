@@ -628,9 +628,11 @@ def extra_masked_prefill():
     for mode in (0, 1):
         flops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L), mode) * batch.B
         for order, oname in ((0, "as_given"), (1, "retained_first")):
-            ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+            call = lambda ws=None: sonic.sonic_attn_prefill(
                 Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks, q_len=kl, max_q_len=L,
-                max_k_len=L, nexus_vis=mode, key_order=order))
+                max_k_len=L, nexus_vis=mode, key_order=order, workspace=ws)
+            ws = call()
+            ms = _ev_time(lambda: call(ws))
             res[f"all_rows_{'full' if mode == 0 else 'causal_segments'}_{oname}"] = {
                 "ms": round(ms, 3), "tflops": round(flops / ms / 1e9, 1)}
     ql = np.full(batch.B, d.curr_len, np.int32)
@@ -638,10 +640,13 @@ def extra_masked_prefill():
     Qc = inputs.randn((1, int(ql.sum()), hd.hq, hd.d), seed=4, device=dev)
     Oc = torch.empty_like(Qc)
     flops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L - d.curr_len, L), 0) * batch.B
+    qst, qlt = t(qs), t(ql)
     for order, oname in ((0, "as_given"), (1, "retained_first")):
-        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
-            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=t(qs), q_len=t(ql),
-            max_q_len=int(ql.max()), max_k_len=L, key_order=order))
+        call = lambda ws=None: sonic.sonic_attn_prefill(
+            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=qst, q_len=qlt,
+            max_q_len=int(ql.max()), max_k_len=L, key_order=order, workspace=ws)
+        ws = call()
+        ms = _ev_time(lambda: call(ws))
         res[f"current_rows_{oname}"] = {"ms": round(ms, 3), "tflops": round(flops / ms / 1e9, 1)}
     return {"workload": "masked prefill, batch 8 x 5632 rows, 32/8 heads, D=128, 1 layer",
             "results": res}
@@ -669,17 +674,22 @@ def extra_prefill_d64():
         Q = inputs.randn((1, batch.total, 32, D), seed=3, device=dev)
         O = torch.empty_like(Q)
         flops = 4.0 * D * 32 * _visible_pairs(role, seg, range(L), 0) * batch.B
-        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
+        call = lambda ws=None: sonic.sonic_attn_prefill(
             Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks, q_len=kl, max_q_len=L,
-            max_k_len=L, key_order=1))
+            max_k_len=L, key_order=1, workspace=ws)
+        ws = call()
+        ms = _ev_time(lambda: call(ws))
         res[f"all_rows_retained_first_d{D}"] = {"ms": round(ms, 3),
                                                 "tflops": round(flops / ms / 1e9, 1)}
         Qc = inputs.randn((1, int(ql.sum()), 32, D), seed=4, device=dev)
         Oc = torch.empty_like(Qc)
         flops = 4.0 * D * 32 * _visible_pairs(role, seg, range(L - d.curr_len, L), 0) * batch.B
-        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
-            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=t(qs), q_len=t(ql),
-            max_q_len=int(ql.max()), max_k_len=L, key_order=1))
+        qst, qlt = t(qs), t(ql)
+        call = lambda ws=None: sonic.sonic_attn_prefill(
+            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=qst, q_len=qlt,
+            max_q_len=int(ql.max()), max_k_len=L, key_order=1, workspace=ws)
+        ws = call()
+        ms = _ev_time(lambda: call(ws))
         res[f"current_rows_retained_first_d{D}"] = {"ms": round(ms, 3),
                                                     "tflops": round(flops / ms / 1e9, 1)}
     return {"workload": "masked prefill, batch 8 x 5632 rows, 32/8 heads, head_dim 64 and 128",
@@ -803,14 +813,16 @@ def extra_nexus_gen():
 
     def prefills():
         for s in steps:
-            sonic.sonic_attn_prefill(s["Q"], s["K"], s["V"], s["seg"], s["role"], s["O"],
-                                     k_start=s["ks"], k_len=s["kl"], q_start=s["qs"],
-                                     q_len=s["ql"], max_q_len=s["nk"], max_k_len=s["L"])
+            s["ws_p"] = sonic.sonic_attn_prefill(
+                s["Q"], s["K"], s["V"], s["seg"], s["role"], s["O"], k_start=s["ks"],
+                k_len=s["kl"], q_start=s["qs"], q_len=s["ql"], max_q_len=s["nk"],
+                max_k_len=s["L"], workspace=s.get("ws_p"))
 
     def compactions():
         for s in steps:
-            sonic.sonic_compact_kv(s["K"], s["V"], s["seg"], s["role"], s["oK"], s["oV"],
-                                   s["off"], k_start=s["ks"], k_len=s["kl"])
+            s["ws_c"] = sonic.sonic_compact_kv(s["K"], s["V"], s["seg"], s["role"], s["oK"],
+                                               s["oV"], s["off"], k_start=s["ks"], k_len=s["kl"],
+                                               workspace=s.get("ws_c"))
 
     p_ms = _ev_time(prefills)
     c_ms = _ev_time(compactions)
