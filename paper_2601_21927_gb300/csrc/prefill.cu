@@ -2,9 +2,11 @@
 // mask (Sec. 3.2: Eq. 3 causal rule, Eq. 4 historical body removal, Eq. 5
 // bidirectional Nexus visibility), on the sm_103a tensor cores.
 //
-// A work unit is two 128-row query tiles of one (layer, sequence, query head
-// group).  One persistent block per SM claims units from a counter; eleven
-// warps:
+// A work unit is two 128-row query tiles of one (layer, sequence): one query
+// block of two query heads that share a KV head (so both tiles see the same
+// keys), or, where the heads do not pair, two consecutive query blocks of one
+// query head group.  One persistent block per SM claims units from a counter;
+// eleven warps:
 //   warp 0     TMA producer: each unit's Q tiles, then K and V tiles (128
 //              keys) into a 2-stage ring, with the column masks of the tiles
 //              the mask cuts;
@@ -96,7 +98,10 @@ struct PfParams {
     int B, Hq, G;
     int64_t total_k_rows;  // rows of role, seg_id (and K, V) per layer
     int pack_log2;  // query heads per tile row group: a tile is 128 >> pack_log2 rows x (1 << pack_log2) heads
+    int pair;       // 1: a unit's two query tiles are one 128-row block of two query heads
+                    // sharing a KV head (else two consecutive 128-row blocks of one)
     int64_t o_ls;
+    int o_v8;  // O and its layer stride 32-byte aligned: the epilogue writes whole 32-byte sectors
     int total_q_rows;
     float scale_log2;
     int nexus_mode;
@@ -460,8 +465,11 @@ __device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8
 }
 
 // One persistent block per SM walks work units: a unit is two 128-row query
-// tiles (tile 0 = rows 0..127 of its 256, tile 1 = rows 128..255) of one
-// (layer, sequence, query-head group).  Eleven warps (352 threads):
+// tiles of one (layer, sequence).  Paired (pair = 1: unpacked heads, an even
+// number per KV head): one query block of heads h0 (tile 0) and h0 + 1
+// (tile 1), whose key-tile lists are then the same.  Otherwise: rows 0..127
+// (tile 0) and 128..255 (tile 1) of a 256-row block of one query-head group.
+// Eleven warps (352 threads):
 //   warp 0       TMA producer: the unit's Q tiles, then K, V (and the key
 //                metadata of cut tiles) into a 2-stage ring that runs on
 //                across units;
@@ -523,6 +531,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     // R = 128 / P): tile row r is query row r / P, head h0 + r % P.  P > 1 packs
     // the heads of short query blocks so the tile rows are not left empty.
     const int pl2 = p.pack_log2, R = kBM >> pl2;
+    // query rows of a unit, and the row offset of its second query tile
+    const int urows = p.pair ? R : 2 * R, qstep = p.pair ? 0 : R;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     if (tid == 0) {
@@ -589,7 +599,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     if (lane == 0 && hg == 0 && qt == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
                     continue;
                 }
-                if (qt * 2 * R >= qlen) continue;  // no query rows in this block
+                if (qt * urows >= qlen) continue;  // no query rows in this block
                 kklen = p.key_len[b];
                 if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
                     // the host-side bounds were wrong for this sequence: refuse it
@@ -618,8 +628,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
                 break;
             }
-            const int pbase = klen - qlen + qt * 2 * R;  // position of query row 0 of tile 0
-            const bool tile1 = qt * 2 * R + R < qlen;
+            const int pbase = klen - qlen + qt * urows;  // position of query row 0 of tile 0
+            const bool tile1 = p.pair || qt * 2 * R + R < qlen;
             // summaries of the query tiles: segment range, Nexus rows and their
             // segment range
             int qf[2], qs0[2], qs1[2], qn0[2], qn1[2];
@@ -627,7 +637,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             for (int qi = 0; qi < 2; ++qi) {
                 int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
                 for (int r = lane; r < R; r += 32) {
-                    const int pos = pbase + qi * R + r;
+                    const int pos = pbase + qi * qstep + r;
                     if (pos <= klen - 1) {
                         const int ro = p.role[kstart + pos];
                         const int s = p.seg[kstart + pos];
@@ -672,7 +682,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     entry = (t << 6) | ((kn ? ((kb || ko) ? 2 : 1) : 0) << 4);
 #pragma unroll
                     for (int qi = 0; qi < 2; ++qi) {
-                        const int p0 = pbase + qi * R;
+                        const int p0 = pbase + qi * qstep;
                         const int p1 = min(p0 + R - 1, klen - 1);
                         if (p0 > p1) continue;
                         const bool q_has_nexus = qf[qi] & 2;
@@ -713,7 +723,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 ui->flags = dense ? 2 : 0;
                 ui->layer = layer;
                 ui->b = b;
-                ui->h0 = hg << pl2;
+                ui->h0 = p.pair ? 2 * hg : hg << pl2;
                 ui->qt = qt;
                 ui->nq = tile1 ? 2 : 1;
                 ui->n_list = n_list;
@@ -760,7 +770,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                         for (int hh = 0; hh < C::kHalves; ++hh)
                             tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
-                                        hh * 64, ui->h0, ui->qstart + ui->qt * 2 * R + qi * R,
+                                        hh * 64, ui->h0 + qi * p.pair,
+                                        ui->qstart + ui->qt * urows + qi * qstep,
                                         layer);
                 }
                 ++issued_q;
@@ -1015,7 +1026,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const bool udense = ui->flags & 2;
                 const int last = udense ? n_list - 1 : ui->last[qi];
                 const int kklen = ui->kklen;
-                const int pos = ui->pbase + qi * R + qr;
+                const int pos = ui->pbase + qi * qstep + qr;
                 int rp = SONIC_ROLE_SYS, sp = 0;
                 if (pos <= ui->klen - 1) {
                     rp = p.role[ui->kstart + pos];
@@ -1186,8 +1197,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     m_used = m_new;
                 }
                 if (!ok) break;
-                const int layer = ui->layer, h = ui->h0 + hoff;
-                const int qidx = ui->qt * 2 * R + qi * R + qr;  // query row within the sequence
+                const int layer = ui->layer, h = ui->h0 + qi * p.pair + hoff;
+                const int qidx = ui->qt * urows + qi * qstep + qr;  // query row within the sequence
                 const bool row_ok = pos <= ui->klen - 1 && qidx < ui->qlen;
                 const int64_t qrow = (int64_t)ui->qstart + qidx;
                 uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
@@ -1210,15 +1221,21 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                             mbar_arrive(&o_free[qi]);
                         }
                         if (row_ok) {
-                            uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+                            // a thread writes its own row: in 32-byte stores a warp's
+                            // store fills 32 whole L2 sectors, in 16-byte ones half of each
+                            uint32_t w[16];
 #pragma unroll
-                            for (int u = 0; u < 4; ++u) {
-                                uint32_t w[4];
+                            for (int x = 0; x < 16; ++x)
+                                w[x] = pack_bf16x2(__uint_as_float(o[2 * x]) * inv,
+                                                   __uint_as_float(o[2 * x + 1]) * inv);
+                            if (p.o_v8) {
+                                st_global_v8(orow + c * 32, w);
+                                st_global_v8(orow + c * 32 + 16, w + 8);
+                            } else {
+                                uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
 #pragma unroll
-                                for (int x = 0; x < 4; ++x)
-                                    w[x] = pack_bf16x2(__uint_as_float(o[u * 8 + 2 * x]) * inv,
-                                                       __uint_as_float(o[u * 8 + 2 * x + 1]) * inv);
-                                dst[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                                for (int u = 0; u < 4; ++u)
+                                    dst[u] = make_uint4(w[4 * u], w[4 * u + 1], w[4 * u + 2], w[4 * u + 3]);
                             }
                         }
                     }
@@ -1557,8 +1574,12 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
            (long long)a->max_q_len * (2 << pack_log2) <= 2 * kBM)
         ++pack_log2;
     const int R = kBM >> pack_log2;
-    const long long qtiles = (a->max_q_len + 2 * R - 1) / (2 * R);
-    const long long HG = a->n_heads_q >> pack_log2;
+    // Unpacked heads in pairs sharing a KV head: a unit's two query tiles
+    // then see the same keys (no key tile visited by one tile alone).
+    const bool pair = pack_log2 == 0 && G % 2 == 0;
+    const long long urows = pair ? R : 2 * R;
+    const long long qtiles = (a->max_q_len + urows - 1) / urows;
+    const long long HG = pair ? a->n_heads_q / 2 : a->n_heads_q >> pack_log2;
     const long long n_units = qtiles * HG * a->batch * a->n_layers;
     if (n_units > 0x7fffffff) return SONIC_ERR_UNSUPPORTED;
 
@@ -1623,7 +1644,9 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.G = G;
     p.total_k_rows = a->total_k_rows;
     p.pack_log2 = pack_log2;
+    p.pair = pair ? 1 : 0;
     p.o_ls = a->o_layer_stride;
+    p.o_v8 = (reinterpret_cast<uintptr_t>(O) % 32 == 0) && (a->o_layer_stride * 2) % 32 == 0;
     p.total_q_rows = a->total_q_rows;
     const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / sqrtf((float)D);
     p.scale_log2 = scale * kLog2ef;

@@ -170,6 +170,14 @@ __device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *map, u
         : "memory");
 }
 
+// Eight words (32 bytes, one L2 sector) to global memory in one store; dst must
+// be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void *dst, const uint32_t *w) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(w[0]),
+                 "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+
 // Make this thread's generic-proxy shared-memory writes visible to the async
 // proxy (tensor cores, TMA).
 __device__ __forceinline__ void fence_proxy_async_smem() {

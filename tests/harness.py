@@ -45,8 +45,10 @@ def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed
                 nexus_vis: int = sonic.NEXUS_FULL, n_layers: int = 1, with_lse: bool = True,
                 K=None, V=None, Q=None, key_order: int = sonic.KEYS_AS_GIVEN,
                 expect_status: int = 0, k_start=None, total_k_rows=None,
-                with_mass: bool = False):
+                with_mass: bool = False, o_offset: int = 0):
     """Prefill of the last q_len[b] rows of every sequence (all rows if None).
+    o_offset > 0: O starts o_offset elements into a NaN-filled buffer whose
+    layers are o_offset elements apart (res["O_buf"]).
     Returns a dict with the device tensors and the query layout."""
     role, seg, k_start_b, k_len = meta(batch)
     k_start = k_start_b if k_start is None else i32(k_start)
@@ -61,7 +63,15 @@ def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed
         V = inputs.randn((n_layers, T, hkv, D), seed=seed + 2, device=dev())
     if Q is None:
         Q = inputs.randn((n_layers, Tq, hq, D), seed=seed + 3, device=dev())
-    O = torch.full_like(Q, float("nan"))
+    O_buf = None
+    if o_offset:
+        n = Tq * hq * D
+        O_buf = torch.full((n_layers * (n + o_offset) + o_offset,), float("nan"),
+                           dtype=torch.bfloat16, device=dev())
+        O = O_buf.as_strided((n_layers, Tq, hq, D), (n + o_offset, hq * D, D, 1),
+                             storage_offset=o_offset)
+    else:
+        O = torch.full_like(Q, float("nan"))
     lse = torch.full((n_layers, Tq, hq), float("nan"), device=dev()) if with_lse else None
     mass = torch.full((n_layers, Tq, hq), float("nan"), device=dev()) if with_mass else None
     status = torch.zeros(1, dtype=torch.int32, device=dev())
@@ -72,7 +82,7 @@ def run_prefill(batch: inputs.Batch, hq: int, hkv: int, D: int, q_len=None, seed
                              nexus_mass=mass)
     torch.cuda.synchronize()
     assert sonic.read_status(status) == expect_status
-    return dict(K=K, V=V, Q=Q, O=O, lse=lse, mass=mass, q_len=q_len, q_start=q_start)
+    return dict(K=K, V=V, Q=Q, O=O, lse=lse, mass=mass, q_len=q_len, q_start=q_start, O_buf=O_buf)
 
 
 def oracle_prefill_rows(batch: inputs.Batch, res: dict, b: int, rows, layer: int = 0,

@@ -38,6 +38,29 @@ def test_random_dialogues_multi_tile(mode, order):
     _all_rows(inputs.Batch(ds), 4, 2, 128, mode=mode, seed=5, order=order)
 
 
+@pytest.mark.parametrize("D", [64, 128])
+def test_output_only_16_byte_aligned(D):
+    """O 16 bytes past a 32-byte boundary, with a layer stride that is not a
+    multiple of 32 bytes: the epilogue takes its 16-byte stores, every row
+    matches the oracle on both layers, and no element outside O is written."""
+    rng = np.random.default_rng(17)
+    batch = inputs.Batch([inputs.random_dialogue(rng, max_segments=4, max_body=150, max_nexus=30,
+                                                 max_curr=140) for _ in range(3)])
+    off = 8  # bf16 elements: 16 bytes
+    res = H.run_prefill(batch, 4, 2, D, seed=21, n_layers=2, o_offset=off)
+    assert res["O"].data_ptr() % 32 == 16 and (res["O"].stride(0) * 2) % 32 == 16
+    for layer in (0, 1):
+        for b in range(batch.B):
+            n = int(batch.k_len[b])
+            O, lse, got, got_lse = H.oracle_prefill_rows(batch, res, b, np.arange(n), layer=layer)
+            H.check_close(got, O, f"layer {layer} seq {b}")
+            np.testing.assert_allclose(got_lse, lse, rtol=0, atol=2e-3)
+    n = res["O"][0].numel()
+    buf = res["O_buf"]
+    gaps = torch.cat([buf[:off], buf[off + n:2 * off + n], buf[2 * off + 2 * n:]])
+    assert gaps.numel() == 3 * off and torch.isnan(gaps.float()).all()
+
+
 @pytest.mark.parametrize("order", ORDERS)
 def test_head_dim_64_and_gqa_ratios(order):
     rng = np.random.default_rng(3)
