@@ -1082,6 +1082,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
                     // row maximum (masked keys set to -inf on a cut tile)
                     float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    // 32-key chunks hidden from every row of the warp: no maximum, no
+                    // exponentials, zero probabilities (bit c; warp-uniform)
+                    uint32_t zchunk = 0;
                     if (!cut) {
 #pragma unroll
                         for (int c = 0; c < 4; ++c)
@@ -1092,11 +1095,24 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     } else {
 #pragma unroll
                         for (int c = 0; c < 4; ++c)
+                        {
+                            // chunks the whole warp sees, or sees none of, skip the
+                            // per-key mask (both common away from a causal diagonal)
+                            if (__all_sync(0xffffffffu, mbits[c] == 0xffffffffu)) {
 #pragma unroll
-                            for (int x = 0; x < 32; ++x) {
-                                if (!((mbits[c] >> x) & 1)) sr[c][x] = __float_as_uint(-INFINITY);
-                                mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][x]));
+                                for (int x = 0; x < 32; x += 2)
+                                    mx4[c] = fmax3(mx4[c], __uint_as_float(sr[c][x]),
+                                                   __uint_as_float(sr[c][x + 1]));
+                            } else if (__all_sync(0xffffffffu, mbits[c] == 0u)) {
+                                zchunk |= 1u << c;
+                            } else {
+#pragma unroll
+                                for (int x = 0; x < 32; ++x) {
+                                    if (!((mbits[c] >> x) & 1)) sr[c][x] = __float_as_uint(-INFINITY);
+                                    mx4[c] = fmaxf(mx4[c], __uint_as_float(sr[c][x]));
+                                }
                             }
+                        }
                     }
                     const float mx =
                         fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * p.scale_log2;
@@ -1133,6 +1149,12 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                         for (int c = 0; c < 4; ++c) {
                             uint32_t pk[16];
+                            if ((zchunk >> c) & 1) {
+#pragma unroll
+                                for (int x = 0; x < 16; ++x) pk[x] = 0u;
+                                tmem_st16(tS + c * 16, pk);
+                                continue;
+                            }
 #pragma unroll
                             for (int x = 0; x < 32; x += 2) {
                                 const float2 v = __ffma2_rn(make_float2(__uint_as_float(sr[c][x]),
