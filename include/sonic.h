@@ -93,11 +93,14 @@ typedef enum {
 
 /* Order in which sonic_attn_prefill walks a sequence's keys.
  * AS_GIVEN: the key rows as laid out (S_aug order).
- * RETAINED_FIRST: the library first copies each sequence's keys (K and V of
- * every layer, role, segment) into its workspace as [system prompt, Nexus and
+ * RETAINED_FIRST: the library first lays each sequence's keys out in its
+ * workspace (role, segment, position) as [system prompt, Nexus and
  * current-turn rows | history bodies], each part in S_aug order and the
  * bodies starting on a 128-row boundary; the mask still compares S_aug
- * positions.  Every query row then sees one prefix of the retained part plus
+ * positions.  A 128-key tile of that order made of 128 consecutive rows of
+ * K and V (a stretch of one body, of the system prompt or of the current
+ * turn) is read from K and V in place; the K and V rows of every other tile
+ * are copied into the workspace, for every layer.  Every query row then sees one prefix of the retained part plus
  * (for body and Nexus rows) the body of its own segment, so far fewer key
  * tiles are visited and cut by the mask when all rows of S_aug are queried.
  * Results equal AS_GIVEN up to floating-point summation order.  The copy
@@ -232,8 +235,8 @@ SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K
  * batch).  AS_GIVEN: 256 bytes for the counter the persistent blocks claim
  * work units from, then 32 + 256 bytes per 128-key tile (its summary and its
  * column masks), batch * ceil(max_k_len / 128) tiles, each part rounded up to
- * 256 bytes.  RETAINED_FIRST counts one more tile per sequence and adds, for
- * R = min(batch * (align128(max_k_len) + 128),
+ * 256 bytes.  RETAINED_FIRST counts one more tile per sequence and adds 4
+ * bytes per tile and, for R = min(batch * (align128(max_k_len) + 128),
  * total_k_rows + 256 * batch) rows: 13 bytes of metadata per row and a K and
  * a V copy of R rows for every layer (2 * n_layers * R * n_heads_kv *
  * head_dim * 2 bytes).  Sequence b takes align128(k_len[b]) + 128 of the R

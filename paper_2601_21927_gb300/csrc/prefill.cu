@@ -86,6 +86,10 @@ struct PfParams {
     const uint8_t *key_role;
     const int32_t *key_seg;
     const int32_t *key_pos;  // S_aug position of each key row; NULL: the row index
+    // per key tile of the retained-first order: the first of the 128 consecutive
+    // rows of K and V the tile is made of (loaded from them directly), or -1 (the
+    // tile is loaded from the permuted copy); NULL in the given order
+    const int32_t *key_direct;
     uint16_t *O;
     float *lse;
     float *nexus_mass;
@@ -490,7 +494,8 @@ __device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8
 template <int D, int kOut>
 __global__ void __maxnreg__(168)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-               const __grid_constant__ CUtensorMap tmV, const PfParams p) {
+               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmK0,
+               const __grid_constant__ CUtensorMap tmV0, const PfParams p) {
     using C = PfCfg<D>;
     constexpr bool kLse = kOut & 1, kMass = kOut & 2;
     extern __shared__ uint8_t smem_raw[];
@@ -747,6 +752,10 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             tma_prefetch_desc(&tmQ);
             tma_prefetch_desc(&tmK);
             tma_prefetch_desc(&tmV);
+            if (p.key_direct != nullptr) {
+                tma_prefetch_desc(&tmK0);
+                tma_prefetch_desc(&tmV0);
+            }
         }
         int g = 0;  // K/V tiles issued over all units (ring position)
         bool ok = true;
@@ -778,12 +787,17 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const int kvh = ui->h0 / p.G;
                 for (int i = 0; i < n_list; ++i, ++g) {
                     const int st = g & 1;
+                    const int e = lst[i];
+                    const int kt = e >> 6;
+                    // a retained-first tile made of 128 consecutive input rows is
+                    // copied from K and V themselves (the load overlaps the wait)
+                    const int dsrc = p.key_direct != nullptr
+                                         ? p.key_direct[(int64_t)b * p.max_k_tiles + kt]
+                                         : -1;
                     if (g >= 2 && !mbar_wait(&kv_empty[st], ((g >> 1) - 1) & 1, p.status, abort_flag)) {
                         ok = false;
                         break;
                     }
-                    const int e = lst[i];
-                    const int kt = e >> 6;
                     // query tiles visiting the key tile that read its metadata: cut
                     // by the mask, or (Nexus mass) some of its keys are Nexus keys
                     const bool mass_tile = kMass && ((e >> 4) & 3) == 2;
@@ -794,12 +808,15 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // tile waits for the copy alone
                     if (lane == 0) {
                         mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
-                        const int row = kkstart + kt * kBN;
+                        const bool direct = dsrc >= 0;
+                        const int row = direct ? dsrc : kkstart + kt * kBN;
+                        const CUtensorMap *mk = direct ? &tmK0 : &tmK;
+                        const CUtensorMap *mv = direct ? &tmV0 : &tmV;
 #pragma unroll
                         for (int hh = 0; hh < C::kHalves; ++hh) {
-                            tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), &tmK, &kv_full[st],
+                            tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), mk, &kv_full[st],
                                         hh * 64, kvh, row, layer);
-                            tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), &tmV, &kv_full[st],
+                            tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), mv, &kv_full[st],
                                         hh * 64, kvh, row, layer);
                         }
                     }
@@ -1315,7 +1332,8 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
                  int32_t *__restrict__ key_start,
                  int32_t *__restrict__ key_len, uint8_t *__restrict__ o_role,
                  int32_t *__restrict__ o_seg, int32_t *__restrict__ o_pos,
-                 int32_t *__restrict__ o_src, int32_t *__restrict__ status) {
+                 int32_t *__restrict__ o_src, int32_t *__restrict__ direct, int max_k_tiles,
+                 int32_t *__restrict__ status) {
     const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int sh[2][32];
     __shared__ long long sh_base;
@@ -1424,6 +1442,28 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     const int first = min(sh_first, len - R);  // body rows before it: unseen
     for (int i = body0 + tid; i < body0 + (first / kBN) * kBN; i += kOrderThreads)
         o_src[start + i] = -2;
+    // A tile whose 128 rows are 128 consecutive rows of the input (a run of one
+    // body, of the system prompt, of the current turn) is read by the attention
+    // kernel from K and V themselves: it is not copied (source -2) and its first
+    // input row is recorded; every other tile records -1 and is copied.
+    __syncthreads();
+    const int n_tiles = span / kBN;
+    for (int t = warp; t < max_k_tiles; t += kOrderThreads / 32) {
+        int d = -1;
+        if (t < n_tiles) {
+            const int64_t r0 = start + (int64_t)t * kBN;
+            const int32_t s0 = o_src[r0];
+            bool run = s0 >= 0;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) run = run && o_src[r0 + w * 32 + lane] == s0 + w * 32 + lane;
+            if (__all_sync(0xffffffffu, run)) {
+                d = s0;
+#pragma unroll
+                for (int w = 0; w < 4; ++w) o_src[r0 + w * 32 + lane] = -2;
+            }
+        }
+        if (lane == 0) direct[(int64_t)b * max_k_tiles + t] = d;
+    }
     if (tid == 0) {
         key_start[b] = (int32_t)start;
         key_len[b] = lp;
@@ -1480,7 +1520,8 @@ kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
 
 template <int D>
 cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
-                           const PfParams &p, int grid, cudaStream_t s) {
+                           const CUtensorMap &tk0, const CUtensorMap &tv0, const PfParams &p,
+                           int grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
     const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
@@ -1491,7 +1532,7 @@ cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const C
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kPfThreads, smem, s>>>(tq, tk, tv, p);
+    kern<<<grid, kPfThreads, smem, s>>>(tq, tk, tv, tk0, tv0, p);
     return cudaGetLastError();
 }
 
@@ -1504,7 +1545,7 @@ int max_k_tiles_of(const sonic_prefill_args *a) {
 // the retained-first order also the permuted key metadata and the permuted K
 // and V of every layer.
 struct PfWorkspace {
-    size_t counter, sums, masks, key_start, key_len, role, seg, pos, src, kp, vp, total;
+    size_t counter, sums, masks, key_start, key_len, role, seg, pos, src, direct, kp, vp, total;
     int64_t rows;  // rows of the permuted K/V per layer
 };
 
@@ -1530,6 +1571,7 @@ PfWorkspace workspace_layout(const sonic_prefill_args *a) {
         w.seg = take((size_t)w.rows * 4);
         w.pos = take((size_t)w.rows * 4);
         w.src = take((size_t)w.rows * 4);
+        w.direct = take(tiles * 4);
         const size_t layer = (size_t)w.rows * a->n_heads_kv * a->head_dim * 2;
         w.kp = take(layer * a->n_layers);
         w.vp = take(layer * a->n_layers);
@@ -1625,10 +1667,21 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, kt_layer};
     const uint32_t box[4] = {64, 1, 128, 1};
     const uint32_t qbox[4] = {64, 1u << pack_log2, (uint32_t)R, 1};  // R rows x P heads
-    CUtensorMap tq, tk, tv;
+    CUtensorMap tq, tk, tv, tk0, tv0;
     if (!make_tmap_bf16_4d(&tq, Q, qd, qs, qbox) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
         !make_tmap_bf16_4d(&tv, Vt, kd, ks, box))
         return SONIC_ERR_INVALID_ARGUMENT;
+    // the inputs themselves, for the retained-first tiles read in place
+    const uint64_t kd0[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_k_rows,
+                             (uint64_t)a->n_layers};
+    const uint64_t ks0[3] = {(uint64_t)D * 2, krow * 2, k_layer};
+    if (reorder) {
+        if (!make_tmap_bf16_4d(&tk0, K, kd0, ks0, box) || !make_tmap_bf16_4d(&tv0, V, kd0, ks0, box))
+            return SONIC_ERR_INVALID_ARGUMENT;
+    } else {
+        tk0 = tk;
+        tv0 = tv;
+    }
 
     PfParams p{};
     p.k_start = a->k_start;
@@ -1642,12 +1695,14 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.key_role = role;
     p.key_seg = seg_id;
     p.key_pos = nullptr;
+    p.key_direct = nullptr;
     if (reorder) {
         p.key_start = reinterpret_cast<const int32_t *>(wsb + ws.key_start);
         p.key_len = reinterpret_cast<const int32_t *>(wsb + ws.key_len);
         p.key_role = wsb + ws.role;
         p.key_seg = reinterpret_cast<const int32_t *>(wsb + ws.seg);
         p.key_pos = reinterpret_cast<const int32_t *>(wsb + ws.pos);
+        p.key_direct = reinterpret_cast<const int32_t *>(wsb + ws.direct);
     }
     p.O = O;
     p.lse = a->lse;
@@ -1681,7 +1736,8 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
             reinterpret_cast<int32_t *>(wsb + ws.key_start),
             reinterpret_cast<int32_t *>(wsb + ws.key_len), wsb + ws.role,
             reinterpret_cast<int32_t *>(wsb + ws.seg), reinterpret_cast<int32_t *>(wsb + ws.pos),
-            reinterpret_cast<int32_t *>(wsb + ws.src), a->status);
+            reinterpret_cast<int32_t *>(wsb + ws.src), reinterpret_cast<int32_t *>(wsb + ws.direct),
+            max_k_tiles_of(a), a->status);
         const int sms = device_sm_count();
         // ~32 blocks per SM in all, as in the compaction copy
         const int per_slice = std::max(1, (sms * 32 + 2 * a->n_layers - 1) / (2 * a->n_layers));
@@ -1698,7 +1754,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status, p.counter);
     // one persistent block per SM (fewer when there are fewer units)
     const int grid = (int)std::min<long long>(device_sm_count(), n_units);
-    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, p, grid, stream)
-                               : launch_prefill<64>(tq, tk, tv, p, grid, stream);
+    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, tk0, tv0, p, grid, stream)
+                               : launch_prefill<64>(tq, tk, tv, tk0, tv0, p, grid, stream);
     return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
 }
