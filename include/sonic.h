@@ -100,7 +100,12 @@ typedef enum {
  * positions.  A 128-key tile of that order made of 128 consecutive rows of
  * K and V (a stretch of one body, of the system prompt or of the current
  * turn) is read from K and V in place; the K and V rows of every other tile
- * are copied into the workspace, for every layer.  Every query row then sees one prefix of the retained part plus
+ * are copied into the workspace, for every layer.  The query rows are walked
+ * in the same order, by 32-row chunks of runs (one body, or consecutive rows
+ * that are not body rows), so a query tile holds rows that see nearly the same
+ * keys; Q and O stay where they are.  A sequence with more than 1024 such
+ * runs, or whose runs padded to 32 rows exceed align128(q_len) + 1024 rows,
+ * keeps the given query order.  Every query row then sees one prefix of the retained part plus
  * (for body and Nexus rows) the body of its own segment, so far fewer key
  * tiles are visited and cut by the mask when all rows of S_aug are queried.
  * Results equal AS_GIVEN up to floating-point summation order.  The copy
@@ -236,7 +241,8 @@ SONIC_API sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *K
  * work units from, then 32 + 256 bytes per 128-key tile (its summary and its
  * column masks), batch * ceil(max_k_len / 128) tiles, each part rounded up to
  * 256 bytes.  RETAINED_FIRST counts one more tile per sequence and adds 4
- * bytes per tile and, for R = min(batch * (align128(max_k_len) + 128),
+ * bytes per tile, batch * (align128(max_q_len) + 1024) / 8 bytes (the query
+ * order's chunk table) and, for R = min(batch * (align128(max_k_len) + 128),
  * total_k_rows + 256 * batch) rows: 13 bytes of metadata per row and a K and
  * a V copy of R rows for every layer (2 * n_layers * R * n_heads_kv *
  * head_dim * 2 bytes).  Sequence b takes align128(k_len[b]) + 128 of the R

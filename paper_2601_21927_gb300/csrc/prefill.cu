@@ -90,6 +90,11 @@ struct PfParams {
     // rows of K and V the tile is made of (loaded from them directly), or -1 (the
     // tile is loaded from the permuted copy); NULL in the given order
     const int32_t *key_direct;
+    // query chunks of the retained-first query order (query_order_kernel): per
+    // sequence qchunks_per_seq words, four per 128-row query tile; NULL: the
+    // query rows in the given order
+    const int32_t *qchunks;
+    int qchunks_per_seq;
     uint16_t *O;
     float *lse;
     float *nexus_mass;
@@ -120,8 +125,10 @@ struct UnitInfo {
     int32_t kstart, klen, kkstart, kklen, qstart, qlen;
     int32_t pbase;    // S_aug position of query row 0 of tile 0
     int32_t last[2];  // list index of the last key tile each query tile visits (-1: none)
+    int32_t qc[2][4];  // chunk words of the query tiles (query chunk table)
+    int32_t pad[8];
 };
-static_assert(sizeof(UnitInfo) == 64, "unit record: 64 bytes");
+static_assert(sizeof(UnitInfo) == 128, "unit record: 128 bytes");
 
 template <int D>
 struct PfCfg {
@@ -491,11 +498,14 @@ __device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8
 // the epilogue has read it (o_free), S/P only after the last P.V read it (the
 // tensor pipe runs in order).
 // kOut: bit 0 writes the log-sum-exp, bit 1 the attention mass on Nexus keys.
-template <int D, int kOut>
+// kQC: the query tiles come from the chunk table of the retained-first query
+// order (query_order_kernel) instead of consecutive query rows.
+template <int D, int kOut, bool kQC>
 __global__ void __maxnreg__(168)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmK0,
-               const __grid_constant__ CUtensorMap tmV0, const PfParams p) {
+               const __grid_constant__ CUtensorMap tmV0, const __grid_constant__ CUtensorMap tmQ32,
+               const PfParams p) {
     using C = PfCfg<D>;
     constexpr bool kLse = kOut & 1, kMass = kOut & 2;
     extern __shared__ uint8_t smem_raw[];
@@ -574,7 +584,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // ------------------------------------------------------------ scheduler
         for (int k = 0;; ++k) {
             const int slot = k & 1;
-            int end = 0, layer = 0, b = 0, hg = 0, qt = 0;
+            int end = 0, layer = 0, b = 0, hg = 0, qt = 0, cw = 0;
             int kstart = 0, klen = 0, qstart = 0, qlen = 0, kkstart = 0, kklen = 0;
             for (;;) {
                 int u = p.n_units;
@@ -604,7 +614,19 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     if (lane == 0 && hg == 0 && qt == 0) set_status(p.status, SONIC_ERR_INVALID_ARGUMENT);
                     continue;
                 }
-                if (qt * urows >= qlen) continue;  // no query rows in this block
+                if constexpr (kQC) {
+                    // lane l < 8: chunk l & 3 of query tile l >> 2 (paired: both
+                    // tiles are the same rows)
+                    cw = 0;
+                    if (lane < 8) {
+                        const int vt = p.pair ? qt : 2 * qt + (lane >> 2);
+                        if ((vt + 1) * 4 <= p.qchunks_per_seq)
+                            cw = p.qchunks[(int64_t)b * p.qchunks_per_seq + vt * 4 + (lane & 3)];
+                    }
+                    if (!__any_sync(0xffffffffu, (cw >> 24) != 0)) continue;  // no query rows
+                } else {
+                    if (qt * urows >= qlen) continue;  // no query rows in this block
+                }
                 kklen = p.key_len[b];
                 if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
                     // the host-side bounds were wrong for this sequence: refuse it
@@ -634,40 +656,91 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 break;
             }
             const int pbase = klen - qlen + qt * urows;  // position of query row 0 of tile 0
-            const bool tile1 = p.pair || qt * 2 * R + R < qlen;
-            // summaries of the query tiles: segment range, Nexus rows and their
-            // segment range
-            int qf[2], qs0[2], qs1[2], qn0[2], qn1[2];
+            // summaries of the query tiles: S_aug position range (smallest and
+            // largest), segment range, Nexus rows and their segment range
+            int qf[2], qs0[2], qs1[2], qn0[2], qn1[2], qp0[2], qp1[2];
+            bool tile1;
+            if constexpr (kQC) {
+                // Chunk words (lane l < 8: chunk l & 3 of tile l >> 2) turned into
+                // (query rows << 24) | S_aug position of the chunk's first row;
+                // tile row r is row r & 31 of chunk r >> 5.
+                cw = (cw & ~0xffffff) | (klen - qlen + (cw & 0xffffff));
 #pragma unroll
-            for (int qi = 0; qi < 2; ++qi) {
-                int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
-                for (int r = lane; r < R; r += 32) {
-                    const int pos = pbase + qi * qstep + r;
-                    if (pos <= klen - 1) {
-                        const int ro = p.role[kstart + pos];
-                        const int s = p.seg[kstart + pos];
-                        s0 = min(s0, s);
-                        s1 = max(s1, s);
-                        if (ro == SONIC_ROLE_NEXUS) {
-                            f = 2;
-                            n0 = min(n0, s);
-                            n1 = max(n1, s);
+                for (int qi = 0; qi < 2; ++qi) {
+                    int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
+                    int pmin = INT_MAX, pmax = INT_MIN;
+#pragma unroll
+                    for (int c = 0; c < kBM / 32; ++c) {
+                        const int w = __shfl_sync(0xffffffffu, cw, qi * 4 + c);
+                        const int pos = (w & 0xffffff) + lane;
+                        if (lane < (w >> 24)) {
+                            const int ro = p.role[kstart + pos];
+                            const int s = p.seg[kstart + pos];
+                            pmin = min(pmin, pos);
+                            pmax = max(pmax, pos);
+                            s0 = min(s0, s);
+                            s1 = max(s1, s);
+                            if (ro == SONIC_ROLE_NEXUS) {
+                                f = 2;
+                                n0 = min(n0, s);
+                                n1 = max(n1, s);
+                            }
                         }
                     }
-                }
 #pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    f |= __shfl_xor_sync(0xffffffffu, f, o);
-                    s0 = min(s0, __shfl_xor_sync(0xffffffffu, s0, o));
-                    s1 = max(s1, __shfl_xor_sync(0xffffffffu, s1, o));
-                    n0 = min(n0, __shfl_xor_sync(0xffffffffu, n0, o));
-                    n1 = max(n1, __shfl_xor_sync(0xffffffffu, n1, o));
+                    for (int o = 16; o > 0; o >>= 1) {
+                        f |= __shfl_xor_sync(0xffffffffu, f, o);
+                        s0 = min(s0, __shfl_xor_sync(0xffffffffu, s0, o));
+                        s1 = max(s1, __shfl_xor_sync(0xffffffffu, s1, o));
+                        n0 = min(n0, __shfl_xor_sync(0xffffffffu, n0, o));
+                        n1 = max(n1, __shfl_xor_sync(0xffffffffu, n1, o));
+                        pmin = min(pmin, __shfl_xor_sync(0xffffffffu, pmin, o));
+                        pmax = max(pmax, __shfl_xor_sync(0xffffffffu, pmax, o));
+                    }
+                    qf[qi] = f;
+                    qs0[qi] = s0;
+                    qs1[qi] = s1;
+                    qn0[qi] = n0;
+                    qn1[qi] = n1;
+                    qp0[qi] = pmin;
+                    qp1[qi] = pmax;
                 }
-                qf[qi] = f;
-                qs0[qi] = s0;
-                qs1[qi] = s1;
-                qn0[qi] = n0;
-                qn1[qi] = n1;
+                tile1 = p.pair || qp0[1] <= qp1[1];
+            } else {
+                tile1 = p.pair || qt * 2 * R + R < qlen;
+#pragma unroll
+                for (int qi = 0; qi < 2; ++qi) {
+                    int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
+                    for (int r = lane; r < R; r += 32) {
+                        const int pos = pbase + qi * qstep + r;
+                        if (pos <= klen - 1) {
+                            const int ro = p.role[kstart + pos];
+                            const int s = p.seg[kstart + pos];
+                            s0 = min(s0, s);
+                            s1 = max(s1, s);
+                            if (ro == SONIC_ROLE_NEXUS) {
+                                f = 2;
+                                n0 = min(n0, s);
+                                n1 = max(n1, s);
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) {
+                        f |= __shfl_xor_sync(0xffffffffu, f, o);
+                        s0 = min(s0, __shfl_xor_sync(0xffffffffu, s0, o));
+                        s1 = max(s1, __shfl_xor_sync(0xffffffffu, s1, o));
+                        n0 = min(n0, __shfl_xor_sync(0xffffffffu, n0, o));
+                        n1 = max(n1, __shfl_xor_sync(0xffffffffu, n1, o));
+                    }
+                    qf[qi] = f;
+                    qs0[qi] = s0;
+                    qs1[qi] = s1;
+                    qn0[qi] = n0;
+                    qn1[qi] = n1;
+                    qp0[qi] = pbase + qi * qstep;
+                    qp1[qi] = min(qp0[qi] + R - 1, klen - 1);
+                }
             }
             // Key tiles to visit: a key tile is listed when either query tile
             // sees some of it.  entry: (tile << 6) | (Nexus keys: 0 none, 1 all,
@@ -687,8 +760,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     entry = (t << 6) | ((kn ? ((kb || ko) ? 2 : 1) : 0) << 4);
 #pragma unroll
                     for (int qi = 0; qi < 2; ++qi) {
-                        const int p0 = pbase + qi * qstep;
-                        const int p1 = min(p0 + R - 1, klen - 1);
+                        // S_aug positions of the query tile's rows: smallest, largest
+                        const int p0 = qp0[qi], p1 = qp1[qi];
                         if (p0 > p1) continue;
                         const bool q_has_nexus = qf[qi] & 2;
                         const bool causal_part = (k0 <= p1) && (kn || ko);
@@ -742,6 +815,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 ui->last[0] = last0;
                 ui->last[1] = last1;
             }
+            if (kQC && lane < 8) ui->qc[lane >> 2][lane & 3] = cw;
             // every lane's list entries are written before lane 0 publishes the slot
             __syncwarp();
             if (lane == 0) mbar_arrive(&unit_full[slot]);
@@ -756,6 +830,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 tma_prefetch_desc(&tmK0);
                 tma_prefetch_desc(&tmV0);
             }
+            if (p.qchunks != nullptr) tma_prefetch_desc(&tmQ32);
         }
         int g = 0;  // K/V tiles issued over all units (ring position)
         bool ok = true;
@@ -773,7 +848,50 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 if (issued_q > 0 &&
                     !mbar_wait(q_empty, (issued_q - 1) & 1, p.status, abort_flag))
                     break;
-                if (lane == 0) {
+                if (kQC && lane == 0) {
+                    // a query tile of 128 consecutive query rows in one copy, any
+                    // other from its 32-row chunks (a chunk without rows is not
+                    // loaded: its tile rows are computed and never written)
+                    const int q0 = ui->qstart - (ui->klen - ui->qlen);  // Q row of position 0
+                    int bytes = 0;
+                    bool whole[2] = {false, false};
+#pragma unroll
+                    for (int qi = 0; qi < 2; ++qi) {
+                        if (qi >= nq) break;
+                        const int w0 = ui->qc[qi][0];
+                        whole[qi] = true;
+#pragma unroll
+                        for (int c = 0; c < kBM / 32; ++c) {
+                            const int w = ui->qc[qi][c];
+                            whole[qi] = whole[qi] && w == w0 + c * 32;
+                            if ((w >> 24) != 0) bytes += 32 * D * 2;
+                        }
+                        whole[qi] = whole[qi] && (w0 >> 24) == 32;
+                    }
+                    mbar_arrive_expect_tx(q_full, bytes);
+#pragma unroll
+                    for (int qi = 0; qi < 2; ++qi) {
+                        if (qi >= nq) break;
+                        if (whole[qi]) {
+#pragma unroll
+                            for (int hh = 0; hh < C::kHalves; ++hh)
+                                tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
+                                            hh * 64, ui->h0 + qi * p.pair,
+                                            q0 + (ui->qc[qi][0] & 0xffffff), layer);
+                            continue;
+                        }
+#pragma unroll
+                        for (int c = 0; c < kBM / 32; ++c) {
+                            const int w = ui->qc[qi][c];
+                            if ((w >> 24) == 0) continue;
+#pragma unroll
+                            for (int hh = 0; hh < C::kHalves; ++hh)
+                                tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128) + c * (32 * 128),
+                                            &tmQ32, q_full, hh * 64, ui->h0 + qi * p.pair,
+                                            q0 + (w & 0xffffff), layer);
+                        }
+                    }
+                } else if (!kQC && lane == 0) {
                     mbar_arrive_expect_tx(q_full, nq * C::kQBytes);
                     for (int qi = 0; qi < nq; ++qi)
 #pragma unroll
@@ -1043,9 +1161,18 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 const bool udense = ui->flags & 2;
                 const int last = udense ? n_list - 1 : ui->last[qi];
                 const int kklen = ui->kklen;
-                const int pos = ui->pbase + qi * qstep + qr;
+                // S_aug position of this thread's query row (-1: the tile row holds
+                // no query row of the unit, and sees no key)
+                int pos;
+                if constexpr (kQC) {
+                    // -1: the tile row holds no query row (it sees no key)
+                    const int w = ui->qc[qi][r >> 5];
+                    pos = lane < (w >> 24) ? (w & 0xffffff) + lane : -1;
+                } else {
+                    pos = ui->pbase + qi * qstep + qr;
+                }
                 int rp = SONIC_ROLE_SYS, sp = 0;
-                if (pos <= ui->klen - 1) {
+                if (kQC ? pos >= 0 : pos <= ui->klen - 1) {
                     rp = p.role[ui->kstart + pos];
                     sp = p.seg[ui->kstart + pos];
                 }
@@ -1237,8 +1364,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
                 if (!ok) break;
                 const int layer = ui->layer, h = ui->h0 + qi * p.pair + hoff;
-                const int qidx = ui->qt * urows + qi * qstep + qr;  // query row within the sequence
-                const bool row_ok = pos <= ui->klen - 1 && qidx < ui->qlen;
+                // query row within the sequence
+                const int qidx = kQC ? pos - (ui->klen - ui->qlen) : ui->qt * urows + qi * qstep + qr;
+                const bool row_ok = kQC ? pos >= 0 : pos <= ui->klen - 1 && qidx < ui->qlen;
                 const int64_t qrow = (int64_t)ui->qstart + qidx;
                 uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
                 const int64_t sidx = ((int64_t)layer * p.total_q_rows + qrow) * p.Hq + h;
@@ -1470,6 +1598,133 @@ key_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ s
     }
 }
 
+// ---------------------------------------------------------------- query order
+// Retained-first query order.  A sequence's query rows (its last q_len rows)
+// are walked as [body rows | every other row], each part in S_aug order and
+// cut into runs: consecutive rows of one body, or consecutive rows that are
+// not body rows.  Each run starts on a 32-row boundary and the second part on
+// a 128-row boundary, so a 128-row query tile is four 32-row chunks, each
+// chunk a stretch of at most 32 consecutive query rows of one run, and the
+// rows of one body fill whole tiles of their own (the rows a body row sees are
+// the same for its whole segment; in the given order a tile straddles two
+// segments and the Nexus rows between them).  The chunk table holds, per
+// sequence, chunks_per_seq words: (rows << 24) | first query row, 0 for a
+// chunk without rows.  A sequence with more than kQRunsMax runs, or whose runs
+// need more than align128(q_len) + kQSlack rows, keeps the given order (chunks
+// of 32 consecutive query rows).
+constexpr int kQOrderThreads = 1024;
+constexpr int kQRunsMax = 1024;
+constexpr int kQSlack = 1024;
+
+// Exclusive prefix sum over the block (kQOrderThreads threads) and the total.
+__device__ __forceinline__ int block_excl_scan(int v, int *sh, int &total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = sh[lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        sh[lane] = w;
+    }
+    __syncthreads();
+    total = sh[31];
+    const int r = x - v + (warp > 0 ? sh[warp - 1] : 0);
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kQOrderThreads)
+query_order_kernel(const uint8_t *__restrict__ role, const int32_t *__restrict__ seg,
+                   const int32_t *__restrict__ k_start, const int32_t *__restrict__ k_len,
+                   const int32_t *__restrict__ q_len, int max_k_len, int64_t total_rows,
+                   int chunks_per_seq, int32_t *__restrict__ qchunks) {
+    const int b = blockIdx.x, tid = threadIdx.x;
+    __shared__ int sh[32];
+    __shared__ int rs[kQRunsMax + 1];   // first query row of each run
+    __shared__ int vs[kQRunsMax + 1];   // runs sorted by their place: first chunk row
+    __shared__ int ss[kQRunsMax];       // ... first query row
+    __shared__ int ls[kQRunsMax];       // ... rows
+    const int ks = k_start[b];
+    const int len = seq_rows(ks, k_len[b], max_k_len, total_rows);
+    // a sequence the attention kernel refuses gets the given order; nothing
+    // of it is read here beyond its rows
+    const int ql = min(max(q_len[b], 0), len);
+    const int q0 = ks + len - ql;  // row of query 0
+    int32_t *out = qchunks + (int64_t)b * chunks_per_seq;
+    // runs: their first rows in order
+    int nr = 0;
+    for (int c0 = 0; c0 < ql; c0 += kQOrderThreads) {
+        const int i = c0 + tid;
+        bool start = false;
+        if (i < ql) {
+            const bool body = role[q0 + i] == SONIC_ROLE_BODY;
+            if (i == 0) {
+                start = true;
+            } else {
+                const bool pbody = role[q0 + i - 1] == SONIC_ROLE_BODY;
+                start = body != pbody || (body && seg[q0 + i] != seg[q0 + i - 1]);
+            }
+        }
+        int total;
+        const int at = block_excl_scan(start ? 1 : 0, sh, total);
+        if (start && nr + at < kQRunsMax) rs[nr + at] = i;
+        nr += total;
+    }
+    const bool many = nr > kQRunsMax;
+    if (tid == 0 && !many) rs[nr] = ql;
+    __syncthreads();
+    // each run's place: body runs first, in order, then the other runs
+    int rows = 0, isb = 0;
+    if (!many && tid < nr) {
+        rows = rs[tid + 1] - rs[tid];
+        isb = role[q0 + rs[tid]] == SONIC_ROLE_BODY;
+    }
+    const int a32 = (rows + 31) & ~31;
+    int tb, tn, nb_runs, n_other;
+    const int eb = block_excl_scan(isb ? a32 : 0, sh, tb);
+    const int en = block_excl_scan(isb ? 0 : a32, sh, tn);
+    const int rb = block_excl_scan(isb ? 1 : 0, sh, nb_runs);
+    const int ro = block_excl_scan((!many && tid < nr && !isb) ? 1 : 0, sh, n_other);
+    const int other0 = (tb + 127) & ~127;
+    const int span = other0 + tn;
+    const bool given = many || span > ((ql + 127) & ~127) + kQSlack;
+    if (!given && tid < nr) {
+        const int k = isb ? rb : nb_runs + ro;
+        vs[k] = isb ? eb : other0 + en;
+        ss[k] = rs[tid];
+        ls[k] = rows;
+    }
+    if (tid == 0 && !given) vs[nr] = INT_MAX;
+    __syncthreads();
+    for (int c = tid; c < chunks_per_seq; c += kQOrderThreads) {
+        int w = 0;
+        const int v = c * 32;
+        if (given) {
+            if (v < ql) w = (min(32, ql - v) << 24) | v;
+        } else if (v < span) {
+            // the last run placed at or before row v
+            int lo = 0, hi = nr - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (vs[mid] <= v) lo = mid; else hi = mid - 1;
+            }
+            const int off = v - vs[lo];
+            if (off >= 0 && off < ls[lo]) w = (min(32, ls[lo] - off) << 24) | (ss[lo] + off);
+        }
+        out[c] = w;
+    }
+}
+
 // K and V rows of every layer into the retained-first order (warp per row;
 // rows with source -1 are zeroed).
 constexpr int kPermThreads = 256;
@@ -1520,20 +1775,31 @@ kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
 
 template <int D>
 cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
-                           const CUtensorMap &tk0, const CUtensorMap &tv0, const PfParams &p,
-                           int grid, cudaStream_t s) {
+                           const CUtensorMap &tk0, const CUtensorMap &tv0, const CUtensorMap &tq32,
+                           const PfParams &p, int grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
     const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
-    auto kern = out == 0   ? prefill_kernel<D, 0>
-                : out == 1 ? prefill_kernel<D, 1>
-                : out == 2 ? prefill_kernel<D, 2>
-                           : prefill_kernel<D, 3>;
+    auto kern = p.qchunks != nullptr
+                    ? (out == 0   ? prefill_kernel<D, 0, true>
+                       : out == 1 ? prefill_kernel<D, 1, true>
+                       : out == 2 ? prefill_kernel<D, 2, true>
+                                  : prefill_kernel<D, 3, true>)
+                    : (out == 0   ? prefill_kernel<D, 0, false>
+                       : out == 1 ? prefill_kernel<D, 1, false>
+                       : out == 2 ? prefill_kernel<D, 2, false>
+                                  : prefill_kernel<D, 3, false>);
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kPfThreads, smem, s>>>(tq, tk, tv, tk0, tv0, p);
+    kern<<<grid, kPfThreads, smem, s>>>(tq, tk, tv, tk0, tv0, tq32, p);
     return cudaGetLastError();
+}
+
+// Chunk words per sequence of the retained-first query order: room for
+// align128(max_q_len) + kQSlack query-tile rows.
+int query_chunks_of(const sonic_prefill_args *a) {
+    return ((a->max_q_len + kBM - 1) / kBM * kBM + kQSlack) / 32;
 }
 
 int max_k_tiles_of(const sonic_prefill_args *a) {
@@ -1545,7 +1811,8 @@ int max_k_tiles_of(const sonic_prefill_args *a) {
 // the retained-first order also the permuted key metadata and the permuted K
 // and V of every layer.
 struct PfWorkspace {
-    size_t counter, sums, masks, key_start, key_len, role, seg, pos, src, direct, kp, vp, total;
+    size_t counter, sums, masks, key_start, key_len, role, seg, pos, src, direct, qchunks, kp, vp,
+        total;
     int64_t rows;  // rows of the permuted K/V per layer
 };
 
@@ -1572,6 +1839,7 @@ PfWorkspace workspace_layout(const sonic_prefill_args *a) {
         w.pos = take((size_t)w.rows * 4);
         w.src = take((size_t)w.rows * 4);
         w.direct = take(tiles * 4);
+        w.qchunks = take((size_t)a->batch * query_chunks_of(a) * 4);
         const size_t layer = (size_t)w.rows * a->n_heads_kv * a->head_dim * 2;
         w.kp = take(layer * a->n_layers);
         w.vp = take(layer * a->n_layers);
@@ -1642,7 +1910,11 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     // then see the same keys (no key tile visited by one tile alone).
     const bool pair = pack_log2 == 0 && G % 2 == 0;
     const long long urows = pair ? R : 2 * R;
-    const long long qtiles = (a->max_q_len + urows - 1) / urows;
+    // retained-first keys with unpacked heads: the query rows are walked in
+    // the retained-first order too, as 32-row chunks (query_order_kernel)
+    const bool qchunked = reorder && pack_log2 == 0;
+    const long long qrows_v = qchunked ? (long long)query_chunks_of(a) * 32 : a->max_q_len;
+    const long long qtiles = (qrows_v + urows - 1) / urows;
     const long long HG = pair ? a->n_heads_q / 2 : a->n_heads_q >> pack_log2;
     const long long n_units = qtiles * HG * a->batch * a->n_layers;
     if (n_units > 0x7fffffff) return SONIC_ERR_UNSUPPORTED;
@@ -1667,7 +1939,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, kt_layer};
     const uint32_t box[4] = {64, 1, 128, 1};
     const uint32_t qbox[4] = {64, 1u << pack_log2, (uint32_t)R, 1};  // R rows x P heads
-    CUtensorMap tq, tk, tv, tk0, tv0;
+    CUtensorMap tq, tk, tv, tk0, tv0, tq32;
     if (!make_tmap_bf16_4d(&tq, Q, qd, qs, qbox) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
         !make_tmap_bf16_4d(&tv, Vt, kd, ks, box))
         return SONIC_ERR_INVALID_ARGUMENT;
@@ -1681,6 +1953,12 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     } else {
         tk0 = tk;
         tv0 = tv;
+    }
+    const uint32_t qbox32[4] = {64, 1, 32, 1};  // one 32-row query chunk of one head
+    if (qchunked) {
+        if (!make_tmap_bf16_4d(&tq32, Q, qd, qs, qbox32)) return SONIC_ERR_INVALID_ARGUMENT;
+    } else {
+        tq32 = tq;
     }
 
     PfParams p{};
@@ -1696,6 +1974,12 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     p.key_seg = seg_id;
     p.key_pos = nullptr;
     p.key_direct = nullptr;
+    p.qchunks = nullptr;
+    p.qchunks_per_seq = 0;
+    if (qchunked) {
+        p.qchunks = reinterpret_cast<const int32_t *>(wsb + ws.qchunks);
+        p.qchunks_per_seq = query_chunks_of(a);
+    }
     if (reorder) {
         p.key_start = reinterpret_cast<const int32_t *>(wsb + ws.key_start);
         p.key_len = reinterpret_cast<const int32_t *>(wsb + ws.key_len);
@@ -1747,6 +2031,10 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
             reinterpret_cast<const int32_t *>(wsb + ws.key_start), a->batch, (int64_t)krow * 2,
             (int64_t)k_layer, (int64_t)kt_layer);
     }
+    if (qchunked)
+        query_order_kernel<<<a->batch, kQOrderThreads, 0, stream>>>(
+            role, seg_id, a->k_start, a->k_len, a->q_len, a->max_k_len, a->total_k_rows,
+            p.qchunks_per_seq, reinterpret_cast<int32_t *>(wsb + ws.qchunks));
     tile_summary_kernel<<<dim3(p.max_k_tiles, a->batch), 128, 0, stream>>>(
         p.key_role, p.key_seg, p.key_pos, p.key_start, p.key_len,
         reinterpret_cast<TileSum *>(wsb + ws.sums), reinterpret_cast<TileMasks *>(wsb + ws.masks),
@@ -1754,7 +2042,7 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status, p.counter);
     // one persistent block per SM (fewer when there are fewer units)
     const int grid = (int)std::min<long long>(device_sm_count(), n_units);
-    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, tk0, tv0, p, grid, stream)
-                               : launch_prefill<64>(tq, tk, tv, tk0, tv0, p, grid, stream);
+    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, tk0, tv0, tq32, p, grid, stream)
+                               : launch_prefill<64>(tq, tk, tv, tk0, tv0, tq32, p, grid, stream);
     return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
 }

@@ -119,8 +119,9 @@ def test_retained_first_workspace_size():
     """Workspace of the retained-first order: the work-unit counter (256 B),
     tile summaries (32 B) and column masks (256 B) of one extra tile per
     sequence, 13 bytes of metadata per permuted row, the first input row of
-    each tile read in place (4 B per tile), and a K and a V copy of every
-    layer; each part rounded up to 256 bytes."""
+    each tile read in place (4 B per tile), the query chunk table (4 B per
+    32 rows of align128(max_q_len) + 1024 rows per sequence), and a K and a V
+    copy of every layer; each part rounded up to 256 bytes."""
     lib = sonic.load()
     p = sonic.sonic_prefill_args()
     p.batch, p.n_layers, p.n_heads_q, p.n_heads_kv, p.head_dim = 2, 3, 8, 4, 128
@@ -133,7 +134,7 @@ def test_retained_first_workspace_size():
 
     def expect(rows):
         return (256 + r256(2 * 4 * 32) + r256(2 * 4 * 256) + r256(3 * 4) + r256(2 * 4) + r256(rows)
-                + 3 * r256(4 * rows) + r256(2 * 4 * 4)
+                + 3 * r256(4 * rows) + r256(2 * 4 * 4) + r256(2 * (384 + 1024) // 32 * 4)
                 + 2 * r256(3 * rows * 4 * 128 * 2))
 
     # spans of 384 + 128 rows per sequence, below total_k_rows + 256 per sequence

@@ -79,6 +79,15 @@ def test_retained_first_many_runs_per_tile(mode):
     _all_rows(inputs.Batch(ds), 4, 1, 128, mode=mode, seed=13, order=sonic.KEYS_RETAINED_FIRST)
 
 
+def test_retained_first_query_runs_beyond_the_table():
+    """Retained-first walks the query rows by runs (one body, or consecutive
+    other rows) in 32-row chunks; 520 one-token segments make 1,040 runs,
+    more than the run table holds, so that sequence keeps the given query
+    order, beside a sequence whose runs fit (chunked order)."""
+    ds = [inputs.Dialogue(4, [(1, 1)] * 520, 8), inputs.Dialogue(40, [(200, 40)] * 3, 90)]
+    _all_rows(inputs.Batch(ds), 4, 2, 128, seed=15, order=sonic.KEYS_RETAINED_FIRST)
+
+
 @pytest.mark.parametrize("order", ORDERS)
 def test_first_key_tile_not_listed_first(order):
     """No system prompt and a 300-token first body: as given, key tile 0 holds
