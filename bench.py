@@ -1074,29 +1074,36 @@ def config_workloads():
         "ms": round(ms, 4), "gb": round(by / 1e9, 3), "value": round(gbs, 1), "unit": "GB/s",
         "roofline": hbm(gbs)}
 
-    # masked prefill: 8 x 5632 rows, every row a query, full mask, one layer;
-    # then the current turn's rows alone; then compaction of all 32 layers
+    # masked prefill: 8 x 5632 rows, every row a query, full mask, all 32 layers
+    # in one launch (and one layer alone); then the current turn's rows alone;
+    # then compaction of all 32 layers
     batch, hd = inputs.masked_prefill()
     d = batch.dialogues[0]
     role, seg = d.arrays()
     L = d.length
-    K = inputs.randn((1, batch.total, hd.hkv, hd.d), seed=1, device=dev)
-    V = inputs.randn((1, batch.total, hd.hkv, hd.d), seed=2, device=dev)
-    Q = inputs.randn((1, batch.total, hd.hq, hd.d), seed=3, device=dev)
+    NL = hd.n_layers
+    K = inputs.randn((NL, batch.total, hd.hkv, hd.d), seed=1, device=dev)
+    V = inputs.randn((NL, batch.total, hd.hkv, hd.d), seed=2, device=dev)
+    Q = inputs.randn((NL, batch.total, hd.hq, hd.d), seed=3, device=dev)
     O = torch.empty_like(Q)
     r_, s_, ks, kl = t(batch.role), t(batch.seg), t(batch.k_start), t(batch.k_len)
-    flops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L), 0) * batch.B
+    flops1 = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L), 0) * batch.B
     res = {}
-    for order, oname in ((1, "retained_first"), (0, "as_given")):
-        ws = sonic.sonic_attn_prefill(Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks,
-                                      q_len=kl, max_q_len=L, max_k_len=L, key_order=order)
-        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
-            Q, K, V, s_, r_, O, k_start=ks, k_len=kl, q_start=ks, q_len=kl, max_q_len=L,
-            max_k_len=L, key_order=order, workspace=ws), reps=10, warm=3)
-        tf = flops / ms / 1e9
-        res[f"all_rows_{oname}"] = {"ms": round(ms, 4), "value": round(tf, 1), "unit": "TFLOP/s",
-                                    "frac": round(tf / pk["bf16"], 4)}
+
+    def timed(name, Qx, Ox, nl, fl, order, q_start, q_len, max_q):
+        call = lambda ws=None: sonic.sonic_attn_prefill(
+            Qx[:nl], K[:nl], V[:nl], s_, r_, Ox[:nl], k_start=ks, k_len=kl, q_start=q_start,
+            q_len=q_len, max_q_len=max_q, max_k_len=L, key_order=order, workspace=ws)
+        ws = call()
+        ms = _ev_time(lambda: call(ws), reps=10 if nl == 1 else 4, warm=3)
+        tf = fl * nl / ms / 1e9
+        res[name] = {"layers": nl, "ms": round(ms, 4), "value": round(tf, 1), "unit": "TFLOP/s",
+                     "frac": round(tf / pk["bf16"], 4)}
         del ws
+
+    for order, oname in ((1, "retained_first"), (0, "as_given")):
+        timed(f"all_rows_{oname}", Q, O, NL, flops1, order, ks, kl, L)
+    timed("all_rows_retained_first_one_layer", Q, O, 1, flops1, 1, ks, kl, L)
     ql = np.full(batch.B, d.curr_len, np.int32)
     qs = np.concatenate([[0], np.cumsum(ql)[:-1]]).astype(np.int32)
     Qc = Q[:, :int(ql.sum())]
@@ -1104,25 +1111,15 @@ def config_workloads():
     cflops = 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L - d.curr_len, L), 0) * batch.B
     qst, qlt = t(qs), t(ql)
     for order, oname in ((1, "retained_first"), (0, "as_given")):
-        ws = sonic.sonic_attn_prefill(Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=qst,
-                                      q_len=qlt, max_q_len=int(ql.max()), max_k_len=L,
-                                      key_order=order)
-        ms = _ev_time(lambda: sonic.sonic_attn_prefill(
-            Qc, K, V, s_, r_, Oc, k_start=ks, k_len=kl, q_start=qst, q_len=qlt,
-            max_q_len=int(ql.max()), max_k_len=L, key_order=order, workspace=ws),
-            reps=10, warm=3)
-        tf = cflops / ms / 1e9
-        res[f"current_rows_{oname}"] = {"ms": round(ms, 4), "value": round(tf, 1),
-                                        "unit": "TFLOP/s", "frac": round(tf / pk["bf16"], 4)}
-        del ws
+        timed(f"current_rows_{oname}", Qc, Oc, NL, cflops, order, qst, qlt, int(ql.max()))
     del K, V, Q, O, Qc, Oc
     _free_cuda()
     head = res["all_rows_retained_first"]
     prefill = {"workload": "masked prefill, batch 8 x 5632 rows (512 system, 16 x (256 body + 32 "
                            "Nexus), 512 current), every row a query, full Sec. 3.2 mask, 32/8 "
-                           "heads, D=128, bf16, 1 layer; key order retained-first (its K/V "
-                           "permutation included)",
-               "flops": flops, "value": head["value"], "unit": "TFLOP/s",
+                           "heads, D=128, bf16, 32 layers in one launch; retained-first order "
+                           "(its key and query order and K/V copies included)",
+               "flops": flops1 * NL, "ms": head["ms"], "value": head["value"], "unit": "TFLOP/s",
                "roofline": {"bound": "tensor", "peak": pk["bf16"], "unit": "TFLOP/s",
                             "frac": head["frac"], "peak_source": pk["source"] + " bf16 burst"},
                "variants": res}
