@@ -79,6 +79,19 @@ def test_retained_first_many_runs_per_tile(mode):
     _all_rows(inputs.Batch(ds), 4, 1, 128, mode=mode, seed=13, order=sonic.KEYS_RETAINED_FIRST)
 
 
+@pytest.mark.parametrize("hq,hkv", [(8, 1), (12, 2), (4, 1)])
+@pytest.mark.parametrize("mode", [sonic.NEXUS_FULL, sonic.NEXUS_CAUSAL_SEGMENTS])
+def test_retained_first_query_runs(mode, hq, hkv):
+    """Retained-first query order by runs in 32-row chunks, at head ratios 8,
+    6 and 4: Nexus runs shorter and longer than a chunk, empty runs (K_i = 0),
+    adjacent Nexus runs of two segments (an empty body between them), bodies
+    that are not multiples of 32 rows (padded chunks) and one-token runs."""
+    ds = [inputs.Dialogue(40, [(100, 7), (0, 40), (130, 70), (60, 0), (20, 33)], 50),
+          inputs.Dialogue(0, [(256, 32)] * 5, 64),
+          inputs.Dialogue(9, [(3, 1)] * 6 + [(200, 100)], 1)]
+    _all_rows(inputs.Batch(ds), hq, hkv, 128, mode=mode, seed=25, order=sonic.KEYS_RETAINED_FIRST)
+
+
 def test_retained_first_query_runs_beyond_the_table():
     """Retained-first walks the query rows by runs (one body, or consecutive
     other rows) in 32-row chunks; 520 one-token segments make 1,040 runs,
