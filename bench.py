@@ -785,7 +785,7 @@ def extra_nexus_gen():
     B, NL = batch.B, hd.n_layers
     sysl, segs = d.sys_len, d.segments
     steps = []
-    flops = comp_bytes = 0.0
+    flops = comp_bytes = pf_bytes = 0.0
     for i, (nb, nk) in enumerate(segs, start=1):
         r_len = sysl + sum(k for _, k in segs[:i - 1])
         L = r_len + nb + nk
@@ -810,6 +810,9 @@ def extra_nexus_gen():
                           role=t(np.tile(role, B)), seg=t(np.tile(seg, B)), oK=oK, oV=oV, off=off))
         flops += 4.0 * hd.d * hd.hq * _visible_pairs(role, seg, range(L - nk, L), 0) * B * NL
         comp_bytes += 2.0 * R * B * hd.hkv * hd.d * 2 * 2 * NL
+        # the prefill's bytes: every key row is visible to the Nexus rows, so K and
+        # V of all L rows are read once per KV head, Q read and O written once
+        pf_bytes += (2.0 * L * hd.hkv + 2.0 * nk * hd.hq) * B * hd.d * 2 * NL
 
     def prefills():
         for s in steps:
@@ -826,10 +829,22 @@ def extra_nexus_gen():
 
     p_ms = _ev_time(prefills)
     c_ms = _ev_time(compactions)
+    pk = _peaks()
+    # 32 query rows of 4 heads per K/V row: the prefill is bound by HBM, not by
+    # the tensor cores (flops per byte below the ridge point peak_bf16 / peak_hbm)
+    intensity = flops / pf_bytes
     return {"workload": "Nexus generation: batch 8, 32 layers, 32/8 heads, D=128, "
                         "16 segments of 256 body + 32 Nexus after 512 system tokens",
             "results": {"prefill_ms_all_segments": round(p_ms, 3),
                         "prefill_tflops": round(flops / p_ms / 1e9, 1),
+                        "prefill_frac_of_bf16_peak": round(flops / p_ms / 1e9 / pk["bf16"], 4),
+                        "prefill_gb": round(pf_bytes / 1e9, 3),
+                        "prefill_gbs": round(pf_bytes / p_ms / 1e6, 1),
+                        "prefill_flops_per_byte": round(intensity, 1),
+                        "prefill_roofline": {
+                            "bound": "hbm", "peak": pk["hbm"], "unit": "GB/s",
+                            "frac": round(pf_bytes / p_ms / 1e6 / pk["hbm"], 4),
+                            "tflops_at_peak_hbm": round(intensity * pk["hbm"] / 1e3, 1)},
                         "compaction_ms_all_segments": round(c_ms, 3),
                         "compaction_gbs": round(comp_bytes / c_ms / 1e6, 1),
                         "ms_per_segment": round((p_ms + c_ms) / len(segs), 3)}}
