@@ -145,7 +145,7 @@ struct PfCfg {
     static constexpr int kOffList = kOffPos + 2 * kBN * 4;    // [2 units][kMaxKTiles] int32
     static constexpr int kOffUnit = kOffList + 2 * kMaxKTiles * 4;  // [2] UnitInfo
     static constexpr int kOffBar = kOffUnit + 2 * (int)sizeof(UnitInfo);
-    static constexpr int kNumBars = 24;
+    static constexpr int kNumBars = 30;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;   // 16 ints
     static constexpr int kBytes = kOffMisc + 16 * 4;
     static constexpr size_t kSmem = 1024 + kBytes;
@@ -500,7 +500,11 @@ __device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8
 // kOut: bit 0 writes the log-sum-exp, bit 1 the attention mass on Nexus keys.
 // kQC: the query tiles come from the chunk table of the retained-first query
 // order (query_order_kernel) instead of consecutive query rows.
-template <int D, int kOut, bool kQC>
+// kSolo: every unit has one query tile (packed heads, short query blocks).  Its
+// S/P then alternates between the two tiles' TMEM blocks, so the S product of
+// key tile j + 1 runs while the softmax works on tile j, and K takes a ring of
+// three stages (the unused second Q tile's buffer is the third), V of two.
+template <int D, int kOut, bool kQC, bool kSolo>
 __global__ void __maxnreg__(168)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmK0,
@@ -538,6 +542,10 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     uint64_t *unit_full = bars + 18;  // [2] per unit slot
     uint64_t *unit_empty = bars + 20; // [2]
     uint64_t *mma_idle = bars + 22;
+    // kSolo only: K ring stages (written / free again), and one P.V product done
+    uint64_t *k_full = bars + 23;   // [3]
+    uint64_t *k_empty = bars + 26;  // [3]
+    uint64_t *pv_done = bars + 29;
     int32_t *misc = reinterpret_cast<int32_t *>(smem + C::kOffMisc);
     // misc: 0 tmem base, 2 abort
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + 2);
@@ -566,6 +574,13 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             mbar_init(&unit_empty[s], kUnitConsumers);
         }
         mbar_init(mma_idle, 1);
+        if (kSolo) {
+            for (int s = 0; s < 3; ++s) {
+                mbar_init(&k_full[s], 1);
+                mbar_init(&k_empty[s], 1);
+            }
+            mbar_init(pv_done, 1);
+        }
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -578,7 +593,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
     // what the producer issued, for the drain after an abort
-    int issued_q = 0, issued_kv = 0;
+    int issued_q = 0, issued_kv = 0, issued_k = 0;
 
     if (warp == kSchedWarp) {
         // ------------------------------------------------------------ scheduler
@@ -903,46 +918,13 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 }
                 ++issued_q;
                 const int kvh = ui->h0 / p.G;
-                for (int i = 0; i < n_list; ++i, ++g) {
-                    const int st = g & 1;
-                    const int e = lst[i];
+                // The key tile's column masks (built once per key tile by the summary
+                // kernel; 8 bytes per lane), where a query tile is cut or the Nexus
+                // mass needs the Nexus bits, into the metadata of ring stage st; the
+                // keys' roles / segments / S_aug positions only where the masks fall
+                // back to the per-key rule.
+                auto stage_meta = [&](int st, int e, bool need_m0, bool need_m1) {
                     const int kt = e >> 6;
-                    // a retained-first tile made of 128 consecutive input rows is
-                    // copied from K and V themselves (the load overlaps the wait)
-                    const int dsrc = p.key_direct != nullptr
-                                         ? p.key_direct[(int64_t)b * p.max_k_tiles + kt]
-                                         : -1;
-                    if (g >= 2 && !mbar_wait(&kv_empty[st], ((g >> 1) - 1) & 1, p.status, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    // query tiles visiting the key tile that read its metadata: cut
-                    // by the mask, or (Nexus mass) some of its keys are Nexus keys
-                    const bool mass_tile = kMass && ((e >> 4) & 3) == 2;
-                    const bool need_m0 = (udense || (e & 4)) && ((e & 1) || mass_tile);
-                    const bool need_m1 = nq == 2 && (udense || (e & 8)) && ((e & 2) || mass_tile);
-                    // K/V copies first; the key metadata is built while they are in
-                    // flight and has a barrier of its own, so the S product of a cut
-                    // tile waits for the copy alone
-                    if (lane == 0) {
-                        mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
-                        const bool direct = dsrc >= 0;
-                        const int row = direct ? dsrc : kkstart + kt * kBN;
-                        const CUtensorMap *mk = direct ? &tmK0 : &tmK;
-                        const CUtensorMap *mv = direct ? &tmV0 : &tmV;
-#pragma unroll
-                        for (int hh = 0; hh < C::kHalves; ++hh) {
-                            tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), mk, &kv_full[st],
-                                        hh * 64, kvh, row, layer);
-                            tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), mv, &kv_full[st],
-                                        hh * 64, kvh, row, layer);
-                        }
-                    }
-                    issued_kv = g + 1;
-                    // The tile's column masks (built once per key tile by the summary
-                    // kernel; 8 bytes per lane) where a query tile is cut or the Nexus
-                    // mass needs the Nexus bits; the keys' roles / segments / S_aug
-                    // positions only where the masks fall back to the per-key rule.
                     const bool cut_any = (e & 3) != 0;
                     if (need_m0 || need_m1) {
                         const uint2 mw = reinterpret_cast<const uint2 *>(
@@ -977,6 +959,102 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                             if (need_m0) mbar_arrive(&meta_full[2 * st]);
                             if (need_m1) mbar_arrive(&meta_full[2 * st + 1]);
                         }
+                    }
+                };
+                // a retained-first tile made of 128 consecutive input rows is copied
+                // from K and V themselves (the load overlaps the wait that follows)
+                auto src_of = [&](int kt) {
+                    return p.key_direct != nullptr
+                               ? p.key_direct[(int64_t)b * p.max_k_tiles + kt]
+                               : -1;
+                };
+                if constexpr (kSolo) {
+                    // One query tile: K of key tile i + 1 is copied before V of tile
+                    // i, into a ring of three stages (Ks, Ks + one stage, and the
+                    // second Q tile's buffer), V into a ring of two; key tile i's
+                    // metadata goes with its V stage.
+                    int gk = g;
+                    auto issue_k = [&](int i) -> bool {
+                        const int kt = lst[i] >> 6;
+                        const int dsrc = src_of(kt);
+                        const int ks = gk % 3;
+                        if (gk >= 3 &&
+                            !mbar_wait(&k_empty[ks], ((gk / 3) - 1) & 1, p.status, abort_flag))
+                            return false;
+                        if (lane == 0) {
+                            mbar_arrive_expect_tx(&k_full[ks], C::kKVBytes);
+                            uint8_t *dst = ks < 2 ? Ks + ks * C::kKVBytes : Qs + C::kQBytes;
+#pragma unroll
+                            for (int hh = 0; hh < C::kHalves; ++hh)
+                                tma_load_4d(dst + hh * (kBN * 128), dsrc >= 0 ? &tmK0 : &tmK,
+                                            &k_full[ks], hh * 64, kvh,
+                                            dsrc >= 0 ? dsrc : kkstart + kt * kBN, layer);
+                        }
+                        issued_k = ++gk;
+                        return true;
+                    };
+                    if (!issue_k(0)) ok = false;
+                    for (int i = 0; ok && i < n_list; ++i, ++g) {
+                        if (i + 1 < n_list && !issue_k(i + 1)) {
+                            ok = false;
+                            break;
+                        }
+                        const int st = g & 1;
+                        const int e = lst[i];
+                        const int kt = e >> 6;
+                        const int dsrc = src_of(kt);
+                        if (g >= 2 &&
+                            !mbar_wait(&kv_empty[st], ((g >> 1) - 1) & 1, p.status, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        if (lane == 0) {
+                            mbar_arrive_expect_tx(&kv_full[st], C::kKVBytes);
+#pragma unroll
+                            for (int hh = 0; hh < C::kHalves; ++hh)
+                                tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128),
+                                            dsrc >= 0 ? &tmV0 : &tmV, &kv_full[st], hh * 64, kvh,
+                                            dsrc >= 0 ? dsrc : kkstart + kt * kBN, layer);
+                        }
+                        issued_kv = g + 1;
+                        stage_meta(st, e, (e & 1) || (kMass && ((e >> 4) & 3) == 2), false);
+                    }
+                } else {
+                    for (int i = 0; i < n_list; ++i, ++g) {
+                        const int st = g & 1;
+                        const int e = lst[i];
+                        const int kt = e >> 6;
+                        const int dsrc = src_of(kt);
+                        if (g >= 2 &&
+                            !mbar_wait(&kv_empty[st], ((g >> 1) - 1) & 1, p.status, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        // query tiles visiting the key tile that read its metadata: cut
+                        // by the mask, or (Nexus mass) some of its keys are Nexus keys
+                        const bool mass_tile = kMass && ((e >> 4) & 3) == 2;
+                        const bool need_m0 = (udense || (e & 4)) && ((e & 1) || mass_tile);
+                        const bool need_m1 =
+                            nq == 2 && (udense || (e & 8)) && ((e & 2) || mass_tile);
+                        // K/V copies first; the key metadata is built while they are in
+                        // flight and has a barrier of its own, so the S product of a cut
+                        // tile waits for the copy alone
+                        if (lane == 0) {
+                            mbar_arrive_expect_tx(&kv_full[st], 2 * C::kKVBytes);
+                            const bool direct = dsrc >= 0;
+                            const int row = direct ? dsrc : kkstart + kt * kBN;
+                            const CUtensorMap *mk = direct ? &tmK0 : &tmK;
+                            const CUtensorMap *mv = direct ? &tmV0 : &tmV;
+#pragma unroll
+                            for (int hh = 0; hh < C::kHalves; ++hh) {
+                                tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), mk,
+                                            &kv_full[st], hh * 64, kvh, row, layer);
+                                tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), mv,
+                                            &kv_full[st], hh * 64, kvh, row, layer);
+                            }
+                        }
+                        issued_kv = g + 1;
+                        stage_meta(st, e, need_m0, need_m1);
                     }
                 }
             }
@@ -1112,7 +1190,69 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         return true;
                     };
                     const bool dense = ui->flags & 2;
-                    if (ok) {
+                    if constexpr (kSolo) {
+                        // One query tile (kSolo): key tile j's S/P sits in TMEM block j & 1,
+                        // its K in K stage (g + j) % 3, its V in ring stage (g + j) & 1.
+                        // S of tile j + 2 goes out right after P.V of tile j (in order on
+                        // the tensor pipe, so it never overwrites a P still being read),
+                        // while the softmax works on tile j + 1.
+                        auto run_solo = [&]() -> bool {
+                            auto issue_s_solo = [&](int j) -> bool {
+                                const int t = g + j, ks = t % 3, sb = j & 1;
+                                if (!mbar_wait(&k_full[ks], (t / 3) & 1, p.status, abort_flag))
+                                    return false;
+                                tc_fence_after();
+                                const uint32_t kst = ks < 2 ? k_of(ks) : q_lo + (C::kQBytes >> 4);
+#pragma unroll
+                                for (int kk = 0; kk < D / 16; ++kk) {
+                                    const uint32_t off = ((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4;
+                                    tc_mma_ss(tmem + sb * kBN, desc_join(q_lo + off, dhi),
+                                              desc_join(kst + off, dhi), idS, kk > 0 ? 1u : 0u);
+                                }
+                                tc_commit(&s_full[sb]);
+                                tc_commit(&k_empty[ks]);
+                                return true;
+                            };
+                            if (!issue_s_solo(0)) return false;
+                            if (n_list > 1 && !issue_s_solo(1)) return false;
+                            if (n_list <= 2) tc_commit(q_empty);
+                            for (int j = 0; j < n_list; ++j) {
+                                const int sb = j & 1, ST = (g + j) & 1;
+                                // (the two P phase counters selected, not indexed: registers)
+                                const uint32_t par = (sb ? pw[1] : pw[0]) & 1;
+                                if (!mbar_wait(&p_full[sb], par, p.status, abort_flag))
+                                    return false;
+                                if (sb) ++pw[1]; else ++pw[0];
+                                tc_fence_after();
+                                if (j == 0 && uo[0] > 0) {
+                                    // O still holds the previous unit until its epilogue
+                                    // has read it
+                                    if (!mbar_wait(&o_free[0], (uo[0] - 1) & 1, p.status, abort_flag))
+                                        return false;
+                                    tc_fence_after();
+                                }
+                                if (!mbar_wait(&kv_full[ST], ((g + j) >> 1) & 1, p.status, abort_flag))
+                                    return false;
+                                tc_fence_after();
+                                const uint32_t vst = v_of(ST);
+#pragma unroll
+                                for (int kk = 0; kk < kBN / 16; ++kk)
+                                    tc_mma_ts(tmem + 256, tmem + sb * kBN + kk * 8,
+                                              desc_join(vst + ((kk * (16 * 128)) >> 4), dhi), idPV,
+                                              (j > 0 || kk > 0) ? 1u : 0u);
+                                tc_commit(pv_done);
+                                if (j == n_list - 1) tc_commit(&o_done[0]);
+                                tc_commit(&kv_empty[ST]);
+                                if (j + 2 < n_list) {
+                                    if (!issue_s_solo(j + 2)) return false;
+                                    // every S product of the unit is issued: Q may be replaced
+                                    if (j + 3 == n_list) tc_commit(q_empty);
+                                }
+                            }
+                            return true;
+                        };
+                        if (ok) ok = run_solo();
+                    } else if (ok) {
                         if (nq == 2)
                             ok = dense ? run(std::integral_constant<int, 2>{}, std::true_type{})
                                        : run(std::integral_constant<int, 2>{}, std::false_type{});
@@ -1142,10 +1282,12 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // Parities of the phases this warpgroup waits next, one bit each (all it
         // needs of its counters; one register across the key-tile loop):
         //   bit 0 / 1  metadata barrier of ring stage 0 / 1,
-        //   bit 2      S barrier,
+        //   bit 2      S barrier (kSolo: of S/P block 0),
         //   bit 3      O barrier (o_done),
-        //   bit 4      ring stage of the unit's first key tile.
+        //   bit 4      ring stage of the unit's first key tile,
+        //   bit 5      kSolo: S barrier of S/P block 1.
         uint32_t ph = 0;
+        int npv = 0;  // kSolo: P.V products this warpgroup has handed P to so far
         bool ok = true;
         for (int k = 0; ok; ++k) {
             const int slot = k & 1;
@@ -1211,16 +1353,21 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     uint32_t mbits[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
                     if (cut) tile_mask_bits(tmasks + st, meta_role + st * kBN, meta_seg + st * kBN,
                                             meta_pos + st * kBN, pos, rp, sp, p.nexus_mode, mbits);
-                    if (!mbar_wait(&s_full[qi], (ph >> 2) & 1, p.status, abort_flag)) {
+                    // kSolo: key tile j's S/P block and barriers are those of tile j & 1
+                    // (parity bit 5 for block 1)
+                    const int sb = kSolo ? (j & 1) : qi;
+                    const uint32_t sbit = (kSolo && sb) ? 32u : 4u;
+                    const uint32_t tSj = kSolo ? tS + (uint32_t)(sb * kBN) : tS;
+                    if (!mbar_wait(&s_full[sb], (ph & sbit) ? 1u : 0u, p.status, abort_flag)) {
                         ok = false;
                         break;
                     }
-                    ph ^= 4u;
+                    ph ^= sbit;
                     tc_fence_after();
                     // S row into registers: four 32-column loads, one wait
                     uint32_t sr[4][32];
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+                    for (int c = 0; c < 4; ++c) tmem_ld32(tSj + c * 32, sr[c]);
                     tmem_ld_wait();
 #pragma unroll
                     for (int c = 0; c < 4; ++c) reg_fence32(sr[c]);
@@ -1296,7 +1443,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                             if ((zchunk >> c) & 1) {
 #pragma unroll
                                 for (int x = 0; x < 16; ++x) pk[x] = 0u;
-                                tmem_st16(tS + c * 16, pk);
+                                tmem_st16(tSj + c * 16, pk);
                                 continue;
                             }
 #pragma unroll
@@ -1317,7 +1464,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                     add_bf16x2_to_f32_if(lsn[0], lsn[1], pr, nxb[c] & (1u << x),
                                                          nxb[c] & (2u << x));
                             }
-                            tmem_st16(tS + c * 16, pk);
+                            tmem_st16(tSj + c * 16, pk);
                         }
                     };
                     if (kMass && nexus_keys == 2)
@@ -1331,6 +1478,16 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // O rescale (the previous P.V of this tile is complete: this S
                     // was issued after it, and S is done)
                     if (__any_sync(0xffffffffu, alpha != 1.f)) {
+                        if constexpr (kSolo) {
+                            // the last P.V may still be accumulating into O: it is P.V
+                            // number npv, and the one before it is done (this S was
+                            // issued after it), so its phase is the one to wait for
+                            if (!mbar_wait(pv_done, (npv - 1) & 1, p.status, abort_flag)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                        }
 #pragma unroll
                         for (int c = 0; c < D / 32; ++c) {
                             uint32_t o[32];
@@ -1359,7 +1516,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         fence_proxy_async_smem();
                     }
                     tc_fence_before();
-                    mbar_arrive(&p_full[qi]);
+                    mbar_arrive(&p_full[sb]);
+                    if (kSolo) ++npv;
                     m_used = m_new;
                 }
                 if (!ok) break;
@@ -1433,6 +1591,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         if (issued_q > 0) mbar_drain(q_full, (issued_q - 1) & 1);
         for (int u = max(0, issued_kv - 2); u < issued_kv; ++u)
             mbar_drain(&kv_full[u & 1], (u >> 1) & 1);
+        if (kSolo)
+            for (int u = max(0, issued_k - 3); u < issued_k; ++u)
+                mbar_drain(&k_full[u % 3], (u / 3) & 1);
     }
     __syncthreads();
     if (warp == 1) tmem_dealloc(tmem, 512);
@@ -1776,19 +1937,23 @@ kv_permute_kernel(const uint8_t *__restrict__ K, const uint8_t *__restrict__ V,
 template <int D>
 cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
                            const CUtensorMap &tk0, const CUtensorMap &tv0, const CUtensorMap &tq32,
-                           const PfParams &p, int grid, cudaStream_t s) {
+                           const PfParams &p, bool solo, int grid, cudaStream_t s) {
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
     const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
     auto kern = p.qchunks != nullptr
-                    ? (out == 0   ? prefill_kernel<D, 0, true>
-                       : out == 1 ? prefill_kernel<D, 1, true>
-                       : out == 2 ? prefill_kernel<D, 2, true>
-                                  : prefill_kernel<D, 3, true>)
-                    : (out == 0   ? prefill_kernel<D, 0, false>
-                       : out == 1 ? prefill_kernel<D, 1, false>
-                       : out == 2 ? prefill_kernel<D, 2, false>
-                                  : prefill_kernel<D, 3, false>);
+                    ? (out == 0   ? prefill_kernel<D, 0, true, false>
+                       : out == 1 ? prefill_kernel<D, 1, true, false>
+                       : out == 2 ? prefill_kernel<D, 2, true, false>
+                                  : prefill_kernel<D, 3, true, false>)
+                : solo ? (out == 0   ? prefill_kernel<D, 0, false, true>
+                          : out == 1 ? prefill_kernel<D, 1, false, true>
+                          : out == 2 ? prefill_kernel<D, 2, false, true>
+                                     : prefill_kernel<D, 3, false, true>)
+                       : (out == 0   ? prefill_kernel<D, 0, false, false>
+                          : out == 1 ? prefill_kernel<D, 1, false, false>
+                          : out == 2 ? prefill_kernel<D, 2, false, false>
+                                     : prefill_kernel<D, 3, false, false>);
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -2042,7 +2207,11 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
         reorder ? (int64_t)ws.rows : (int64_t)a->total_k_rows, a->status, p.counter);
     // one persistent block per SM (fewer when there are fewer units)
     const int grid = (int)std::min<long long>(device_sm_count(), n_units);
-    cudaError_t e = (D == 128) ? launch_prefill<128>(tq, tk, tv, tk0, tv0, tq32, p, grid, stream)
-                               : launch_prefill<64>(tq, tk, tv, tk0, tv0, tq32, p, grid, stream);
+    // every unit holds one query tile: packed heads with every query block within
+    // one tile (R rows), so the second tile's TMEM block and Q buffer are free
+    const bool solo = !qchunked && pack_log2 > 0 && a->max_q_len <= R;
+    cudaError_t e = (D == 128)
+                        ? launch_prefill<128>(tq, tk, tv, tk0, tv0, tq32, p, solo, grid, stream)
+                        : launch_prefill<64>(tq, tk, tv, tk0, tv0, tq32, p, solo, grid, stream);
     return e == cudaSuccess ? SONIC_OK : SONIC_ERR_CUDA;
 }
