@@ -126,7 +126,9 @@ struct UnitInfo {
     int32_t pbase;    // S_aug position of query row 0 of tile 0
     int32_t last[2];  // list index of the last key tile each query tile visits (-1: none)
     int32_t qc[2][4];  // chunk words of the query tiles (query chunk table)
-    int32_t pad[8];
+    int32_t pairu;     // the two query tiles are one block of heads h0 and h0 + 1
+    int32_t qstepu;    // query rows between tile 0 and tile 1 (0 when paired)
+    int32_t pad[6];
 };
 static_assert(sizeof(UnitInfo) == 128, "unit record: 128 bytes");
 
@@ -504,7 +506,9 @@ __device__ __forceinline__ void tile_mask_bits(const TileMasks *tmk, const uint8
 // S/P then alternates between the two tiles' TMEM blocks, so the S product of
 // key tile j + 1 runs while the softmax works on tile j, and K takes a ring of
 // three stages (the unused second Q tile's buffer is the third), V of two.
-template <int D, int kOut, bool kQC, bool kSolo>
+// kPair: paired units (an even number of query heads per KV head, heads not
+// packed): a unit is one 128-row query block of heads h0 and h0 + 1.
+template <int D, int kOut, bool kQC, bool kSolo, bool kPair>
 __global__ void __maxnreg__(168)
 prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmK0,
@@ -555,7 +559,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     // the heads of short query blocks so the tile rows are not left empty.
     const int pl2 = p.pack_log2, R = kBM >> pl2;
     // query rows of a unit, and the row offset of its second query tile
-    const int urows = p.pair ? R : 2 * R, qstep = p.pair ? 0 : R;
+    const int urows = kPair ? R : 2 * R, qstep = kPair ? 0 : R;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     if (tid == 0) {
@@ -600,6 +604,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int k = 0;; ++k) {
             const int slot = k & 1;
             int end = 0, layer = 0, b = 0, hg = 0, qt = 0, cw = 0;
+            bool lpair = false;  // a last query block shared by two heads (below)
             int kstart = 0, klen = 0, qstart = 0, qlen = 0, kkstart = 0, kklen = 0;
             for (;;) {
                 int u = p.n_units;
@@ -634,13 +639,25 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     // tiles are the same rows)
                     cw = 0;
                     if (lane < 8) {
-                        const int vt = p.pair ? qt : 2 * qt + (lane >> 2);
+                        const int vt = kPair ? qt : 2 * qt + (lane >> 2);
                         if ((vt + 1) * 4 <= p.qchunks_per_seq)
                             cw = p.qchunks[(int64_t)b * p.qchunks_per_seq + vt * 4 + (lane & 3)];
                     }
                     if (!__any_sync(0xffffffffu, (cw >> 24) != 0)) continue;  // no query rows
                 } else {
                     if (qt * urows >= qlen) continue;  // no query rows in this block
+                    // Unpaired units (an odd head ratio) are 256-row blocks of one head;
+                    // the last block of a sequence with an odd number of 128-row blocks
+                    // has one tile, and one tile alone leaves the tensor pipe idle
+                    // during its softmax.  Heads 2i and 2i + 1 of a KV group share that
+                    // block instead (same rows, same keys: the paired form); the last
+                    // head of an odd group keeps a unit of its own.
+                    lpair = false;
+                    if (!kSolo && !kPair && pl2 == 0 && p.G > 1 && qt * urows + R >= qlen) {
+                        const int i = hg % p.G;
+                        if (i & 1) continue;  // in the unit of head hg - 1
+                        lpair = i + 1 < p.G;
+                    }
                 }
                 kklen = p.key_len[b];
                 if (qlen > klen || klen > p.max_k_len || kklen > p.max_k_tiles * kBN) {
@@ -720,14 +737,14 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     qp0[qi] = pmin;
                     qp1[qi] = pmax;
                 }
-                tile1 = p.pair || qp0[1] <= qp1[1];
+                tile1 = kPair || qp0[1] <= qp1[1];
             } else {
-                tile1 = p.pair || qt * 2 * R + R < qlen;
+                tile1 = kPair || (!kPair && lpair) || qt * 2 * R + R < qlen;
 #pragma unroll
                 for (int qi = 0; qi < 2; ++qi) {
                     int f = 0, s0 = INT_MAX, s1 = INT_MIN, n0 = INT_MAX, n1 = INT_MIN;
                     for (int r = lane; r < R; r += 32) {
-                        const int pos = pbase + qi * qstep + r;
+                        const int pos = pbase + qi * (lpair ? 0 : qstep) + r;
                         if (pos <= klen - 1) {
                             const int ro = p.role[kstart + pos];
                             const int s = p.seg[kstart + pos];
@@ -753,7 +770,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     qs1[qi] = s1;
                     qn0[qi] = n0;
                     qn1[qi] = n1;
-                    qp0[qi] = pbase + qi * qstep;
+                    qp0[qi] = pbase + qi * (lpair ? 0 : qstep);
                     qp1[qi] = min(qp0[qi] + R - 1, klen - 1);
                 }
             }
@@ -816,7 +833,11 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 ui->flags = dense ? 2 : 0;
                 ui->layer = layer;
                 ui->b = b;
-                ui->h0 = p.pair ? 2 * hg : hg << pl2;
+                ui->h0 = kPair ? 2 * hg : hg << pl2;
+                if (!kPair) {
+                    ui->pairu = lpair;
+                    ui->qstepu = lpair ? 0 : qstep;
+                }
                 ui->qt = qt;
                 ui->nq = tile1 ? 2 : 1;
                 ui->n_list = n_list;
@@ -891,7 +912,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                             for (int hh = 0; hh < C::kHalves; ++hh)
                                 tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
-                                            hh * 64, ui->h0 + qi * p.pair,
+                                            hh * 64, ui->h0 + qi * (kPair ? 1 : 0),
                                             q0 + (ui->qc[qi][0] & 0xffffff), layer);
                             continue;
                         }
@@ -902,7 +923,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                             for (int hh = 0; hh < C::kHalves; ++hh)
                                 tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128) + c * (32 * 128),
-                                            &tmQ32, q_full, hh * 64, ui->h0 + qi * p.pair,
+                                            &tmQ32, q_full, hh * 64, ui->h0 + qi * (kPair ? 1 : 0),
                                             q0 + (w & 0xffffff), layer);
                         }
                     }
@@ -912,8 +933,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
                         for (int hh = 0; hh < C::kHalves; ++hh)
                             tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
-                                        hh * 64, ui->h0 + qi * p.pair,
-                                        ui->qstart + ui->qt * urows + qi * qstep,
+                                        hh * 64, ui->h0 + qi * (kPair ? 1 : ui->pairu),
+                                        ui->qstart + ui->qt * urows + qi * (kPair ? 0 : ui->qstepu),
                                         layer);
                 }
                 ++issued_q;
@@ -1311,7 +1332,7 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     const int w = ui->qc[qi][r >> 5];
                     pos = lane < (w >> 24) ? (w & 0xffffff) + lane : -1;
                 } else {
-                    pos = ui->pbase + qi * qstep + qr;
+                    pos = ui->pbase + qi * (kPair ? 0 : ui->qstepu) + qr;
                 }
                 int rp = SONIC_ROLE_SYS, sp = 0;
                 if (kQC ? pos >= 0 : pos <= ui->klen - 1) {
@@ -1521,9 +1542,11 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     m_used = m_new;
                 }
                 if (!ok) break;
-                const int layer = ui->layer, h = ui->h0 + qi * p.pair + hoff;
+                const int layer = ui->layer, h = ui->h0 + qi * (kPair ? 1 : ui->pairu) + hoff;
                 // query row within the sequence
-                const int qidx = kQC ? pos - (ui->klen - ui->qlen) : ui->qt * urows + qi * qstep + qr;
+                const int qidx =
+                    kQC ? pos - (ui->klen - ui->qlen)
+                        : ui->qt * urows + qi * (kPair ? 0 : ui->qstepu) + qr;
                 const bool row_ok = kQC ? pos >= 0 : pos <= ui->klen - 1 && qidx < ui->qlen;
                 const int64_t qrow = (int64_t)ui->qstart + qidx;
                 uint16_t *orow = p.O + layer * p.o_ls + (qrow * p.Hq + h) * D;
@@ -1941,19 +1964,25 @@ cudaError_t launch_prefill(const CUtensorMap &tq, const CUtensorMap &tk, const C
     constexpr size_t smem = PfCfg<D>::kSmem;
     static_assert(smem <= 232448, "prefill shared memory");
     const int out = (p.lse != nullptr ? 1 : 0) | (p.nexus_mass != nullptr ? 2 : 0);
-    auto kern = p.qchunks != nullptr
-                    ? (out == 0   ? prefill_kernel<D, 0, true, false>
-                       : out == 1 ? prefill_kernel<D, 1, true, false>
-                       : out == 2 ? prefill_kernel<D, 2, true, false>
-                                  : prefill_kernel<D, 3, true, false>)
-                : solo ? (out == 0   ? prefill_kernel<D, 0, false, true>
-                          : out == 1 ? prefill_kernel<D, 1, false, true>
-                          : out == 2 ? prefill_kernel<D, 2, false, true>
-                                     : prefill_kernel<D, 3, false, true>)
-                       : (out == 0   ? prefill_kernel<D, 0, false, false>
-                          : out == 1 ? prefill_kernel<D, 1, false, false>
-                          : out == 2 ? prefill_kernel<D, 2, false, false>
-                                     : prefill_kernel<D, 3, false, false>);
+    // instances: chunked query order (paired or not), single-tile units, or the
+    // given order (paired or not)
+    using K = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, CUtensorMap, CUtensorMap,
+                       CUtensorMap, PfParams);
+    auto pick = [&](auto qc, auto solo_t, auto pair_t) -> K {
+        constexpr bool a = decltype(qc)::value, b = decltype(solo_t)::value,
+                       c = decltype(pair_t)::value;
+        return out == 0   ? (K)prefill_kernel<D, 0, a, b, c>
+               : out == 1 ? (K)prefill_kernel<D, 1, a, b, c>
+               : out == 2 ? (K)prefill_kernel<D, 2, a, b, c>
+                          : (K)prefill_kernel<D, 3, a, b, c>;
+    };
+    using T = std::true_type;
+    using F = std::false_type;
+    const bool paired = p.pair != 0;
+    K kern = p.qchunks != nullptr ? (paired ? pick(T{}, F{}, T{}) : pick(T{}, F{}, F{}))
+             : solo               ? pick(F{}, T{}, F{})
+             : paired             ? pick(F{}, F{}, T{})
+                                  : pick(F{}, F{}, F{});
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
