@@ -768,21 +768,22 @@ def extra_context(n_layers: int = 8):
                         "28/4 heads, D=128", "results": res}
 
 
-def extra_nexus_gen():
+def extra_nexus_gen(n_layers: int = 0):
     """Nexus generation with incremental compaction (Sec. 3.1, Table 3's
     "Nexus Gen." step) at the masked-prefill shapes: batch 8, 32 layers, 32/8
     heads, D = 128, 512 system tokens, 16 segments of 256 body + 32 Nexus.
     Segment i: the 32 Nexus rows attend over [retained | body_i | Nexus_i]
     (one prefill launch for the batch and all layers), then compaction drops
     body_i.  Inputs of every segment step are staged beforehand; the timed
-    region is the 16 prefill and 16 compaction launches."""
+    region is the 16 prefill and 16 compaction launches.  n_layers > 0 runs
+    that many layers instead of 32 (small profiler captures)."""
     import torch
     from paper_2601_21927_gb300 import inputs, sonic
     dev = torch.device("cuda", 0)
     t = lambda a: torch.as_tensor(np.asarray(a)).to(dev)
     batch, hd = inputs.masked_prefill()
     d = batch.dialogues[0]
-    B, NL = batch.B, hd.n_layers
+    B, NL = batch.B, (n_layers if n_layers > 0 else hd.n_layers)
     sysl, segs = d.sys_len, d.segments
     steps = []
     flops = comp_bytes = pf_bytes = 0.0
@@ -833,7 +834,7 @@ def extra_nexus_gen():
     # 32 query rows of 4 heads per K/V row: the prefill is bound by HBM, not by
     # the tensor cores (flops per byte below the ridge point peak_bf16 / peak_hbm)
     intensity = flops / pf_bytes
-    return {"workload": "Nexus generation: batch 8, 32 layers, 32/8 heads, D=128, "
+    return {"workload": f"Nexus generation: batch 8, {NL} layers, 32/8 heads, D=128, "
                         "16 segments of 256 body + 32 Nexus after 512 system tokens",
             "results": {"prefill_ms_all_segments": round(p_ms, 3),
                         "prefill_tflops": round(flops / p_ms / 1e9, 1),
@@ -1110,10 +1111,14 @@ def config_workloads():
             Qx[:nl], K[:nl], V[:nl], s_, r_, Ox[:nl], k_start=ks, k_len=kl, q_start=q_start,
             q_len=q_len, max_q_len=max_q, max_k_len=L, key_order=order, workspace=ws)
         ws = call()
-        ms = _ev_time(lambda: call(ws), reps=10 if nl == 1 else 4, warm=3)
+        sampler = ClockSampler(0)
+        sampler.start()
+        ms = _ev_time(lambda: call(ws), reps=10, warm=3)
+        clk = sampler.stop()
         tf = fl * nl / ms / 1e9
         res[name] = {"layers": nl, "ms": round(ms, 4), "value": round(tf, 1), "unit": "TFLOP/s",
-                     "frac": round(tf / pk["bf16"], 4)}
+                     "frac": round(tf / pk["bf16"], 4),
+                     "frac_of_sustained": round(tf / pk["bf16_sus"], 4), "clocks": clk}
         del ws
 
     for order, oname in ((1, "retained_first"), (0, "as_given")):
@@ -1136,8 +1141,10 @@ def config_workloads():
                            "(its key and query order and K/V copies included)",
                "flops": flops1 * NL, "ms": head["ms"], "value": head["value"], "unit": "TFLOP/s",
                "roofline": {"bound": "tensor", "peak": pk["bf16"], "unit": "TFLOP/s",
-                            "frac": head["frac"], "peak_source": pk["source"] + " bf16 burst"},
-               "variants": res}
+                            "frac": head["frac"], "peak_source": pk["source"] + " bf16 burst",
+                            "peak_sustained": pk["bf16_sus"],
+                            "frac_of_sustained": head["frac_of_sustained"]},
+               "clocks": head["clocks"], "variants": res}
     # compaction of all 32 layers' K/V (raw 5.91 GB in, 3.22 GB moved)
     K = inputs.randn((hd.n_layers, batch.total, hd.hkv, hd.d), seed=5, device=dev)
     V = inputs.randn((hd.n_layers, batch.total, hd.hkv, hd.d), seed=6, device=dev)
@@ -1195,7 +1202,8 @@ def main():
 
     if args.extra:
         if rank == 0:
-            out = EXTRAS[args.extra]()
+            kw = {"n_layers": args.layers} if args.layers and args.extra == "nexus_gen" else {}
+            out = EXTRAS[args.extra](**kw)
             out["extra"] = args.extra
             print(json.dumps(out))
         return
