@@ -38,6 +38,21 @@ bool make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4
     return r == CUDA_SUCCESS;
 }
 
+bool make_tmap_bf16_5d(CUtensorMap *map, const void *base, const uint64_t dims[5],
+                       const uint64_t strides[4], const uint32_t box[5]) {
+    auto fn = encode_fn();
+    if (fn == nullptr) return false;
+    cuuint64_t gdim[5] = {dims[0], dims[1], dims[2], dims[3], dims[4]};
+    cuuint64_t gstride[4] = {strides[0], strides[1], strides[2], strides[3]};
+    cuuint32_t bdim[5] = {box[0], box[1], box[2], box[3], box[4]};
+    cuuint32_t estride[5] = {1, 1, 1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(base), gdim,
+                    gstride, bdim, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 int device_sm_count() {
     static int cache[64] = {0};
     int dev = 0;

@@ -909,11 +909,11 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                     for (int qi = 0; qi < 2; ++qi) {
                         if (qi >= nq) break;
                         if (whole[qi]) {
-#pragma unroll
-                            for (int hh = 0; hh < C::kHalves; ++hh)
-                                tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
-                                            hh * 64, ui->h0 + qi * (kPair ? 1 : 0),
-                                            q0 + (ui->qc[qi][0] & 0xffffff), layer);
+                            // both 64-column halves in one copy (5-D map: the half is a
+                            // dimension of its own, outside the rows)
+                            tma_load_5d(Qs + qi * C::kQBytes, &tmQ, q_full, 0,
+                                        ui->h0 + qi * (kPair ? 1 : 0),
+                                        q0 + (ui->qc[qi][0] & 0xffffff), 0, layer);
                             continue;
                         }
 #pragma unroll
@@ -930,12 +930,10 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                 } else if (!kQC && lane == 0) {
                     mbar_arrive_expect_tx(q_full, nq * C::kQBytes);
                     for (int qi = 0; qi < nq; ++qi)
-#pragma unroll
-                        for (int hh = 0; hh < C::kHalves; ++hh)
-                            tma_load_4d(Qs + qi * C::kQBytes + hh * (kBM * 128), &tmQ, q_full,
-                                        hh * 64, ui->h0 + qi * (kPair ? 1 : ui->pairu),
-                                        ui->qstart + ui->qt * urows + qi * (kPair ? 0 : ui->qstepu),
-                                        layer);
+                        tma_load_5d(Qs + qi * C::kQBytes, &tmQ, q_full, 0,
+                                    ui->h0 + qi * (kPair ? 1 : ui->pairu),
+                                    ui->qstart + ui->qt * urows + qi * (kPair ? 0 : ui->qstepu), 0,
+                                    layer);
                 }
                 ++issued_q;
                 const int kvh = ui->h0 / p.G;
@@ -1005,11 +1003,8 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         if (lane == 0) {
                             mbar_arrive_expect_tx(&k_full[ks], C::kKVBytes);
                             uint8_t *dst = ks < 2 ? Ks + ks * C::kKVBytes : Qs + C::kQBytes;
-#pragma unroll
-                            for (int hh = 0; hh < C::kHalves; ++hh)
-                                tma_load_4d(dst + hh * (kBN * 128), dsrc >= 0 ? &tmK0 : &tmK,
-                                            &k_full[ks], hh * 64, kvh,
-                                            dsrc >= 0 ? dsrc : kkstart + kt * kBN, layer);
+                            tma_load_5d(dst, dsrc >= 0 ? &tmK0 : &tmK, &k_full[ks], 0, kvh,
+                                        dsrc >= 0 ? dsrc : kkstart + kt * kBN, 0, layer);
                         }
                         issued_k = ++gk;
                         return true;
@@ -1031,11 +1026,9 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                         }
                         if (lane == 0) {
                             mbar_arrive_expect_tx(&kv_full[st], C::kKVBytes);
-#pragma unroll
-                            for (int hh = 0; hh < C::kHalves; ++hh)
-                                tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128),
-                                            dsrc >= 0 ? &tmV0 : &tmV, &kv_full[st], hh * 64, kvh,
-                                            dsrc >= 0 ? dsrc : kkstart + kt * kBN, layer);
+                            tma_load_5d(Vs + st * C::kKVBytes, dsrc >= 0 ? &tmV0 : &tmV,
+                                        &kv_full[st], 0, kvh, dsrc >= 0 ? dsrc : kkstart + kt * kBN,
+                                        0, layer);
                         }
                         issued_kv = g + 1;
                         stage_meta(st, e, (e & 1) || (kMass && ((e >> 4) & 3) == 2), false);
@@ -1066,13 +1059,10 @@ prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                             const int row = direct ? dsrc : kkstart + kt * kBN;
                             const CUtensorMap *mk = direct ? &tmK0 : &tmK;
                             const CUtensorMap *mv = direct ? &tmV0 : &tmV;
-#pragma unroll
-                            for (int hh = 0; hh < C::kHalves; ++hh) {
-                                tma_load_4d(Ks + st * C::kKVBytes + hh * (kBN * 128), mk,
-                                            &kv_full[st], hh * 64, kvh, row, layer);
-                                tma_load_4d(Vs + st * C::kKVBytes + hh * (kBN * 128), mv,
-                                            &kv_full[st], hh * 64, kvh, row, layer);
-                            }
+                            tma_load_5d(Ks + st * C::kKVBytes, mk, &kv_full[st], 0, kvh, row, 0,
+                                        layer);
+                            tma_load_5d(Vs + st * C::kKVBytes, mv, &kv_full[st], 0, kvh, row, 0,
+                                        layer);
                         }
                         issued_kv = g + 1;
                         stage_meta(st, e, need_m0, need_m1);
@@ -2128,21 +2118,28 @@ extern "C" sonic_status_t sonic_attn_prefill(const uint16_t *Q, const uint16_t *
     const void *Vt = reorder ? (const void *)(wsb + ws.vp) : (const void *)V;
     const uint64_t kt_rows = reorder ? (uint64_t)ws.rows : (uint64_t)a->total_k_rows;
     const uint64_t kt_layer = reorder ? (uint64_t)ws.rows * krow * 2 : k_layer;
-    const uint64_t kd[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, kt_rows,
-                            (uint64_t)a->n_layers};
-    const uint64_t ks[3] = {(uint64_t)D * 2, krow * 2, kt_layer};
-    const uint32_t box[4] = {64, 1, 128, 1};
-    const uint32_t qbox[4] = {64, 1u << pack_log2, (uint32_t)R, 1};  // R rows x P heads
+    // Whole Q, K and V tiles: 5-D maps (64 columns, head, row, 64-column half,
+    // layer), so one copy brings both halves of a head_dim-128 tile, each half a
+    // [row][128-byte] block as the 128-byte swizzle wants it.
+    const uint64_t nh = (uint64_t)D / 64;
+    const uint64_t qd5[5] = {64, (uint64_t)a->n_heads_q, (uint64_t)a->total_q_rows, nh,
+                             (uint64_t)a->n_layers};
+    const uint64_t qs5[4] = {(uint64_t)D * 2, qrow * 2, 128, q_layer};
+    const uint32_t qbox5[5] = {64, 1u << pack_log2, (uint32_t)R, (uint32_t)nh, 1};  // R rows x P heads
+    const uint64_t kd5[5] = {64, (uint64_t)a->n_heads_kv, kt_rows, nh, (uint64_t)a->n_layers};
+    const uint64_t ks5[4] = {(uint64_t)D * 2, krow * 2, 128, kt_layer};
+    const uint32_t box5[5] = {64, 1, 128, (uint32_t)nh, 1};
     CUtensorMap tq, tk, tv, tk0, tv0, tq32;
-    if (!make_tmap_bf16_4d(&tq, Q, qd, qs, qbox) || !make_tmap_bf16_4d(&tk, Kt, kd, ks, box) ||
-        !make_tmap_bf16_4d(&tv, Vt, kd, ks, box))
+    if (!make_tmap_bf16_5d(&tq, Q, qd5, qs5, qbox5) || !make_tmap_bf16_5d(&tk, Kt, kd5, ks5, box5) ||
+        !make_tmap_bf16_5d(&tv, Vt, kd5, ks5, box5))
         return SONIC_ERR_INVALID_ARGUMENT;
     // the inputs themselves, for the retained-first tiles read in place
-    const uint64_t kd0[4] = {(uint64_t)D, (uint64_t)a->n_heads_kv, (uint64_t)a->total_k_rows,
+    const uint64_t kd0[5] = {64, (uint64_t)a->n_heads_kv, (uint64_t)a->total_k_rows, nh,
                              (uint64_t)a->n_layers};
-    const uint64_t ks0[3] = {(uint64_t)D * 2, krow * 2, k_layer};
+    const uint64_t ks0[4] = {(uint64_t)D * 2, krow * 2, 128, k_layer};
     if (reorder) {
-        if (!make_tmap_bf16_4d(&tk0, K, kd0, ks0, box) || !make_tmap_bf16_4d(&tv0, V, kd0, ks0, box))
+        if (!make_tmap_bf16_5d(&tk0, K, kd0, ks0, box5) ||
+            !make_tmap_bf16_5d(&tv0, V, kd0, ks0, box5))
             return SONIC_ERR_INVALID_ARGUMENT;
     } else {
         tk0 = tk;

@@ -18,6 +18,10 @@ namespace sonic {
 bool make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4],
                        const uint64_t strides[3], const uint32_t box[4]);
 
+// The same with 5 dimensions (strides of dims 1..4).
+bool make_tmap_bf16_5d(CUtensorMap *map, const void *base, const uint64_t dims[5],
+                       const uint64_t strides[4], const uint32_t box[5]);
+
 // Number of SMs of the current device (cached per device).
 int device_sm_count();
 
