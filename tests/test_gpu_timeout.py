@@ -1,6 +1,7 @@
 """The bounded-wait failure path on the GPU.
 
-A test copy of the prefill and decode kernels is built with a wait limit of
+A test copy of the prefill and decode kernels (every prefill instance: paired,
+retained-first chunked, unpaired and single-tile units) is built with a wait limit of
 200 ns (SONIC_WAIT_LIMIT_NS) checked on every poll, far shorter than a TMA
 round trip, so waits run out while the work they wait for is still in flight.  The
 call must then report SONIC_ERR_DEVICE_TIMEOUT in the status word, and its
@@ -48,11 +49,26 @@ def _with(lib, fn):
         sonic._lib = saved
 
 
-def test_prefill_wait_timeout_then_normal_call(short_wait_lib):
+# Every kind of prefill kernel instance: paired units (head ratio 4, given
+# order), the retained-first query chunks, unpaired units with last query blocks
+# shared by two heads (head ratio 3), and single-tile units with packed heads
+# (32 query rows per sequence), whose K ring has three stages.
+PREFILL_CASES = {
+    "paired": dict(hq=8, hkv=2, order=sonic.KEYS_AS_GIVEN, short=False),
+    "retained_first": dict(hq=8, hkv=2, order=sonic.KEYS_RETAINED_FIRST, short=False),
+    "unpaired": dict(hq=6, hkv=2, order=sonic.KEYS_AS_GIVEN, short=False),
+    "single_tile": dict(hq=8, hkv=2, order=sonic.KEYS_AS_GIVEN, short=True),
+}
+
+
+@pytest.mark.parametrize("case", sorted(PREFILL_CASES))
+def test_prefill_wait_timeout_then_normal_call(short_wait_lib, case):
+    c = PREFILL_CASES[case]
     rng = np.random.default_rng(21)
     batch = inputs.Batch([inputs.random_dialogue(rng, max_segments=5, max_body=400,
                                                  max_nexus=40, max_curr=300) for _ in range(6)])
-    args = dict(hq=8, hkv=2, D=128, seed=3)
+    q_len = np.minimum(batch.k_len, 32).astype(np.int32) if c["short"] else None
+    args = dict(hq=c["hq"], hkv=c["hkv"], D=128, seed=3, key_order=c["order"], q_len=q_len)
     _with(short_wait_lib, lambda: H.run_prefill(batch, expect_status=TIMEOUT, **args))
     torch.cuda.synchronize()  # the context is still usable
     res = H.run_prefill(batch, **args)
