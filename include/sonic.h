@@ -91,25 +91,26 @@ typedef enum {
     SONIC_NEXUS_CAUSAL_SEGMENTS = 1
 } sonic_nexus_vis_t;
 
-/* Order in which sonic_attn_prefill walks a sequence's keys.
+/* Order in which sonic_attn_prefill walks a sequence's keys (and queries).
  * AS_GIVEN: the key rows as laid out (S_aug order).
  * RETAINED_FIRST: the library first lays each sequence's keys out in its
  * workspace (role, segment, position) as [system prompt, Nexus and
  * current-turn rows | history bodies], each part in S_aug order and the
  * bodies starting on a 128-row boundary; the mask still compares S_aug
- * positions.  A 128-key tile of that order made of 128 consecutive rows of
- * K and V (a stretch of one body, of the system prompt or of the current
- * turn) is read from K and V in place; the K and V rows of every other tile
- * are copied into the workspace, for every layer.  The query rows are walked
- * in the same order, by 32-row chunks of runs (one body, or consecutive rows
- * that are not body rows), so a query tile holds rows that see nearly the same
- * keys; Q and O stay where they are.  A sequence with more than 1024 such
- * runs, or whose runs padded to 32 rows exceed align128(q_len) + 1024 rows,
- * keeps the given query order.  Every query row then sees one prefix of the retained part plus
+ * positions.  Every query row then sees one prefix of the retained part plus
  * (for body and Nexus rows) the body of its own segment, so far fewer key
  * tiles are visited and cut by the mask when all rows of S_aug are queried.
- * Results equal AS_GIVEN up to floating-point summation order.  The copy
- * costs workspace: see sonic_prefill_workspace_size. */
+ * A 128-key tile of that order made of 128 consecutive rows of K and V (a
+ * stretch of one body, of the system prompt or of the current turn) is read
+ * from K and V in place; the K and V rows of every other tile are copied into
+ * the workspace, for every layer.  Unless query heads are packed (short query
+ * blocks), the query rows are walked in the same order too, by 32-row chunks
+ * of runs (one body, or consecutive rows that are not body rows), so a query
+ * tile holds rows that see nearly the same keys; Q and O stay where they are.
+ * A sequence with more than 1024 such runs, or whose runs padded to 32 rows
+ * exceed align128(q_len) + 1024 rows, keeps the given query order.  Results
+ * equal AS_GIVEN up to floating-point summation order.  The layout and the
+ * copies cost workspace: see sonic_prefill_workspace_size. */
 typedef enum {
     SONIC_KEYS_AS_GIVEN = 0,
     SONIC_KEYS_RETAINED_FIRST = 1
